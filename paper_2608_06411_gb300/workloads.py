@@ -1,0 +1,191 @@
+"""Seeded synthetic inputs shaped like the paper's LLaVA-NeXT / Qwen2.5-VL workloads.
+
+This module is the ONE place both the CUDA path and the CPU oracle take their inputs
+from.  It holds none of the method's arithmetic: it only draws random numbers and
+rounds them to bf16 storage.  Everything is numpy (PCG64), so the same seed gives
+the same bytes on x86 and Arm.
+
+Shapes follow the paper's workloads (section "Experiments", Tables 2 and 3):
+LLaVA-NeXT-7B feeds N = 2880 visual tokens (5 AnyRes crops of a 24x24 grid) of width
+D = 4096 to the language model and keeps K = 160 of them (5.56%); LLaVA-1.5 uses one
+24x24 grid (N = 576).  The benchmarks' images and questions are not available, so
+visual tokens are drawn as spatially clustered features (cluster centroid + noise),
+which gives the diversity term of Eq. 4 real redundancy to remove, and question
+tokens are standard normal.
+
+Visual features are returned as uint16 bf16 bit patterns [B, N, D]; question tokens
+as packed uint16 [sum(lens), D] plus the per-image lengths.
+"""
+from __future__ import annotations
+
+import dataclasses
+from concurrent.futures import ThreadPoolExecutor
+
+import numpy as np
+
+__all__ = [
+    "PredictorDims", "Workload", "WORKLOADS", "f32_to_bf16_bits", "bf16_bits_to_f32",
+    "make_weights", "make_image", "make_text", "make_batch", "k0_for",
+]
+
+
+def f32_to_bf16_bits(x: np.ndarray) -> np.ndarray:
+    """Round float32 values to bf16 (round to nearest, ties to even); return uint16 bits."""
+    x = np.ascontiguousarray(x, dtype=np.float32)
+    u = x.view(np.uint32).astype(np.uint64)
+    u = (u + 0x7FFF + ((u >> 16) & 1)) >> 16
+    return u.astype(np.uint16)
+
+
+def bf16_bits_to_f32(b: np.ndarray) -> np.ndarray:
+    """Exact widening of bf16 bit patterns to float32."""
+    b = np.ascontiguousarray(b, dtype=np.uint16)
+    return (b.astype(np.uint32) << 16).view(np.float32)
+
+
+@dataclasses.dataclass(frozen=True)
+class PredictorDims:
+    """Predictor widths.  The paper calls the predictor lightweight but gives no
+    widths; these are the reading used throughout (2-layer MLPs of width Dh, one
+    query/key head of width dp)."""
+    D: int = 4096
+    Dh: int = 1024
+    dp: int = 128
+
+
+@dataclasses.dataclass(frozen=True)
+class Workload:
+    name: str
+    config_id: int
+    B: int
+    crops: int          # AnyRes crops / tiles per image
+    grid: int           # tokens per crop side (24 for LLaVA, 27 for the Qwen-like tiles)
+    D: int
+    centroids: int      # centroids per crop
+    block_rows: int     # centroid grid: rows of blocks per crop
+    block_cols: int
+    noise: float
+    m_lo: int           # question length range (inclusive)
+    m_hi: int
+    K: int
+    near_dup_every: int = 0     # images with b % near_dup_every == 0 repeat crop 0
+    near_dup_noise: float = 0.05
+
+    @property
+    def N(self) -> int:
+        return self.crops * self.grid * self.grid
+
+
+WORKLOADS = {
+    # one 24x24 grid, 16 centroids on 6x6-token blocks, M = 32, keep 32
+    "c0": Workload("c0_single_n576", 0, 1, 1, 24, 4096, 16, 4, 4, 0.3, 32, 32, 32),
+    # LLaVA-NeXT shape: 5 crops x 24x24, 64 centroids per crop on 3x3 blocks, keep 160
+    "c1": Workload("c1_llava_next_n2880", 1, 1, 5, 24, 4096, 64, 8, 8, 0.3, 64, 64, 160),
+    # retention sweep reuses the c1 generator (K and the diversity weight vary)
+    "c2": Workload("c2_sweep_n2880", 2, 1, 5, 24, 4096, 64, 8, 8, 0.3, 64, 64, 160),
+    # batched serving: 64 images, ragged questions, 10% near-duplicate crops
+    "c3": Workload("c3_batch64_n2880_k160", 3, 64, 5, 24, 4096, 64, 8, 8, 0.3, 16, 256, 160,
+                   near_dup_every=10),
+    # high-token regime: 10 tiles x 27x27, D = 3584, 128 centroids per tile, keep 405
+    "c4": Workload("c4_batch16_n7290_k405", 4, 16, 10, 27, 3584, 128, 16, 8, 0.3, 32, 512, 405),
+}
+
+
+def _image_rng(config_id: int, image: int) -> np.random.Generator:
+    return np.random.Generator(np.random.PCG64(1000 * config_id + image))
+
+
+def make_image(w: Workload, image: int, N: int | None = None, D: int | None = None) -> np.ndarray:
+    """Visual tokens of one image as bf16 bits [N, D].
+
+    Token (r, c) of crop t belongs to block (r * block_rows // grid, c * block_cols // grid)
+    of that crop; each block has its own N(0, 1)^D centroid; token = centroid +
+    N(0, noise^2).  For near-duplicate images, crops 1.. copy crop 0 plus N(0, 0.05^2).
+    """
+    D = D or w.D
+    rng = _image_rng(w.config_id, image)
+    per_crop = w.grid * w.grid
+    r = np.arange(w.grid)
+    cid = (r[:, None] * w.block_rows // w.grid) * w.block_cols + (r[None, :] * w.block_cols // w.grid)
+    cid = cid.reshape(-1)
+    dup = w.near_dup_every > 0 and image % w.near_dup_every == 0
+    crops = []
+    for t in range(w.crops):
+        if dup and t > 0:
+            crop = crops[0] + rng.standard_normal((per_crop, D), dtype=np.float32) * np.float32(w.near_dup_noise)
+        else:
+            cent = rng.standard_normal((w.centroids, D), dtype=np.float32)
+            crop = cent[cid] + rng.standard_normal((per_crop, D), dtype=np.float32) * np.float32(w.noise)
+        crops.append(crop)
+    x = np.concatenate(crops, axis=0)
+    if N is not None:
+        x = x[:N]
+    return f32_to_bf16_bits(x)
+
+
+def make_text(w: Workload, image: int, M: int, D: int | None = None) -> np.ndarray:
+    """Question tokens of one image as bf16 bits [M, D], N(0, 1)."""
+    D = D or w.D
+    rng = np.random.Generator(np.random.PCG64(1000 * w.config_id + image + 1_000_000))
+    return f32_to_bf16_bits(rng.standard_normal((M, D), dtype=np.float32))
+
+
+def make_lens(w: Workload, B: int | None = None) -> np.ndarray:
+    """Per-image question lengths, uniform in [m_lo, m_hi]."""
+    B = B or w.B
+    if w.m_lo == w.m_hi:
+        return np.full(B, w.m_lo, dtype=np.int32)
+    rng = np.random.Generator(np.random.PCG64(1000 * w.config_id + 999_999))
+    return rng.integers(w.m_lo, w.m_hi + 1, size=B).astype(np.int32)
+
+
+def make_batch(w: Workload, B: int | None = None, first_image: int = 0, threads: int = 8):
+    """(vis [B, N, D] u16, text [sum(lens), D] u16, lens [B] int32) for images
+    first_image .. first_image + B - 1."""
+    B = B or w.B
+    lens_all = make_lens(w, max(w.B, first_image + B))
+    lens = lens_all[first_image:first_image + B].copy()
+    vis = np.empty((B, w.N, w.D), dtype=np.uint16)
+    texts = [None] * B
+
+    def one(b):
+        vis[b] = make_image(w, first_image + b)
+        texts[b] = make_text(w, first_image + b, int(lens[b]))
+
+    with ThreadPoolExecutor(max_workers=max(1, threads)) as ex:
+        list(ex.map(one, range(B)))
+    text = np.concatenate(texts, axis=0) if B else np.zeros((0, w.D), np.uint16)
+    return vis, text, lens
+
+
+def make_weights(dims: PredictorDims, seed: int = 7, bias_std: float = 0.0) -> dict:
+    """Seeded random-init predictor weights as bf16 bits, PyTorch Linear layout [out, in].
+
+    MLP layers: He-normal N(0, 2/fan_in); W_Q, W_K: N(0, 1/fan_in); biases N(0, bias_std^2)
+    (zero by default).  With these scales the query-key logits have a standard deviation
+    of about 2, so the predicted distribution is far from uniform.
+    """
+    rng = np.random.Generator(np.random.PCG64(seed))
+    D, Dh, dp = dims.D, dims.Dh, dims.dp
+
+    def lin(o, i, var):
+        return f32_to_bf16_bits(rng.standard_normal((o, i), dtype=np.float32) * np.float32(np.sqrt(var)))
+
+    def bias(o):
+        return f32_to_bf16_bits(rng.standard_normal(o, dtype=np.float32) * np.float32(bias_std))
+
+    w = {}
+    w["wT1"] = lin(Dh, D, 2.0 / D); w["bT1"] = bias(Dh)
+    w["wT2"] = lin(Dh, Dh, 2.0 / Dh); w["bT2"] = bias(Dh)
+    w["wQ"] = lin(dp, Dh, 1.0 / Dh)
+    w["wV1"] = lin(Dh, D, 2.0 / D); w["bV1"] = bias(Dh)
+    w["wV2"] = lin(Dh, Dh, 2.0 / Dh); w["bV2"] = bias(Dh)
+    w["wK"] = lin(dp, Dh, 1.0 / Dh)
+    return w
+
+
+def k0_for(K: int, k0_frac: float = 0.5, k0_abs: int = -1) -> int:
+    """Size of the initial top-K0 set R0: k0_abs if given, else floor(k0_frac * K),
+    clamped to [0, K].  The paper does not state K0; K/2 is the default reading."""
+    k0 = k0_abs if k0_abs >= 0 else int(np.floor(k0_frac * K))
+    return max(0, min(K, k0))
