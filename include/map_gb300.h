@@ -1,0 +1,199 @@
+/*
+ * map_gb300.h -- C ABI of the GB300 (sm_103a) implementation of MAP's inference-time
+ * visual-token pruning path (arxiv 2608.06411, "Learning to Predict Middle-layer
+ * Attention in MLLMs for Visual Token Pruning").
+ *
+ * The path:  (T, V) --map_score--> p_hat --map_select--> keep set --map_gather--> tokens
+ *
+ * Conventions for every call
+ *   - Tensors are plain pointers to row-major, densely packed arrays; bf16 tensors are
+ *     passed as void* to 16-bit storage.  Unless a call says otherwise, pointers are
+ *     DEVICE pointers owned by the caller and must stay valid until the stream work
+ *     completes; map_prune alone also accepts host pointers.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).  Work
+ *     is enqueued asynchronously on it; the call returns once enqueued.
+ *   - Return value: MAP_OK (0) or a negative MAP_E* code.  Arguments are validated on
+ *     the host before anything is enqueued; on an argument error nothing is enqueued.
+ *     Device-side failures (a bounded wait that ran out) are recorded in the context
+ *     and reported by map_status.
+ *   - A context is not thread-safe: one host thread (and one stream at a time) per
+ *     context.  Workspace is owned by the context, allocated on first use and grown on
+ *     demand (growth synchronises the device).
+ */
+#ifndef MAP_GB300_H
+#define MAP_GB300_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define MAP_OK            0
+#define MAP_EINVAL       -1   /* bad argument (null pointer, size, alignment) */
+#define MAP_ENOMEM       -2   /* device or host allocation failed */
+#define MAP_ECUDA        -3   /* a CUDA runtime / driver call failed */
+#define MAP_ETIMEOUT     -4   /* a bounded device-side wait ran out (kernel aborted) */
+#define MAP_EUNSUPPORTED -5   /* shape outside what the kernels support (see each call) */
+#define MAP_EINTERNAL    -6   /* device-side consistency check failed */
+
+typedef struct map_ctx map_ctx;   /* opaque, owned by the library */
+
+/*
+ * Predictor and selection settings.
+ *   D, Dh, dp  feature width, predictor MLP width, query/key width d of Eq. 3.
+ *              The paper calls the predictor lightweight without giving widths; the
+ *              defaults are Dh = 1024, dp = 128 (D = 4096 for LLaVA-NeXT-7B).
+ *              Supported: D % 64 == 0, Dh % 256 == 0, dp in {64, 128}.
+ *   rope_theta RoPE base (10000); rope_on = 1 applies RoPE to q and k as the paper's
+ *              predictor does (section "Cross-Modal Attention Distillation"); 0 turns it
+ *              off (used by tests of permutation equivariance).
+ *   k0_frac, k0_abs  |R0| (section "Inference-Time Token Pruning"): k0_abs if >= 0,
+ *              else floor(k0_frac * K); clamped to [0, K].  The paper does not state
+ *              K0; the default is K/2.
+ *   lambda     diversity weight: value_i = p_hat_i * rho_i^lambda.  lambda = 1 is Eq. 4;
+ *              lambda = 0 reduces the selection to the top-K of p_hat.
+ *   tau        a residual with rho_i^2 <= tau * ||v_i||^2 counts as zero (the token is
+ *              already in the span); picking such a token keeps it without extending
+ *              the basis.  Default 1e-5.
+ */
+typedef struct {
+    int   D, Dh, dp;
+    float rope_theta;
+    int   rope_on;
+    float k0_frac;
+    int   k0_abs;
+    float lambda;
+    float tau;
+} map_config;
+
+/* Predictor weights, bf16, PyTorch Linear layout [out, in]; host OR device pointers
+ * (map_init copies them).  f_T: wT1 [Dh, D], bT1 [Dh], wT2 [Dh, Dh], bT2 [Dh];
+ * W_Q: wQ [dp, Dh]; f_V: wV1, bV1, wV2, bV2 likewise; W_K: wK [dp, Dh]. */
+typedef struct {
+    const void *wT1, *bT1, *wT2, *bT2, *wQ;
+    const void *wV1, *bV1, *wV2, *bV2, *wK;
+} map_weights;
+
+/* Fills *cfg with the defaults above (D = 4096, Dh = 1024, dp = 128, theta = 1e4,
+ * rope on, K0 = K/2, lambda = 1, tau = 1e-5).  Returns MAP_EINVAL for NULL. */
+int map_config_default(map_config *cfg);
+
+/* Creates a context on the current CUDA device, copying the weights (synchronous).
+ * Returns MAP_EINVAL for a bad config or NULL pointers, MAP_ENOMEM / MAP_ECUDA on
+ * failure (then *out is NULL). */
+int map_init(const map_config *cfg, const map_weights *w, map_ctx **out);
+
+/*
+ * Predicted attention, Eq. 3 (section "Cross-Modal Attention Distillation"):
+ *   p_hat[b, n] = (1/M_b) sum_m softmax_n( <RoPE(W_Q f_T(t_m)), RoPE(W_K f_V(v_n))> / sqrt(dp) )
+ * with visual token n at position n and question token m at position N + m.
+ *   text_feats  bf16 [sum(lens), D]: the question tokens of all images, packed in
+ *               image order (device).
+ *   vis_feats   bf16 [B, N, D] (device), 16-byte aligned.
+ *   lens        int32 [B] HOST array: question tokens per image, each >= 1.
+ *   scores      float32 [B, N] output (device).
+ * B >= 1, N >= 1.  MLP outputs are rounded to bf16 after each layer; q, k, logits and
+ * p_hat are fp32.
+ */
+int map_score(map_ctx *ctx, const void *text_feats, const void *vis_feats,
+              const int32_t *lens, int B, int N, float *scores, void *stream);
+
+/*
+ * Diversity-aware selection, Eq. 4 (section "Inference-Time Token Pruning"):
+ * R0 = top-K0 by p_hat (ties to the lower index), then greedily
+ *   i_t = argmax_{i in C} p_hat_i * ||v_i - B B^T v_i||^lambda
+ * until k tokens are kept (ties to the lower index).
+ *   scores      float32 [B, N] (device), p_hat from map_score (or any non-negative
+ *               importance).
+ *   vis_feats   bf16 [B, N, D] (device): the embeddings v_i of the diversity term.
+ *   keep_idx    int32 [B, k] output (device): kept token indices restored to ascending
+ *               original order; they are also the kept tokens' position ids.
+ *   pick_order  int32 [B, k] output (device) or NULL: the same tokens in the order they
+ *               were retained (R0 in p_hat order first).
+ * k == N keeps every token (keep_idx = pick_order = 0..N-1); k == 0 is a no-op;
+ * k > N is MAP_EINVAL.  Supported: k <= 4096, N <= 16384 (MAP_EUNSUPPORTED beyond).
+ * Runs a few selection rounds per host synchronisation: the call returns after the
+ * selection has finished on the device (the final gather of indices is still queued).
+ */
+int map_select(map_ctx *ctx, const float *scores, const void *vis_feats, int B, int N,
+               int k, int32_t *keep_idx, int32_t *pick_order, void *stream);
+
+/*
+ * Compaction (last step of section "Inference-Time Token Pruning"):
+ *   out[b, j, :] = vis_feats[b, keep_idx[b, j], :]   (a bit copy of bf16 rows)
+ * vis_feats [B, N, D], out [B, k, D], keep_idx [B, k] (device).  vis_feats and out
+ * must be 16-byte aligned (MAP_EINVAL otherwise).  Indices outside [0, N) are not
+ * copied; they set MAP_EINTERNAL for map_status.
+ */
+int map_gather(map_ctx *ctx, const void *vis_feats, const int32_t *keep_idx, int B, int N,
+               int k, void *out, void *stream);
+
+/*
+ * The whole path in one call: score, select, gather.  Pointers may be HOST or DEVICE
+ * memory (detected per pointer); host inputs are copied in and host outputs copied out
+ * on `stream`, and the call synchronises `stream` before returning when any pointer is
+ * host memory.  text_feats, vis_feats, lens as for map_score (lens is always host);
+ * out bf16 [B, k, D]; keep_idx int32 [B, k]; scores float32 [B, N] or NULL.
+ */
+int map_prune(map_ctx *ctx, const void *text_feats, const void *vis_feats,
+              const int32_t *lens, int B, int N, int k, void *out, int32_t *keep_idx,
+              float *scores, void *stream);
+
+/* Synchronises `stream` and returns the first deferred device-side error recorded by
+ * this context since the last call (MAP_ETIMEOUT, MAP_EINTERNAL), clearing it; else a
+ * CUDA error as MAP_ECUDA; else MAP_OK. */
+int map_status(map_ctx *ctx, void *stream);
+
+/* Frees the context and its workspace (synchronises the device first).  NULL is a no-op. */
+void map_destroy(map_ctx *ctx);
+
+/* Static description of a MAP_E* code. */
+const char *map_strerror(int code);
+
+/* ---------------------------------------------------------------- instrumentation
+ * Counters and per-kernel CUDA-event timing used by the benchmark; not part of the
+ * paper's method. */
+typedef struct {
+    long long launches;       /* kernels this context has launched */
+    long long select_rounds;  /* selection rounds run (one round = choose, Gram, greedy) */
+    long long gram_rows;      /* Gram-block rows evaluated by the selection */
+} map_counters;
+
+int map_get_counters(map_ctx *ctx, map_counters *out);
+
+/* Kernel ids for timing. */
+#define MAP_K_GEMM_FV1    0   /* f_V layer 1: V [B*N, D] x wV1^T, GELU */
+#define MAP_K_GEMM_FV2    1
+#define MAP_K_GEMM_WK     2
+#define MAP_K_GEMM_TEXT   3   /* the three f_T / W_Q launches together */
+#define MAP_K_SCORES      4   /* softmax statistics + mean */
+#define MAP_K_SELECT      5   /* everything in map_select */
+#define MAP_K_GATHER      6
+#define MAP_K_NUM         7
+
+/* enable != 0 records a CUDA event pair around every launch of the kernels above. */
+int map_set_timing(map_ctx *ctx, int enable);
+/* Synchronises the device; returns the summed event time (ms) and count of kernel `id`
+ * since timing was enabled, and resets them. */
+int map_read_timing(map_ctx *ctx, int id, double *total_ms, long long *count);
+
+/* ---------------------------------------------------------------- diagnostics
+ * Entry points that expose internal stages for tests.  Not on the pruning path. */
+
+/* y[M, Nout] = epi(x[M, K] @ w[Nout, K]^T + b) with the library's tcgen05 GEMM.
+ * epi: 0 = GELU then bf16, 1 = bf16, 3 = fp32 (bias ignored for 3; b may be NULL).
+ * Device pointers; x, w bf16; K % 64 == 0, Nout % 64 == 0. */
+int map_linear(map_ctx *ctx, const void *x, const void *w, const void *b, int M, int K,
+               int Nout, int epi, void *y, void *stream);
+
+/* map_score that also writes q [sum(lens), dp] and k [B*N, dp] (fp32, after RoPE). */
+int map_score_debug(map_ctx *ctx, const void *text_feats, const void *vis_feats,
+                    const int32_t *lens, int B, int N, float *scores, float *q_out,
+                    float *k_out, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MAP_GB300_H */

@@ -1,0 +1,622 @@
+// C ABI of libmap_gb300 (include/map_gb300.h): context, workspace, argument checks and
+// the orchestration of the kernels for score (Eq. 3), select (Eq. 4) and gather.
+#include <cmath>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "../../include/map_gb300.h"
+#include "kernels.h"
+#include "ptx.cuh"
+#include "select.h"
+
+using mapk::GemmDesc;
+
+namespace {
+
+constexpr int kSelS = 128;          // active-set size of the selection (Gram block rows)
+constexpr int kMaxK = 4096;
+constexpr int kMaxN = 16384;
+
+struct DevBuf {
+  void* p = nullptr;
+  size_t cap = 0;
+};
+
+struct TimedPair { cudaEvent_t a, b; int id; };
+
+}  // namespace
+
+struct map_ctx {
+  map_config cfg{};
+  int device = 0, num_sms = 148;
+  void* w[10] = {};                 // wT1 bT1 wT2 bT2 wQ wV1 bV1 wV2 bV2 wK (device bf16)
+  DevBuf rope;  int rope_rows = 0;
+  DevBuf h1, h2, kb, th1, th2, qb, stats, qoff, post, sqn;
+  // selection
+  DevBuf sU, sr2, scstep, sstate, sEc, spicks, sr0, sbt, srn, ssmall, stheta, saslot, sVg, sG;
+  // map_prune staging
+  DevBuf pvis, ptext, pout, pkeep, pscores;
+  int* status = nullptr;            // device status word
+  int* h_status = nullptr;          // pinned
+  int32_t* h_done = nullptr;        // pinned
+  void* h_stage = nullptr; size_t h_stage_cap = 0;   // pinned host staging (offsets, positions)
+  cudaEvent_t stage_ev = nullptr; bool stage_pending = false;
+  bool timing = false;
+  std::vector<TimedPair> pairs;
+  std::vector<cudaEvent_t> free_events;
+  double t_ms[MAP_K_NUM] = {};
+  long long t_n[MAP_K_NUM] = {};
+  map_counters counters{};
+  int deferred = MAP_OK;
+};
+
+namespace {
+
+int cuda_err(cudaError_t e) { return e == cudaSuccess ? MAP_OK : (e == cudaErrorMemoryAllocation ? MAP_ENOMEM : MAP_ECUDA); }
+
+#define MAP_TRY(expr)                      \
+  do {                                     \
+    int _rc = (expr);                      \
+    if (_rc != MAP_OK) return _rc;         \
+  } while (0)
+#define CU_TRY(expr) MAP_TRY(cuda_err(expr))
+
+int ensure(DevBuf& b, size_t bytes) {
+  if (bytes <= b.cap) return MAP_OK;
+  if (b.p) {
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) return MAP_ECUDA;
+    cudaFree(b.p);
+    b.p = nullptr;
+    b.cap = 0;
+  }
+  size_t want = bytes + bytes / 8 + 256;
+  if (cudaMalloc(&b.p, want) != cudaSuccess) {
+    cudaGetLastError();
+    return MAP_ENOMEM;
+  }
+  b.cap = want;
+  return MAP_OK;
+}
+
+void release(DevBuf& b) {
+  if (b.p) cudaFree(b.p);
+  b.p = nullptr;
+  b.cap = 0;
+}
+
+cudaEvent_t take_event(map_ctx* c) {
+  if (!c->free_events.empty()) {
+    cudaEvent_t e = c->free_events.back();
+    c->free_events.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  cudaEventCreate(&e);
+  return e;
+}
+
+// Brackets a launch with CUDA events when timing is on.
+struct Timed {
+  map_ctx* c; cudaStream_t st; int id; cudaEvent_t a = nullptr;
+  Timed(map_ctx* c_, cudaStream_t st_, int id_) : c(c_), st(st_), id(id_) {
+    if (c->timing) { a = take_event(c); cudaEventRecord(a, st); }
+  }
+  ~Timed() {
+    if (a) {
+      cudaEvent_t b = take_event(c);
+      cudaEventRecord(b, st);
+      c->pairs.push_back({a, b, id});
+    }
+  }
+};
+
+int dev_status_error(int st) {
+  if (st & mapk::ST_TIMEOUT) return MAP_ETIMEOUT;
+  if (st) return MAP_EINTERNAL;
+  return MAP_OK;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+
+int check_config(const map_config* c) {
+  if (!c) return MAP_EINVAL;
+  if (c->D <= 0 || c->D % 64 != 0) return MAP_EINVAL;
+  if (c->Dh <= 0 || c->Dh % 256 != 0) return MAP_EINVAL;
+  if (c->dp != 64 && c->dp != 128) return MAP_EINVAL;
+  if (!(c->rope_theta > 0.f)) return MAP_EINVAL;
+  if (!(c->lambda >= 0.f) || !(c->tau >= 0.f) || !(c->k0_frac >= 0.f)) return MAP_EINVAL;
+  return MAP_OK;
+}
+
+int resolve_k0(const map_config& c, int K) {
+  long long k0 = c.k0_abs >= 0 ? c.k0_abs : static_cast<long long>(std::floor(static_cast<double>(c.k0_frac) * K));
+  if (k0 < 0) k0 = 0;
+  if (k0 > K) k0 = K;
+  return static_cast<int>(k0);
+}
+
+// RoPE table (cos, sin) of pos * theta^(-2i/dp), i < dp/2, for pos < rows; computed in
+// double on the host, stored as float.
+int ensure_rope(map_ctx* c, int rows_needed) {
+  if (rows_needed <= c->rope_rows) return MAP_OK;
+  const int rows = ((rows_needed + 1023) / 1024) * 1024;
+  const int half = c->cfg.dp / 2;
+  std::vector<float2> tab(static_cast<size_t>(rows) * half);
+  for (int p = 0; p < rows; ++p)
+    for (int i = 0; i < half; ++i) {
+      const double f = std::pow(static_cast<double>(c->cfg.rope_theta), -2.0 * i / c->cfg.dp);
+      const double a = p * f;
+      tab[static_cast<size_t>(p) * half + i] = make_float2(static_cast<float>(std::cos(a)), static_cast<float>(std::sin(a)));
+    }
+  MAP_TRY(ensure(c->rope, tab.size() * sizeof(float2)));
+  CU_TRY(cudaMemcpy(c->rope.p, tab.data(), tab.size() * sizeof(float2), cudaMemcpyHostToDevice));
+  c->rope_rows = rows;
+  return MAP_OK;
+}
+
+int stage_host(map_ctx* c, size_t bytes, void** out) {
+  if (c->stage_pending) {
+    cudaEventSynchronize(c->stage_ev);
+    c->stage_pending = false;
+  }
+  if (bytes > c->h_stage_cap) {
+    if (c->h_stage) cudaFreeHost(c->h_stage);
+    c->h_stage = nullptr;
+    c->h_stage_cap = 0;
+    if (cudaMallocHost(&c->h_stage, bytes + 4096) != cudaSuccess) { cudaGetLastError(); return MAP_ENOMEM; }
+    c->h_stage_cap = bytes + 4096;
+  }
+  *out = c->h_stage;
+  return MAP_OK;
+}
+
+int gemm(map_ctx* c, const GemmDesc& d, cudaStream_t st) {
+  ++c->counters.launches;
+  cudaError_t e = mapk::launch_gemm(d, c->num_sms, st);
+  if (e == cudaErrorInvalidValue) return MAP_EUNSUPPORTED;
+  return cuda_err(e);
+}
+
+GemmDesc linear_desc(map_ctx* c, const void* x, long long rows, int K, const void* w, int Nout, const void* bias,
+                     void* y, int epi) {
+  GemmDesc d{};
+  d.A = x; d.a_rows_total = rows; d.a_row_stride = 0;
+  d.B = w; d.b_rows_total = Nout; d.b_row_stride = 0;
+  d.M = static_cast<int>(rows); d.N = Nout; d.K = K; d.batch = 1;
+  d.n_limit = nullptr; d.C = y; d.ldc = Nout; d.c_batch_stride = 0;
+  d.bias = bias; d.rope = nullptr; d.rope_half = c->cfg.dp / 2; d.pos = nullptr; d.pos_mod = 1;
+  d.epi = epi; d.status = c->status;
+  return d;
+}
+
+// Predictor for one modality: x [rows, D] -> RoPE(W f(x)) [rows, dp] fp32.
+int predictor_branch(map_ctx* c, const void* x, long long rows, const void* w1, const void* b1, const void* w2,
+                     const void* b2, const void* wp, DevBuf& h1, DevBuf& h2, float* out, const int* pos, int pos_mod,
+                     cudaStream_t st, int tid_l1, int tid_l2, int tid_p) {
+  const map_config& g = c->cfg;
+  MAP_TRY(ensure(h1, static_cast<size_t>(rows) * g.Dh * 2));
+  MAP_TRY(ensure(h2, static_cast<size_t>(rows) * g.Dh * 2));
+  {
+    Timed t(c, st, tid_l1);
+    MAP_TRY(gemm(c, linear_desc(c, x, rows, g.D, w1, g.Dh, b1, h1.p, mapk::EPI_GELU_BF16), st));
+  }
+  {
+    Timed t(c, st, tid_l2);
+    MAP_TRY(gemm(c, linear_desc(c, h1.p, rows, g.Dh, w2, g.Dh, b2, h2.p, mapk::EPI_BIAS_BF16), st));
+  }
+  {
+    Timed t(c, st, tid_p);
+    GemmDesc d = linear_desc(c, h2.p, rows, g.Dh, wp, g.dp, nullptr, out, g.rope_on ? mapk::EPI_ROPE_F32 : mapk::EPI_F32);
+    d.rope = static_cast<const float2*>(c->rope.p);
+    d.pos = pos;
+    d.pos_mod = pos_mod;
+    MAP_TRY(gemm(c, d, st));
+  }
+  return MAP_OK;
+}
+
+int score_impl(map_ctx* c, const void* text, const void* vis, const int32_t* lens, int B, int N, float* scores,
+               float* q_out, float* k_out, cudaStream_t st) {
+  if (!c || !text || !vis || !lens || !scores) return MAP_EINVAL;
+  if (B < 1 || N < 1) return MAP_EINVAL;
+  if (!aligned16(text) || !aligned16(vis)) return MAP_EINVAL;
+  long long total_m = 0;
+  int max_m = 0;
+  for (int b = 0; b < B; ++b) {
+    if (lens[b] < 1) return MAP_EINVAL;
+    total_m += lens[b];
+    max_m = lens[b] > max_m ? lens[b] : max_m;
+  }
+  if (total_m > (1ll << 30) || static_cast<long long>(B) * N > (1ll << 30)) return MAP_EUNSUPPORTED;
+  const map_config& g = c->cfg;
+  CU_TRY(cudaSetDevice(c->device));
+  if (g.rope_on) MAP_TRY(ensure_rope(c, N + max_m + 1));
+  // per-image query offsets and question-token positions N + m
+  const size_t off_bytes = static_cast<size_t>(B + 1) * 4, pos_bytes = static_cast<size_t>(total_m) * 4;
+  void* hs = nullptr;
+  MAP_TRY(stage_host(c, off_bytes + pos_bytes, &hs));
+  int32_t* hoff = static_cast<int32_t*>(hs);
+  int32_t* hpos = hoff + (B + 1);
+  hoff[0] = 0;
+  for (int b = 0; b < B; ++b) {
+    hoff[b + 1] = hoff[b] + lens[b];
+    for (int m = 0; m < lens[b]; ++m) hpos[hoff[b] + m] = N + m;
+  }
+  MAP_TRY(ensure(c->qoff, off_bytes));
+  MAP_TRY(ensure(c->post, pos_bytes));
+  CU_TRY(cudaMemcpyAsync(c->qoff.p, hoff, off_bytes, cudaMemcpyHostToDevice, st));
+  CU_TRY(cudaMemcpyAsync(c->post.p, hpos, pos_bytes, cudaMemcpyHostToDevice, st));
+  CU_TRY(cudaEventRecord(c->stage_ev, st));
+  c->stage_pending = true;
+
+  const long long vrows = static_cast<long long>(B) * N;
+  MAP_TRY(ensure(c->kb, static_cast<size_t>(vrows) * g.dp * 4));
+  MAP_TRY(ensure(c->qb, static_cast<size_t>(total_m) * g.dp * 4));
+  MAP_TRY(predictor_branch(c, vis, vrows, c->w[5], c->w[6], c->w[7], c->w[8], c->w[9], c->h1, c->h2,
+                           static_cast<float*>(c->kb.p), nullptr, N, st, MAP_K_GEMM_FV1, MAP_K_GEMM_FV2, MAP_K_GEMM_WK));
+  MAP_TRY(predictor_branch(c, text, total_m, c->w[0], c->w[1], c->w[2], c->w[3], c->w[4], c->th1, c->th2,
+                           static_cast<float*>(c->qb.p), static_cast<const int*>(c->post.p), 1, st, MAP_K_GEMM_TEXT,
+                           MAP_K_GEMM_TEXT, MAP_K_GEMM_TEXT));
+  // Eq. 3: split the keys so that the statistics pass fills the GPU
+  int nsplit = 1;
+  const long long mblocks = static_cast<long long>(B) * ((max_m + 127) / 128);
+  while (nsplit < 64 && mblocks * nsplit < 4LL * c->num_sms && N / (nsplit * 2) >= 64) nsplit *= 2;
+  MAP_TRY(ensure(c->stats, static_cast<size_t>(total_m) * nsplit * 8));
+  mapk::ScoreDesc sd{};
+  sd.q = static_cast<const float*>(c->qb.p); sd.k = static_cast<const float*>(c->kb.p);
+  sd.q_off = static_cast<const int*>(c->qoff.p); sd.B = B; sd.N = N; sd.dp = g.dp; sd.max_m = max_m;
+  sd.stats = static_cast<float*>(c->stats.p); sd.nsplit = nsplit; sd.scores = scores; sd.status = c->status;
+  {
+    Timed t(c, st, MAP_K_SCORES);
+    c->counters.launches += 2;
+    CU_TRY(mapk::launch_scores(sd, st));
+  }
+  if (q_out) CU_TRY(cudaMemcpyAsync(q_out, c->qb.p, static_cast<size_t>(total_m) * g.dp * 4, cudaMemcpyDeviceToDevice, st));
+  if (k_out) CU_TRY(cudaMemcpyAsync(k_out, c->kb.p, static_cast<size_t>(vrows) * g.dp * 4, cudaMemcpyDeviceToDevice, st));
+  return MAP_OK;
+}
+
+template <typename T>
+T* carve(char*& p, size_t n) {
+  T* r = reinterpret_cast<T*>(p);
+  p += ((n * sizeof(T) + 255) / 256) * 256;
+  return r;
+}
+
+int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, int K, int32_t* keep,
+                int32_t* order, cudaStream_t st) {
+  if (!c || !scores || !vis) return MAP_EINVAL;
+  if (B < 1 || N < 1 || K < 0 || K > N) return MAP_EINVAL;
+  if (K == 0) return MAP_OK;
+  if (!keep) return MAP_EINVAL;
+  if (K > kMaxK || N > kMaxN) return MAP_EUNSUPPORTED;
+  if (!aligned16(vis)) return MAP_EINVAL;
+  CU_TRY(cudaSetDevice(c->device));
+  Timed timed(c, st, MAP_K_SELECT);
+  if (K == N) {
+    ++c->counters.launches;
+    CU_TRY(mapk::launch_sel_identity(B, N, keep, order, st));
+    return MAP_OK;
+  }
+  const map_config& g = c->cfg;
+  int K0 = resolve_k0(g, K);
+  if (g.lambda == 0.f) K0 = K;        // values are p_hat alone: plain top-K
+  const long long BN = static_cast<long long>(B) * N;
+  const int S = kSelS, R = kSelS + K;
+
+  mapk::SelState s{};
+  s.B = B; s.N = N; s.D = g.D; s.K = K; s.K0 = K0; s.S = S;
+  s.lambda = g.lambda; s.tau = g.tau;
+  s.scores = scores; s.V = vis; s.status = c->status;
+  // per-token arrays
+  MAP_TRY(ensure(c->sqn, BN * 4));
+  MAP_TRY(ensure(c->sU, BN * 4));
+  MAP_TRY(ensure(c->sr2, BN * 4));
+  MAP_TRY(ensure(c->scstep, BN * 4));
+  MAP_TRY(ensure(c->sstate, BN));
+  MAP_TRY(ensure(c->spicks, static_cast<size_t>(B) * K * 4));
+  MAP_TRY(ensure(c->sr0, static_cast<size_t>(B) * K * 4));
+  MAP_TRY(ensure(c->sbt, static_cast<size_t>(B) * K * 4));
+  MAP_TRY(ensure(c->srn, static_cast<size_t>(B) * K * 4));
+  MAP_TRY(ensure(c->ssmall, static_cast<size_t>(B) * 8 * 256 + 256));
+  MAP_TRY(ensure(c->stheta, static_cast<size_t>(B) * 8));
+  MAP_TRY(ensure(c->saslot, static_cast<size_t>(B) * S * 4));
+  s.sqn = static_cast<float*>(c->sqn.p);
+  s.U = static_cast<float*>(c->sU.p);
+  s.r2 = static_cast<float*>(c->sr2.p);
+  s.cstep = static_cast<int32_t*>(c->scstep.p);
+  s.state = static_cast<uint8_t*>(c->sstate.p);
+  s.picks = static_cast<int32_t*>(c->spicks.p);
+  s.r0 = static_cast<int32_t*>(c->sr0.p);
+  s.basis_tok = static_cast<int32_t*>(c->sbt.p);
+  s.rnorm = static_cast<float*>(c->srn.p);
+  char* sm = static_cast<char*>(c->ssmall.p);
+  s.npicks = carve<int32_t>(sm, B);
+  s.nbasis = carve<int32_t>(sm, B);
+  s.nb_gathered = carve<int32_t>(sm, B);
+  s.done = carve<int32_t>(sm, B);
+  s.mode = carve<int32_t>(sm, B);
+  s.nlimit = carve<int32_t>(sm, B);
+  s.done_count = carve<int32_t>(sm, 1);
+  s.theta = static_cast<uint64_t*>(c->stheta.p);
+  s.aslot = static_cast<int32_t*>(c->saslot.p);
+
+  if (K0 < K) {
+    ++c->counters.launches;
+    CU_TRY(mapk::launch_row_sqnorm(vis, BN, g.D, static_cast<float*>(c->sqn.p), st));
+  } else {
+    CU_TRY(cudaMemsetAsync(c->sqn.p, 0, BN * 4, st));
+  }
+  ++c->counters.launches;
+  CU_TRY(mapk::launch_sel_init(s, st));
+  if (K0 < K) {
+    MAP_TRY(ensure(c->sEc, static_cast<size_t>(BN) * K * 4));
+    MAP_TRY(ensure(c->sVg, static_cast<size_t>(B) * R * g.D * 2));
+    MAP_TRY(ensure(c->sG, static_cast<size_t>(B) * S * R * 4));
+    s.Ec = static_cast<float*>(c->sEc.p);
+    s.Vg = c->sVg.p;
+    s.G = static_cast<float*>(c->sG.p);
+    CU_TRY(cudaMemsetAsync(s.done_count, 0, 4, st));
+    GemmDesc d{};
+    d.A = s.Vg; d.a_rows_total = static_cast<long long>(B) * R; d.a_row_stride = R;
+    d.B = s.Vg; d.b_rows_total = static_cast<long long>(B) * R; d.b_row_stride = R;
+    d.M = S; d.N = R; d.K = g.D; d.batch = B; d.n_limit = s.nlimit;
+    d.C = s.G; d.ldc = R; d.c_batch_stride = static_cast<long long>(S) * R;
+    d.epi = mapk::EPI_F32; d.status = c->status;
+    const long long cap = 8LL * (K + N / S) + 64;
+    long long rounds = 0;
+    int burst = (K0 + S - 1) / S + 2;
+    for (;;) {
+      for (int r = 0; r < burst; ++r) {
+        c->counters.launches += 2;
+        CU_TRY(mapk::launch_sel_choose(s, st));
+        MAP_TRY(gemm(c, d, st));
+        CU_TRY(mapk::launch_sel_greedy(s, st));
+      }
+      rounds += burst;
+      c->counters.select_rounds += burst;
+      CU_TRY(cudaMemcpyAsync(c->h_done, s.done_count, 4, cudaMemcpyDeviceToHost, st));
+      CU_TRY(cudaStreamSynchronize(st));
+      if (*c->h_done >= B) break;
+      if (rounds > cap) {
+        c->deferred = MAP_EINTERNAL;
+        return MAP_EINTERNAL;
+      }
+      burst = 2;
+    }
+  } else {
+    ++c->counters.launches;
+    CU_TRY(mapk::launch_sel_copy_r0(s.r0, B, K, s.picks, st));
+  }
+  ++c->counters.launches;
+  CU_TRY(mapk::launch_sel_finalize(s.picks, B, K, keep, order, st));
+  return MAP_OK;
+}
+
+int gather_impl(map_ctx* c, const void* vis, const int32_t* keep, int B, int N, int K, void* out, cudaStream_t st) {
+  if (!c || !vis) return MAP_EINVAL;
+  if (B < 1 || N < 1 || K < 0) return MAP_EINVAL;
+  if (K == 0) return MAP_OK;
+  if (!keep || !out) return MAP_EINVAL;
+  if (!aligned16(vis) || !aligned16(out)) return MAP_EINVAL;
+  CU_TRY(cudaSetDevice(c->device));
+  Timed t(c, st, MAP_K_GATHER);
+  ++c->counters.launches;
+  CU_TRY(mapk::launch_gather(vis, keep, B, N, K, c->cfg.D, out, c->status, st));
+  return MAP_OK;
+}
+
+bool is_device_ptr(const void* p) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
+}
+
+}  // namespace
+
+extern "C" {
+
+int map_config_default(map_config* cfg) {
+  if (!cfg) return MAP_EINVAL;
+  cfg->D = 4096; cfg->Dh = 1024; cfg->dp = 128;
+  cfg->rope_theta = 10000.f; cfg->rope_on = 1;
+  cfg->k0_frac = 0.5f; cfg->k0_abs = -1;
+  cfg->lambda = 1.0f; cfg->tau = 1e-5f;
+  return MAP_OK;
+}
+
+int map_init(const map_config* cfg, const map_weights* w, map_ctx** out) {
+  if (!out) return MAP_EINVAL;
+  *out = nullptr;
+  if (check_config(cfg) != MAP_OK || !w) return MAP_EINVAL;
+  const void* src[10] = {w->wT1, w->bT1, w->wT2, w->bT2, w->wQ, w->wV1, w->bV1, w->wV2, w->bV2, w->wK};
+  for (const void* p : src)
+    if (!p) return MAP_EINVAL;
+  map_ctx* c = new (std::nothrow) map_ctx();
+  if (!c) return MAP_ENOMEM;
+  c->cfg = *cfg;
+  int rc = MAP_OK;
+  do {
+    if (cudaGetDevice(&c->device) != cudaSuccess) { rc = MAP_ECUDA; break; }
+    if (cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, c->device) != cudaSuccess) { rc = MAP_ECUDA; break; }
+    const size_t D = cfg->D, Dh = cfg->Dh, dp = cfg->dp;
+    const size_t n[10] = {Dh * D, Dh, Dh * Dh, Dh, dp * Dh, Dh * D, Dh, Dh * Dh, Dh, dp * Dh};
+    for (int i = 0; i < 10 && rc == MAP_OK; ++i) {
+      if (cudaMalloc(&c->w[i], n[i] * 2) != cudaSuccess) { rc = MAP_ENOMEM; break; }
+      if (cudaMemcpy(c->w[i], src[i], n[i] * 2, cudaMemcpyDefault) != cudaSuccess) rc = MAP_ECUDA;
+    }
+    if (rc != MAP_OK) break;
+    if (cudaMalloc(&c->status, sizeof(int)) != cudaSuccess) { rc = MAP_ENOMEM; break; }
+    if (cudaMemset(c->status, 0, sizeof(int)) != cudaSuccess) { rc = MAP_ECUDA; break; }
+    if (cudaMallocHost(&c->h_status, sizeof(int)) != cudaSuccess) { rc = MAP_ENOMEM; break; }
+    if (cudaMallocHost(&c->h_done, sizeof(int32_t)) != cudaSuccess) { rc = MAP_ENOMEM; break; }
+    if (cudaEventCreateWithFlags(&c->stage_ev, cudaEventDisableTiming) != cudaSuccess) { rc = MAP_ECUDA; break; }
+  } while (false);
+  if (rc != MAP_OK) {
+    cudaGetLastError();
+    map_destroy(c);
+    return rc;
+  }
+  *out = c;
+  return MAP_OK;
+}
+
+int map_score(map_ctx* ctx, const void* text_feats, const void* vis_feats, const int32_t* lens, int B, int N,
+              float* scores, void* stream) {
+  return score_impl(ctx, text_feats, vis_feats, lens, B, N, scores, nullptr, nullptr, static_cast<cudaStream_t>(stream));
+}
+
+int map_score_debug(map_ctx* ctx, const void* text_feats, const void* vis_feats, const int32_t* lens, int B, int N,
+                    float* scores, float* q_out, float* k_out, void* stream) {
+  return score_impl(ctx, text_feats, vis_feats, lens, B, N, scores, q_out, k_out, static_cast<cudaStream_t>(stream));
+}
+
+int map_select(map_ctx* ctx, const float* scores, const void* vis_feats, int B, int N, int k, int32_t* keep_idx,
+               int32_t* pick_order, void* stream) {
+  return select_impl(ctx, scores, vis_feats, B, N, k, keep_idx, pick_order, static_cast<cudaStream_t>(stream));
+}
+
+int map_gather(map_ctx* ctx, const void* vis_feats, const int32_t* keep_idx, int B, int N, int k, void* out,
+               void* stream) {
+  return gather_impl(ctx, vis_feats, keep_idx, B, N, k, out, static_cast<cudaStream_t>(stream));
+}
+
+int map_prune(map_ctx* ctx, const void* text_feats, const void* vis_feats, const int32_t* lens, int B, int N, int k,
+              void* out, int32_t* keep_idx, float* scores, void* stream) {
+  if (!ctx || !text_feats || !vis_feats || !lens || !out || !keep_idx) return MAP_EINVAL;
+  if (B < 1 || N < 1 || k < 0 || k > N) return MAP_EINVAL;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  map_ctx* c = ctx;
+  CU_TRY(cudaSetDevice(c->device));
+  long long total_m = 0;
+  for (int b = 0; b < B; ++b) {
+    if (lens[b] < 1) return MAP_EINVAL;
+    total_m += lens[b];
+  }
+  const size_t D = c->cfg.D;
+  const size_t vis_bytes = static_cast<size_t>(B) * N * D * 2, text_bytes = static_cast<size_t>(total_m) * D * 2;
+  const size_t out_bytes = static_cast<size_t>(B) * k * D * 2, keep_bytes = static_cast<size_t>(B) * k * 4;
+  const size_t sc_bytes = static_cast<size_t>(B) * N * 4;
+  const bool dv = is_device_ptr(vis_feats), dt = is_device_ptr(text_feats), dout = is_device_ptr(out);
+  const bool dkeep = is_device_ptr(keep_idx), dsc = scores ? is_device_ptr(scores) : true;
+  const void* v = vis_feats;
+  const void* t = text_feats;
+  if (!dv) { MAP_TRY(ensure(c->pvis, vis_bytes)); CU_TRY(cudaMemcpyAsync(c->pvis.p, vis_feats, vis_bytes, cudaMemcpyHostToDevice, st)); v = c->pvis.p; }
+  if (!dt) { MAP_TRY(ensure(c->ptext, text_bytes)); CU_TRY(cudaMemcpyAsync(c->ptext.p, text_feats, text_bytes, cudaMemcpyHostToDevice, st)); t = c->ptext.p; }
+  void* o = out;
+  int32_t* kp = keep_idx;
+  float* sp = scores;
+  if (!dout) { MAP_TRY(ensure(c->pout, out_bytes)); o = c->pout.p; }
+  if (!dkeep) { MAP_TRY(ensure(c->pkeep, keep_bytes)); kp = static_cast<int32_t*>(c->pkeep.p); }
+  if (!dsc || !scores) { MAP_TRY(ensure(c->pscores, sc_bytes)); sp = static_cast<float*>(c->pscores.p); }
+  MAP_TRY(score_impl(c, t, v, lens, B, N, sp, nullptr, nullptr, st));
+  MAP_TRY(select_impl(c, sp, v, B, N, k, kp, nullptr, st));
+  MAP_TRY(gather_impl(c, v, kp, B, N, k, o, st));
+  bool sync = !dv || !dt;
+  if (!dout) { CU_TRY(cudaMemcpyAsync(out, o, out_bytes, cudaMemcpyDeviceToHost, st)); sync = true; }
+  if (!dkeep) { CU_TRY(cudaMemcpyAsync(keep_idx, kp, keep_bytes, cudaMemcpyDeviceToHost, st)); sync = true; }
+  if (scores && !dsc) { CU_TRY(cudaMemcpyAsync(scores, sp, sc_bytes, cudaMemcpyDeviceToHost, st)); sync = true; }
+  if (sync) CU_TRY(cudaStreamSynchronize(st));
+  return MAP_OK;
+}
+
+int map_status(map_ctx* ctx, void* stream) {
+  if (!ctx) return MAP_EINVAL;
+  if (cudaSetDevice(ctx->device) != cudaSuccess) return MAP_ECUDA;
+  cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return MAP_ECUDA;
+  if (cudaMemcpy(ctx->h_status, ctx->status, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess) return MAP_ECUDA;
+  int rc = dev_status_error(*ctx->h_status);
+  if (*ctx->h_status) cudaMemset(ctx->status, 0, sizeof(int));
+  if (rc == MAP_OK && ctx->deferred != MAP_OK) rc = ctx->deferred;
+  ctx->deferred = MAP_OK;
+  e = cudaGetLastError();
+  if (rc == MAP_OK && e != cudaSuccess) rc = MAP_ECUDA;
+  return rc;
+}
+
+void map_destroy(map_ctx* ctx) {
+  if (!ctx) return;
+  cudaSetDevice(ctx->device);
+  cudaDeviceSynchronize();
+  for (void*& p : ctx->w)
+    if (p) cudaFree(p);
+  DevBuf* bufs[] = {&ctx->rope, &ctx->h1, &ctx->h2, &ctx->kb, &ctx->th1, &ctx->th2, &ctx->qb, &ctx->stats,
+                    &ctx->qoff, &ctx->post, &ctx->sqn, &ctx->sU, &ctx->sr2, &ctx->scstep, &ctx->sstate,
+                    &ctx->sEc, &ctx->spicks, &ctx->sr0, &ctx->sbt, &ctx->srn, &ctx->ssmall, &ctx->stheta,
+                    &ctx->saslot, &ctx->sVg, &ctx->sG, &ctx->pvis, &ctx->ptext, &ctx->pout, &ctx->pkeep,
+                    &ctx->pscores};
+  for (DevBuf* b : bufs) release(*b);
+  if (ctx->status) cudaFree(ctx->status);
+  if (ctx->h_status) cudaFreeHost(ctx->h_status);
+  if (ctx->h_done) cudaFreeHost(ctx->h_done);
+  if (ctx->h_stage) cudaFreeHost(ctx->h_stage);
+  if (ctx->stage_ev) cudaEventDestroy(ctx->stage_ev);
+  for (auto& pr : ctx->pairs) { cudaEventDestroy(pr.a); cudaEventDestroy(pr.b); }
+  for (auto e : ctx->free_events) cudaEventDestroy(e);
+  delete ctx;
+}
+
+const char* map_strerror(int code) {
+  switch (code) {
+    case MAP_OK: return "ok";
+    case MAP_EINVAL: return "invalid argument";
+    case MAP_ENOMEM: return "out of memory";
+    case MAP_ECUDA: return "CUDA error";
+    case MAP_ETIMEOUT: return "device-side wait timed out";
+    case MAP_EUNSUPPORTED: return "unsupported shape";
+    case MAP_EINTERNAL: return "device-side consistency check failed";
+    default: return "unknown error";
+  }
+}
+
+int map_get_counters(map_ctx* ctx, map_counters* out) {
+  if (!ctx || !out) return MAP_EINVAL;
+  *out = ctx->counters;
+  return MAP_OK;
+}
+
+int map_set_timing(map_ctx* ctx, int enable) {
+  if (!ctx) return MAP_EINVAL;
+  ctx->timing = enable != 0;
+  return MAP_OK;
+}
+
+int map_read_timing(map_ctx* ctx, int id, double* total_ms, long long* count) {
+  if (!ctx || id < 0 || id >= MAP_K_NUM || !total_ms || !count) return MAP_EINVAL;
+  if (cudaDeviceSynchronize() != cudaSuccess) return MAP_ECUDA;
+  for (auto& pr : ctx->pairs) {
+    float ms = 0.f;
+    cudaEventElapsedTime(&ms, pr.a, pr.b);
+    ctx->t_ms[pr.id] += ms;
+    ctx->t_n[pr.id] += 1;
+    ctx->free_events.push_back(pr.a);
+    ctx->free_events.push_back(pr.b);
+  }
+  ctx->pairs.clear();
+  *total_ms = ctx->t_ms[id];
+  *count = ctx->t_n[id];
+  ctx->t_ms[id] = 0;
+  ctx->t_n[id] = 0;
+  return MAP_OK;
+}
+
+int map_linear(map_ctx* ctx, const void* x, const void* w, const void* b, int M, int K, int Nout, int epi, void* y,
+               void* stream) {
+  if (!ctx || !x || !w || !y || M < 0 || K <= 0 || Nout <= 0) return MAP_EINVAL;
+  if (epi != mapk::EPI_GELU_BF16 && epi != mapk::EPI_BIAS_BF16 && epi != mapk::EPI_F32) return MAP_EINVAL;
+  if (K % 64 != 0 || Nout % 64 != 0) return MAP_EUNSUPPORTED;
+  if (!aligned16(x) || !aligned16(w) || !aligned16(y)) return MAP_EINVAL;
+  if (cudaSetDevice(ctx->device) != cudaSuccess) return MAP_ECUDA;
+  GemmDesc d = linear_desc(ctx, x, M, K, w, Nout, epi == mapk::EPI_F32 ? nullptr : b, y, epi);
+  return gemm(ctx, d, static_cast<cudaStream_t>(stream));
+}
+
+}  // extern "C"

@@ -1,0 +1,360 @@
+// Persistent tcgen05 GEMM for sm_103a:  C = epilogue(A @ B^T), A [M, K], B [N, K] bf16.
+//
+// Used for every dense contraction of the pruning path: the predictor layers f_V, f_T
+// (Linear -> GELU -> Linear), the W_K / W_Q projections with RoPE fused into the
+// epilogue (section "Cross-Modal Attention Distillation"), and the Gram blocks
+// <v_i, v_j> that the diversity term of Eq. 4 needs.
+//
+// Structure (one CTA per SM, 6 warps):
+//   warp 0      one thread issues TMA loads of 128x64 (A) and BNx64 (B) bf16 tiles, 128-byte
+//               swizzled, into a STAGES-deep shared-memory ring (mbarrier full/empty).
+//   warp 1      allocates TMEM (2 accumulators x BN fp32 columns); one thread issues
+//               tcgen05.mma (M=128, N=BN, K=16) x 4 per stage and commits to mbarriers.
+//   warps 2-5   epilogue: tcgen05.ld the accumulator (one TMEM lane = one output row per
+//               thread), apply bias / GELU / RoPE, store; release the accumulator so the
+//               MMA warp can start the tile after next while this one drains.
+// All waits are bounded (ptx.cuh); a timeout sets ST_TIMEOUT and every role drains and exits.
+#include <algorithm>
+#include <cstdio>
+#include <cudaTypedefs.h>
+
+#include "kernels.h"
+#include "ptx.cuh"
+
+namespace mapk {
+
+namespace {
+
+constexpr int kBM = 128;
+constexpr int kBK = 64;
+constexpr int kThreads = 192;
+
+struct KArgs {
+  int M, N, K, batch, a_row_stride, b_row_stride;
+  const int* n_limit;
+  void* C; long long ldc; long long c_batch_stride;
+  const __nv_bfloat16* bias;
+  const float2* rope; int rope_half;
+  const int* pos; int pos_mod;
+  int* status;
+};
+
+__device__ __forceinline__ float gelu_erf(float x) {
+  return 0.5f * x * (1.0f + erff(x * 0.70710678118654752f));
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(a, b);   // .x = a (low half), .y = b
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+
+template <int BN, int STAGES>
+struct Smem {
+  static constexpr uint32_t A_BYTES = kBM * kBK * 2;
+  static constexpr uint32_t B_BYTES = BN * kBK * 2;
+  static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr uint32_t TILES = STAGES * STAGE_BYTES;
+  static constexpr uint32_t BARS = (2 * STAGES + 5) * 8;
+  static constexpr uint32_t TOTAL = 1024 + TILES + BARS + 16;
+  static constexpr uint32_t TMEM_COLS = 2 * BN;
+};
+
+struct TileCoord { int b, m_blk, n_blk; bool skip; };
+
+__device__ __forceinline__ TileCoord tile_coord(const KArgs& a, int t, int m_tiles, int n_tiles, int BN) {
+  TileCoord c;
+  int per = m_tiles * n_tiles;
+  c.b = t / per;
+  int rem = t - c.b * per;
+  c.m_blk = rem / n_tiles;
+  c.n_blk = rem - c.m_blk * n_tiles;
+  int lim = a.n_limit ? min(a.N, __ldg(a.n_limit + c.b)) : a.N;
+  c.skip = c.n_blk * BN >= lim;
+  return c;
+}
+
+template <int BN, int STAGES, int EPI>
+__global__ void __launch_bounds__(kThreads, 1)
+gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, KArgs a) {
+  using S = Smem<BN, STAGES>;
+  constexpr uint32_t IDESC = idesc_bf16(kBM, BN);
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + STAGES * S::A_BYTES;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S::TILES);
+  uint64_t* empty = full + STAGES;
+  uint64_t* tfull = empty + STAGES;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* drain = tempty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
+    for (int i = 0; i < 2; ++i) { mbar_init(&tfull[i], 1); mbar_init(&tempty[i], 128); }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) { tma_prefetch_desc(&tmA); tma_prefetch_desc(&tmB); }
+  if (warp == 1) { tmem_alloc(tmem_slot, S::TMEM_COLS); tmem_relinquish(); }
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  const int m_tiles = (a.M + kBM - 1) / kBM;
+  const int n_tiles = (a.N + BN - 1) / BN;
+  const int total = a.batch * m_tiles * n_tiles;
+  const int KB = a.K / kBK;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------------------------------------------------------- TMA producer
+      uint32_t stage = 0, phase = 0;
+      int last_par[STAGES];
+#pragma unroll
+      for (int s = 0; s < STAGES; ++s) last_par[s] = -1;
+      bool ok = true;
+      for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+        TileCoord c = tile_coord(a, t, m_tiles, n_tiles, BN);
+        if (c.skip) continue;
+        const int arow = c.b * a.a_row_stride + c.m_blk * kBM;
+        const int brow = c.b * a.b_row_stride + c.n_blk * BN;
+        for (int kb = 0; kb < KB; ++kb) {
+          if (!mbar_wait(&empty[stage], phase ^ 1, a.status, abort_flag)) { ok = false; break; }
+          mbar_arrive_expect_tx(&full[stage], S::STAGE_BYTES);
+          tma_load_2d(sA + stage * S::A_BYTES, &tmA, &full[stage], kb * kBK, arow);
+          tma_load_2d(sB + stage * S::B_BYTES, &tmB, &full[stage], kb * kBK, brow);
+          last_par[stage] = static_cast<int>(phase);
+          if (++stage == STAGES) { stage = 0; phase ^= 1; }
+        }
+      }
+      if (!ok) {   // let every copy already in flight land before the CTA exits
+        for (int s = 0; s < STAGES; ++s)
+          if (last_par[s] >= 0) mbar_wait(&full[s], static_cast<uint32_t>(last_par[s]), a.status, nullptr);
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------------------------------------------------------- MMA issuer
+      uint32_t stage = 0, phase = 0, acc = 0, acc_phase = 0;
+      bool issued = false, ok = true;
+      for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+        TileCoord c = tile_coord(a, t, m_tiles, n_tiles, BN);
+        if (c.skip) continue;
+        if (!mbar_wait(&tempty[acc], acc_phase ^ 1, a.status, abort_flag)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * BN;
+        for (int kb = 0; kb < KB; ++kb) {
+          if (!mbar_wait(&full[stage], phase, a.status, abort_flag)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t a0 = smem_u32(sA + stage * S::A_BYTES);
+          const uint32_t b0 = smem_u32(sB + stage * S::B_BYTES);
+#pragma unroll
+          for (int k = 0; k < kBK / 16; ++k)
+            umma_bf16(d_tmem, desc_sw128(a0 + k * 32), desc_sw128(b0 + k * 32), IDESC, (kb | k) != 0);
+          umma_commit(&empty[stage]);
+          issued = true;
+          if (++stage == STAGES) { stage = 0; phase ^= 1; }
+        }
+        if (!ok) break;
+        umma_commit(&tfull[acc]);
+        acc ^= 1;
+        if (acc == 0) acc_phase ^= 1;
+      }
+      if (issued) {   // every MMA of this CTA has completed before TMEM is released
+        umma_commit(drain);
+        mbar_wait(drain, 0, a.status, nullptr);
+      }
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------------------------ epilogue
+    const int lane_grp = warp & 3;                 // TMEM lanes this warp may access
+    const int r_in_tile = lane_grp * 32 + lane;
+    uint32_t acc = 0, acc_phase = 0;
+    for (int t = blockIdx.x; t < total; t += gridDim.x) {
+      TileCoord c = tile_coord(a, t, m_tiles, n_tiles, BN);
+      if (c.skip) continue;
+      if (!mbar_wait(&tfull[acc], acc_phase, a.status, abort_flag)) break;
+      tc_fence_after();
+      const int row = c.m_blk * kBM + r_in_tile;
+      const bool row_ok = row < a.M;
+      const int lim = a.n_limit ? min(a.N, __ldg(a.n_limit + c.b)) : a.N;
+      const int col0 = c.n_blk * BN;
+      const uint32_t tbase = tmem_base + (static_cast<uint32_t>(lane_grp * 32) << 16) + acc * BN;
+      const long long crow = static_cast<long long>(c.b) * a.c_batch_stride + static_cast<long long>(row) * a.ldc;
+
+      if constexpr (EPI == EPI_ROPE_F32) {
+        // BN == dp: the whole row is in this tile; rotate pairs (i, i + dp/2).
+        constexpr int HALF = BN / 2;
+        float* out = reinterpret_cast<float*>(a.C) + crow;
+        int pos = 0;
+        if (row_ok) pos = a.pos ? __ldg(a.pos + row) : row % a.pos_mod;
+        const float2* rt = a.rope + static_cast<long long>(pos) * a.rope_half;
+#pragma unroll 1
+        for (int ch = 0; ch < HALF / 32; ++ch) {
+          uint32_t r1[32], r2[32];
+          tmem_ld32(tbase + ch * 32, r1);
+          tmem_ld32(tbase + HALF + ch * 32, r2);
+          if (row_ok) {
+#pragma unroll
+            for (int j = 0; j < 32; j += 4) {
+              float o1[4], o2[4];
+#pragma unroll
+              for (int u = 0; u < 4; ++u) {
+                const float2 cs = __ldg(rt + ch * 32 + j + u);
+                const float x1 = __uint_as_float(r1[j + u]), x2 = __uint_as_float(r2[j + u]);
+                o1[u] = x1 * cs.x - x2 * cs.y;
+                o2[u] = x2 * cs.x + x1 * cs.y;
+              }
+              *reinterpret_cast<float4*>(out + ch * 32 + j) = make_float4(o1[0], o1[1], o1[2], o1[3]);
+              *reinterpret_cast<float4*>(out + HALF + ch * 32 + j) = make_float4(o2[0], o2[1], o2[2], o2[3]);
+            }
+          }
+        }
+      } else if constexpr (EPI == EPI_F32) {
+        float* out = reinterpret_cast<float*>(a.C) + crow + col0;
+#pragma unroll 1
+        for (int ch = 0; ch < BN / 32; ++ch) {
+          uint32_t r[32];
+          tmem_ld32(tbase + ch * 32, r);
+          const int cbase = col0 + ch * 32;
+          if (row_ok && cbase < lim) {
+            if (cbase + 32 <= lim) {
+#pragma unroll
+              for (int j = 0; j < 32; j += 4)
+                *reinterpret_cast<float4*>(out + ch * 32 + j) =
+                    make_float4(__uint_as_float(r[j]), __uint_as_float(r[j + 1]), __uint_as_float(r[j + 2]),
+                                __uint_as_float(r[j + 3]));
+            } else {
+#pragma unroll
+              for (int j = 0; j < 32; ++j)
+                if (cbase + j < lim) out[ch * 32 + j] = __uint_as_float(r[j]);
+            }
+          }
+        }
+      } else {
+        __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(a.C) + crow + col0;
+#pragma unroll 1
+        for (int ch = 0; ch < BN / 32; ++ch) {
+          uint32_t r[32];
+          tmem_ld32(tbase + ch * 32, r);
+          const int cbase = col0 + ch * 32;
+          if (row_ok && cbase < lim) {
+            uint32_t pk[16];
+#pragma unroll
+            for (int j = 0; j < 32; j += 2) {
+              float x0 = __uint_as_float(r[j]), x1 = __uint_as_float(r[j + 1]);
+              if (a.bias) {
+                const __nv_bfloat162 bb = __ldg(reinterpret_cast<const __nv_bfloat162*>(a.bias + cbase + j));
+                x0 += __bfloat162float(bb.x);
+                x1 += __bfloat162float(bb.y);
+              }
+              if constexpr (EPI == EPI_GELU_BF16) { x0 = gelu_erf(x0); x1 = gelu_erf(x1); }
+              pk[j / 2] = pack_bf16(x0, x1);
+            }
+            uint4* o = reinterpret_cast<uint4*>(out + ch * 32);
+#pragma unroll
+            for (int v = 0; v < 4; ++v) o[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+          }
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(&tempty[acc]);
+      acc ^= 1;
+      if (acc == 0) acc_phase ^= 1;
+    }
+  }
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, S::TMEM_COLS);
+  }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+// 2D bf16 tensor map over [rows, K] (K contiguous), box 64 x box_rows, 128-byte swizzle.
+bool make_map(CUtensorMap* m, const void* base, long long rows, int K, int box_rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(K) * 2};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(kBK), static_cast<cuuint32_t>(box_rows)};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+template <int BN, int STAGES, int EPI>
+cudaError_t run(const GemmDesc& d, const KArgs& ka, int num_sms, cudaStream_t st) {
+  using S = Smem<BN, STAGES>;
+  CUtensorMap ta, tb;
+  if (!make_map(&ta, d.A, d.a_rows_total, d.K, kBM)) return cudaErrorInvalidValue;
+  if (!make_map(&tb, d.B, d.b_rows_total, d.K, BN)) return cudaErrorInvalidValue;
+  auto kern = gemm_tc_kernel<BN, STAGES, EPI>;
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, S::TOTAL);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  const int tiles = d.batch * ((d.M + kBM - 1) / kBM) * ((d.N + BN - 1) / BN);
+  if (tiles == 0) return cudaSuccess;
+  const int grid = std::max(1, std::min(tiles, num_sms));
+  kern<<<grid, kThreads, S::TOTAL, st>>>(ta, tb, ka);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t st) {
+  if (d.K <= 0 || d.K % kBK != 0 || d.M < 0 || d.N <= 0 || d.batch <= 0) return cudaErrorInvalidValue;
+  if ((reinterpret_cast<uintptr_t>(d.A) | reinterpret_cast<uintptr_t>(d.B)) & 15) return cudaErrorInvalidValue;
+  if (d.M == 0) return cudaSuccess;
+  KArgs ka;
+  ka.M = d.M; ka.N = d.N; ka.K = d.K; ka.batch = d.batch;
+  ka.a_row_stride = d.a_row_stride; ka.b_row_stride = d.b_row_stride;
+  ka.n_limit = d.n_limit; ka.C = d.C; ka.ldc = d.ldc; ka.c_batch_stride = d.c_batch_stride;
+  ka.bias = static_cast<const __nv_bfloat16*>(d.bias);
+  ka.rope = d.rope; ka.rope_half = d.rope_half; ka.pos = d.pos; ka.pos_mod = d.pos_mod > 0 ? d.pos_mod : 1;
+  ka.status = d.status;
+  switch (d.epi) {
+    case EPI_GELU_BF16:
+      if (d.N % 256 == 0) return run<256, 4, EPI_GELU_BF16>(d, ka, num_sms, st);
+      if (d.N % 64 == 0) return run<64, 8, EPI_GELU_BF16>(d, ka, num_sms, st);
+      return cudaErrorInvalidValue;
+    case EPI_BIAS_BF16:
+      if (d.N % 256 == 0) return run<256, 4, EPI_BIAS_BF16>(d, ka, num_sms, st);
+      if (d.N % 64 == 0) return run<64, 8, EPI_BIAS_BF16>(d, ka, num_sms, st);
+      return cudaErrorInvalidValue;
+    case EPI_ROPE_F32:
+      if (d.N == 64) return run<64, 8, EPI_ROPE_F32>(d, ka, num_sms, st);
+      if (d.N == 128) return run<128, 6, EPI_ROPE_F32>(d, ka, num_sms, st);
+      if (d.N == 256) return run<256, 4, EPI_ROPE_F32>(d, ka, num_sms, st);
+      return cudaErrorInvalidValue;
+    case EPI_F32:
+      return run<128, 6, EPI_F32>(d, ka, num_sms, st);
+    default:
+      return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace mapk

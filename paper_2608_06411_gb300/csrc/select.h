@@ -1,0 +1,43 @@
+// Selection state and launchers (internal to libmap_gb300); see select.cu.
+#pragma once
+#include <cstddef>
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace mapk {
+
+struct SelState {
+  int B, N, D, K, K0, S;          // S = active-set size (Gram block rows)
+  float lambda, tau;
+  const float* scores;            // [B, N] p_hat
+  const void* V;                  // [B, N, D] bf16
+  const float* sqn;               // [B, N] ||v||^2
+  float* U;                       // [B, N] value bound / exact value
+  float* r2;                      // [B, N] residual^2 as of cstep
+  int32_t* cstep;                 // [B, N] basis coordinates cached
+  uint8_t* state;                 // [B, N] 0 candidate, 1 retained
+  float* Ec;                      // [B, N, K] cached coordinates e_beta[i]
+  int32_t* picks;                 // [B, K] pick order
+  int32_t* r0;                    // [B, K] R0 in p_hat order (first K0 used)
+  int32_t* basis_tok;             // [B, K] token that added basis vector beta
+  float* rnorm;                   // [B, K] its residual norm at that time
+  int32_t* npicks; int32_t* nbasis; int32_t* nb_gathered; int32_t* done; int32_t* mode;
+  int32_t* nlimit;                // [B] Gram block columns (S + nbasis), 0 when done
+  uint64_t* theta;                // [B] key of the best candidate outside A (0: none)
+  int32_t* aslot;                 // [B, S] active tokens (-1 empty)
+  void* Vg;                       // [B, S + K, D] bf16 gathered rows
+  float* G;                       // [B, S, S + K] Gram block
+  int32_t* done_count;            // images finished
+  int* status;
+};
+
+size_t sel_init_smem(int N, int K0);
+size_t sel_choose_smem(int N);
+cudaError_t launch_sel_init(const SelState& s, cudaStream_t st);
+cudaError_t launch_sel_choose(const SelState& s, cudaStream_t st);
+cudaError_t launch_sel_greedy(const SelState& s, cudaStream_t st);
+cudaError_t launch_sel_finalize(const int32_t* picks, int B, int K, int32_t* keep, int32_t* order, cudaStream_t st);
+cudaError_t launch_sel_copy_r0(const int32_t* r0, int B, int K, int32_t* picks, cudaStream_t st);
+cudaError_t launch_sel_identity(int B, int N, int32_t* keep, int32_t* order, cudaStream_t st);
+
+}  // namespace mapk

@@ -1,0 +1,266 @@
+"""GPU parity: the CUDA path through the C ABI against the CPU oracle (and, for the
+GEMM building block, against a plain PyTorch fp32 reference).  Marked gpu."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import map_oracle as O
+from oracle import parity as P
+from paper_2608_06411_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+if not torch.cuda.is_available():
+    pytest.skip("needs a CUDA GPU", allow_module_level=True)
+
+from paper_2608_06411_gb300 import binding as mb  # noqa: E402
+
+DEV = torch.device("cuda:0")
+
+
+def dev_bits(a):
+    return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).to(DEV)
+
+
+def make_ctx(dims, seed=7, bias_std=0.0, **kw):
+    w = W.make_weights(dims, seed=seed, bias_std=bias_std)
+    return mb.Context({k: dev_bits(v) for k, v in w.items()}, dims.D, dims.Dh, dims.dp, **kw), w
+
+
+def run_select(ctx, p32, vis, K):
+    keep, order = ctx.select(torch.from_numpy(p32).to(DEV), dev_bits(vis), K)
+    torch.cuda.synchronize()
+    ctx.check()
+    return keep.cpu().numpy(), order.cpu().numpy()
+
+
+def assert_selection(p32, vis, K, K0, keep, order, lam=1.0, tau=1e-5):
+    for b in range(len(p32)):
+        rep = P.check_selection(p32[b].astype(np.float64), O.bf16_bits_to_f64(vis[b]), K, K0, order[b], keep[b],
+                                lam=lam, tau=tau)
+        assert rep["ok"], f"image {b}: {rep['reason']}"
+
+
+# ------------------------------------------------------------------ GEMM building block
+
+@pytest.mark.parametrize("M,K,N", [(300, 512, 512), (128, 256, 192), (1, 64, 64), (1000, 1024, 256)])
+@pytest.mark.parametrize("epi", [mb.EPI_GELU_BF16, mb.EPI_BIAS_BF16, mb.EPI_F32])
+def test_linear_matches_torch_fp32(M, K, N, epi):
+    ctx, _ = make_ctx(W.PredictorDims(D=256, Dh=256, dp=64))
+    g = torch.Generator(device="cpu").manual_seed(M * 7 + N)
+    x = torch.randn(M, K, generator=g).to(torch.bfloat16).to(DEV)
+    w = (torch.randn(N, K, generator=g) / K ** 0.5).to(torch.bfloat16).to(DEV)
+    b = torch.randn(N, generator=g).to(torch.bfloat16).to(DEV)
+    y = ctx.linear(x, w, b, epi)
+    torch.cuda.synchronize()
+    ctx.check()
+    ref = x.float() @ w.float().T
+    if epi != mb.EPI_F32:
+        ref = ref + b.float()
+    if epi == mb.EPI_GELU_BF16:
+        ref = torch.nn.functional.gelu(ref)
+    if epi == mb.EPI_F32:
+        err = (y - ref).abs().max().item()
+        assert err <= 1e-4 * ref.abs().max().item() + 1e-5
+    else:
+        # bf16 outputs: at most one bf16 rounding step from the fp32 reference
+        torch.testing.assert_close(y.float(), ref, rtol=2 ** -7, atol=1e-3)
+        exact = (y == ref.to(torch.bfloat16)).float().mean().item()
+        assert exact > 0.99
+
+
+# ------------------------------------------------------------------ Eq. 3 scores
+
+def test_scores_match_oracle_llava15_shape():
+    wl = W.WORKLOADS["c0"]
+    dims = W.PredictorDims()
+    ctx, w = make_ctx(dims)
+    vis = W.make_image(wl, 0)[None]
+    lens = np.array([32], np.int32)
+    text = W.make_text(wl, 0, 32)
+    p, q, k = ctx.score_debug(dev_bits(text), dev_bits(vis), lens)
+    torch.cuda.synchronize()
+    ctx.check()
+    q_ref = O.predict_queries(text, wl.N, w)
+    k_ref = O.predict_keys(vis[0], w)
+    assert np.linalg.norm(q.cpu().numpy() - q_ref) / np.linalg.norm(q_ref) < 2e-3
+    assert np.linalg.norm(k.cpu().numpy() - k_ref) / np.linalg.norm(k_ref) < 2e-3
+    p_ref = O.predicted_attention(q_ref, k_ref)
+    assert P.score_rel_err(p.cpu().numpy()[0], p_ref) <= 1e-3
+
+
+def test_scores_ragged_batch_with_biases():
+    dims = W.PredictorDims(D=512, Dh=256, dp=64)
+    ctx, w = make_ctx(dims, seed=3, bias_std=0.1)
+    wl = W.WORKLOADS["c1"]
+    B, N = 3, 300
+    lens = np.array([5, 130, 1], np.int32)
+    vis = np.stack([W.make_image(wl, b, N=N, D=dims.D) for b in range(B)])
+    text = np.concatenate([W.make_text(wl, b, int(lens[b]), D=dims.D) for b in range(B)])
+    p = ctx.score(dev_bits(text), dev_bits(vis), lens)
+    torch.cuda.synchronize()
+    ctx.check()
+    p_ref = O.map_score(text, vis, lens, w)
+    assert P.score_rel_err(p.cpu().numpy(), p_ref) <= 1e-3
+    np.testing.assert_allclose(p.cpu().numpy().sum(1), 1.0, atol=1e-5)
+
+
+def test_scores_without_rope_are_permutation_equivariant():
+    dims = W.PredictorDims(D=256, Dh=256, dp=128)
+    ctx, w = make_ctx(dims, rope_on=False)
+    wl = W.WORKLOADS["c0"]
+    vis = W.make_image(wl, 1, N=257, D=dims.D)
+    text = W.make_text(wl, 1, 7, D=dims.D)
+    perm = np.random.default_rng(0).permutation(257)
+    p1 = ctx.score(dev_bits(text), dev_bits(vis[None]), [7]).cpu().numpy()[0]
+    p2 = ctx.score(dev_bits(text), dev_bits(vis[perm][None]), [7]).cpu().numpy()[0]
+    ctx.check()
+    np.testing.assert_array_equal(p2, p1[perm])
+    p_ref = O.map_score(text, vis[None], [7], w, rope_on=False)[0]
+    assert P.score_rel_err(p1, p_ref) <= 1e-3
+
+
+# ------------------------------------------------------------------ Eq. 4 selection
+
+def _oracle_scores(vis, lens, text, w, **kw):
+    return O.map_score(text, vis, lens, w, **kw).astype(np.float32)
+
+
+def test_select_matches_oracle_llava15_shape():
+    wl = W.WORKLOADS["c0"]
+    dims = W.PredictorDims()
+    ctx, w = make_ctx(dims)
+    vis = W.make_image(wl, 0)[None]
+    text = W.make_text(wl, 0, 32)
+    p32 = _oracle_scores(vis, [32], text, w)
+    keep, order = run_select(ctx, p32, vis, wl.K)
+    assert_selection(p32, vis, wl.K, O.resolve_k0(wl.K), keep, order)
+
+
+@pytest.mark.parametrize("lam,k0_frac,K", [(1.0, 0.0, 40), (1.0, 0.25, 64), (0.5, 0.5, 50), (2.0, 0.5, 33),
+                                           (0.0, 0.5, 40), (1.0, 1.0, 40), (1.0, 0.5, 300), (1.0, 0.0, 200)])
+def test_select_variants(lam, k0_frac, K):
+    dims = W.PredictorDims(D=256, Dh=256, dp=64)
+    ctx, _ = make_ctx(dims, lam=lam, k0_frac=k0_frac)
+    wl = W.WORKLOADS["c1"]
+    rng = np.random.default_rng(int(K + 100 * lam))
+    B, N = 2, 700
+    vis = np.stack([W.make_image(wl, b, N=N, D=dims.D) for b in range(B)])
+    p32 = rng.dirichlet(np.full(N, 0.3), size=B).astype(np.float32)
+    keep, order = run_select(ctx, p32, vis, K)
+    assert_selection(p32, vis, K, O.resolve_k0(K, k0_frac), keep, order, lam=lam)
+
+
+def test_select_duplicates_and_near_duplicates():
+    dims = W.PredictorDims(D=256, Dh=256, dp=64)
+    ctx, _ = make_ctx(dims)
+    rng = np.random.default_rng(5)
+    N = 160
+    base = rng.standard_normal((20, 256)).astype(np.float32)
+    x = base[rng.integers(0, 20, N)]
+    x[::3] += 1e-3 * rng.standard_normal((len(x[::3]), 256)).astype(np.float32)   # near-duplicates
+    vis = W.f32_to_bf16_bits(x)[None]
+    p32 = rng.dirichlet(np.ones(N), size=1).astype(np.float32)
+    for K in (10, 40, 100):
+        keep, order = run_select(ctx, p32, vis, K)
+        assert_selection(p32, vis, K, O.resolve_k0(K), keep, order)
+
+
+def test_select_edge_sizes():
+    dims = W.PredictorDims(D=128, Dh=256, dp=64)
+    ctx, _ = make_ctx(dims)
+    wl = W.WORKLOADS["c0"]
+    N = 37
+    vis = W.make_image(wl, 2, N=N, D=dims.D)[None]
+    p32 = np.random.default_rng(1).dirichlet(np.ones(N), size=1).astype(np.float32)
+    keep, order = run_select(ctx, p32, vis, N)
+    assert keep.tolist() == [list(range(N))] and order.tolist() == [list(range(N))]
+    for K in (1, 2, 36):
+        keep, order = run_select(ctx, p32, vis, K)
+        assert_selection(p32, vis, K, O.resolve_k0(K), keep, order)
+    with pytest.raises(mb.MapError):
+        ctx.select(torch.from_numpy(p32).to(DEV), dev_bits(vis), N + 1)
+    k0, _ = ctx.select(torch.from_numpy(p32).to(DEV), dev_bits(vis), 0)
+    assert k0.shape == (1, 0)
+
+
+def test_select_batch_equals_single_images():
+    dims = W.PredictorDims(D=256, Dh=256, dp=64)
+    ctx, _ = make_ctx(dims)
+    wl = W.WORKLOADS["c3"]
+    B, N, K = 5, 500, 60
+    vis = np.stack([W.make_image(wl, b, N=N, D=dims.D) for b in range(B)])
+    p32 = np.random.default_rng(2).dirichlet(np.full(N, 0.5), size=B).astype(np.float32)
+    keep, order = run_select(ctx, p32, vis, K)
+    for b in range(B):
+        kb, ob = run_select(ctx, p32[b:b + 1], vis[b:b + 1], K)
+        np.testing.assert_array_equal(ob[0], order[b])
+        np.testing.assert_array_equal(kb[0], keep[b])
+
+
+# ------------------------------------------------------------------ gather and the whole path
+
+def test_gather_is_bit_exact():
+    dims = W.PredictorDims(D=512, Dh=256, dp=64)
+    ctx, _ = make_ctx(dims)
+    rng = np.random.default_rng(3)
+    vis = rng.integers(0, 2 ** 16, size=(3, 90, 512), dtype=np.uint16)
+    keep = np.sort(np.stack([rng.choice(90, 17, replace=False) for _ in range(3)]), 1).astype(np.int32)
+    out = ctx.gather(dev_bits(vis), torch.from_numpy(keep).to(DEV))
+    torch.cuda.synchronize()
+    ctx.check()
+    np.testing.assert_array_equal(out.cpu().numpy().view(np.uint16), O.gather(vis, keep))
+
+
+def test_gather_rejects_bad_index_without_faulting():
+    dims = W.PredictorDims(D=512, Dh=256, dp=64)
+    ctx, _ = make_ctx(dims)
+    vis = torch.zeros((1, 10, 512), dtype=torch.int16, device=DEV)
+    keep = torch.tensor([[0, 12]], dtype=torch.int32, device=DEV)
+    ctx.gather(vis, keep)
+    assert ctx.status() == mb.MAP_EINTERNAL
+    assert ctx.status() == mb.MAP_OK
+
+
+def test_prune_host_buffers_equal_device_path():
+    dims = W.PredictorDims(D=512, Dh=256, dp=64)
+    ctx, w = make_ctx(dims)
+    wl = W.WORKLOADS["c1"]
+    B, N, K = 2, 400, 30
+    lens = np.array([12, 40], np.int32)
+    vis = np.stack([W.make_image(wl, b, N=N, D=dims.D) for b in range(B)])
+    text = np.concatenate([W.make_text(wl, b, int(lens[b]), D=dims.D) for b in range(B)])
+    out_h = np.zeros((B, K, dims.D), np.uint16)
+    keep_h = np.zeros((B, K), np.int32)
+    sc_h = np.zeros((B, N), np.float32)
+    ctx.prune(text, vis, lens, K, out_h, keep_h, sc_h)
+    sc = ctx.score(dev_bits(text), dev_bits(vis), lens)
+    keep, _ = ctx.select(sc, dev_bits(vis), K)
+    out = ctx.gather(dev_bits(vis), keep)
+    torch.cuda.synchronize()
+    ctx.check()
+    np.testing.assert_array_equal(sc_h, sc.cpu().numpy())
+    np.testing.assert_array_equal(keep_h, keep.cpu().numpy())
+    np.testing.assert_array_equal(out_h, out.cpu().numpy().view(np.uint16))
+    assert P.score_rel_err(sc_h, O.map_score(text, vis, lens, w)) <= 1e-3
+
+
+def test_llava_next_shape_end_to_end():
+    """N = 2880, K = 160 (c1): scores against the oracle, then selection parity on the
+    oracle's scores, then the gathered tokens bit for bit."""
+    wl = W.WORKLOADS["c1"]
+    dims = W.PredictorDims()
+    ctx, w = make_ctx(dims)
+    vis = W.make_image(wl, 0)[None]
+    text = W.make_text(wl, 0, wl.m_lo)
+    p = ctx.score(dev_bits(text), dev_bits(vis), [wl.m_lo])
+    torch.cuda.synchronize()
+    ctx.check()
+    p_ref = O.map_score(text, vis, [wl.m_lo], w)
+    assert P.score_rel_err(p.cpu().numpy(), p_ref) <= 1e-3
+    p32 = p_ref.astype(np.float32)
+    keep, order = run_select(ctx, p32, vis, wl.K)
+    assert_selection(p32, vis, wl.K, O.resolve_k0(wl.K), keep, order)
+    out = ctx.gather(dev_bits(vis), torch.from_numpy(keep).to(DEV))
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(out.cpu().numpy().view(np.uint16), O.gather(vis, keep))
