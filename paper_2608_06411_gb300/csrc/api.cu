@@ -194,23 +194,30 @@ GemmDesc linear_desc(map_ctx* c, const void* x, long long rows, int K, const voi
 }
 
 // Predictor for one modality: x [rows, D] -> RoPE(W f(x)) [rows, dp] fp32.
+// The hidden activations h1, h2 are kept as bf16 hi/lo pairs [rows, 2 Dh] (about 16
+// significant bits), and the layers after them run with K = 2 Dh against [W | W].
 int predictor_branch(map_ctx* c, const void* x, long long rows, const void* w1, const void* b1, const void* w2,
                      const void* b2, const void* wp, DevBuf& h1, DevBuf& h2, float* out, const int* pos, int pos_mod,
                      cudaStream_t st, int tid_l1, int tid_l2, int tid_p) {
   const map_config& g = c->cfg;
-  MAP_TRY(ensure(h1, static_cast<size_t>(rows) * g.Dh * 2));
-  MAP_TRY(ensure(h2, static_cast<size_t>(rows) * g.Dh * 2));
+  MAP_TRY(ensure(h1, static_cast<size_t>(rows) * g.Dh * 4));
+  MAP_TRY(ensure(h2, static_cast<size_t>(rows) * g.Dh * 4));
   {
     Timed t(c, st, tid_l1);
-    MAP_TRY(gemm(c, linear_desc(c, x, rows, g.D, w1, g.Dh, b1, h1.p, mapk::EPI_GELU_BF16), st));
+    GemmDesc d = linear_desc(c, x, rows, g.D, w1, g.Dh, b1, h1.p, mapk::EPI_GELU_SPLIT);
+    d.ldc = 2LL * g.Dh;
+    MAP_TRY(gemm(c, d, st));
   }
   {
     Timed t(c, st, tid_l2);
-    MAP_TRY(gemm(c, linear_desc(c, h1.p, rows, g.Dh, w2, g.Dh, b2, h2.p, mapk::EPI_BIAS_BF16), st));
+    GemmDesc d = linear_desc(c, h1.p, rows, 2 * g.Dh, w2, g.Dh, b2, h2.p, mapk::EPI_BIAS_SPLIT);
+    d.ldc = 2LL * g.Dh;
+    MAP_TRY(gemm(c, d, st));
   }
   {
     Timed t(c, st, tid_p);
-    GemmDesc d = linear_desc(c, h2.p, rows, g.Dh, wp, g.dp, nullptr, out, g.rope_on ? mapk::EPI_ROPE_F32 : mapk::EPI_F32);
+    GemmDesc d = linear_desc(c, h2.p, rows, 2 * g.Dh, wp, g.dp, nullptr, out,
+                             g.rope_on ? mapk::EPI_ROPE_F32 : mapk::EPI_F32);
     d.rope = static_cast<const float2*>(c->rope.p);
     d.pos = pos;
     d.pos_mod = pos_mod;
@@ -306,10 +313,10 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, 
   int K0 = resolve_k0(g, K);
   if (g.lambda == 0.f) K0 = K;        // values are p_hat alone: plain top-K
   const long long BN = static_cast<long long>(B) * N;
-  const int S = kSelS, R = kSelS + K;
+  const int S = kSelS, R = ((kSelS + K + 15) / 16) * 16;   // row stride of Vg and G (16-byte rows)
 
   mapk::SelState s{};
-  s.B = B; s.N = N; s.D = g.D; s.K = K; s.K0 = K0; s.S = S;
+  s.B = B; s.N = N; s.D = g.D; s.K = K; s.K0 = K0; s.S = S; s.R = R;
   s.lambda = g.lambda; s.tau = g.tau;
   s.scores = scores; s.V = vis; s.status = c->status;
   // per-token arrays
@@ -446,11 +453,19 @@ int map_init(const map_config* cfg, const map_weights* w, map_ctx** out) {
   do {
     if (cudaGetDevice(&c->device) != cudaSuccess) { rc = MAP_ECUDA; break; }
     if (cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, c->device) != cudaSuccess) { rc = MAP_ECUDA; break; }
+    // Layers fed by a hi/lo activation pair (f_T, f_V layer 2, W_Q, W_K) are stored as
+    // [W | W] ([out, 2 * in]); the others as given.
     const size_t D = cfg->D, Dh = cfg->Dh, dp = cfg->dp;
-    const size_t n[10] = {Dh * D, Dh, Dh * Dh, Dh, dp * Dh, Dh * D, Dh, Dh * Dh, Dh, dp * Dh};
+    const size_t rows[10] = {Dh, 1, Dh, 1, dp, Dh, 1, Dh, 1, dp};
+    const size_t cols[10] = {D, Dh, Dh, Dh, Dh, D, Dh, Dh, Dh, Dh};
+    const bool dup[10] = {false, false, true, false, true, false, false, true, false, true};
     for (int i = 0; i < 10 && rc == MAP_OK; ++i) {
-      if (cudaMalloc(&c->w[i], n[i] * 2) != cudaSuccess) { rc = MAP_ENOMEM; break; }
-      if (cudaMemcpy(c->w[i], src[i], n[i] * 2, cudaMemcpyDefault) != cudaSuccess) rc = MAP_ECUDA;
+      const size_t pitch = cols[i] * 2 * (dup[i] ? 2 : 1);
+      if (cudaMalloc(&c->w[i], rows[i] * pitch) != cudaSuccess) { rc = MAP_ENOMEM; break; }
+      for (int h = 0; h < (dup[i] ? 2 : 1) && rc == MAP_OK; ++h)
+        if (cudaMemcpy2D(static_cast<char*>(c->w[i]) + h * cols[i] * 2, pitch, src[i], cols[i] * 2, cols[i] * 2,
+                         rows[i], cudaMemcpyDefault) != cudaSuccess)
+          rc = MAP_ECUDA;
     }
     if (rc != MAP_OK) break;
     if (cudaMalloc(&c->status, sizeof(int)) != cudaSuccess) { rc = MAP_ENOMEM; break; }

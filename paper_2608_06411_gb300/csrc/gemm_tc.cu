@@ -11,7 +11,8 @@
 //   warp 1      allocates TMEM (2 accumulators x BN fp32 columns); one thread issues
 //               tcgen05.mma (M=128, N=BN, K=16) x 4 per stage and commits to mbarriers.
 //   warps 2-5   epilogue: tcgen05.ld the accumulator (one TMEM lane = one output row per
-//               thread), apply bias / GELU / RoPE, store; release the accumulator so the
+//               thread), apply bias / GELU / RoPE, store (bf16, bf16 hi/lo pair, or fp32);
+//               release the accumulator so the
 //               MMA warp can start the tile after next while this one drains.
 // All waits are bounded (ptx.cuh); a timeout sets ST_TIMEOUT and every role drains and exits.
 #include <algorithm>
@@ -245,7 +246,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           tmem_ld32(tbase + ch * 32, r);
           const int cbase = col0 + ch * 32;
           if (row_ok && cbase < lim) {
-            uint32_t pk[16];
+            constexpr bool SPLIT = EPI == EPI_GELU_SPLIT || EPI == EPI_BIAS_SPLIT;
+            uint32_t pk[16], pl[16];
 #pragma unroll
             for (int j = 0; j < 32; j += 2) {
               float x0 = __uint_as_float(r[j]), x1 = __uint_as_float(r[j + 1]);
@@ -254,12 +256,19 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
                 x0 += __bfloat162float(bb.x);
                 x1 += __bfloat162float(bb.y);
               }
-              if constexpr (EPI == EPI_GELU_BF16) { x0 = gelu_erf(x0); x1 = gelu_erf(x1); }
-              pk[j / 2] = pack_bf16(x0, x1);
+              if constexpr (EPI == EPI_GELU_BF16 || EPI == EPI_GELU_SPLIT) { x0 = gelu_erf(x0); x1 = gelu_erf(x1); }
+              const __nv_bfloat162 hi = __floats2bfloat162_rn(x0, x1);
+              pk[j / 2] = *reinterpret_cast<const uint32_t*>(&hi);
+              if constexpr (SPLIT) pl[j / 2] = pack_bf16(x0 - __bfloat162float(hi.x), x1 - __bfloat162float(hi.y));
             }
             uint4* o = reinterpret_cast<uint4*>(out + ch * 32);
 #pragma unroll
             for (int v = 0; v < 4; ++v) o[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+            if constexpr (SPLIT) {
+              uint4* ol = reinterpret_cast<uint4*>(out + a.N + ch * 32);
+#pragma unroll
+              for (int v = 0; v < 4; ++v) ol[v] = make_uint4(pl[4 * v], pl[4 * v + 1], pl[4 * v + 2], pl[4 * v + 3]);
+            }
           }
         }
       }
@@ -329,6 +338,11 @@ cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t st) {
   if (d.K <= 0 || d.K % kBK != 0 || d.M < 0 || d.N <= 0 || d.batch <= 0) return cudaErrorInvalidValue;
   if ((reinterpret_cast<uintptr_t>(d.A) | reinterpret_cast<uintptr_t>(d.B)) & 15) return cudaErrorInvalidValue;
   if (d.M == 0) return cudaSuccess;
+  // every output row and column block is written with 16-byte vector stores
+  const bool f32 = d.epi == EPI_F32 || d.epi == EPI_ROPE_F32;
+  const long long vec = f32 ? 4 : 8;
+  if (d.ldc % vec != 0 || d.c_batch_stride % vec != 0 || (reinterpret_cast<uintptr_t>(d.C) & 15)) return cudaErrorInvalidValue;
+  if ((d.epi == EPI_GELU_SPLIT || d.epi == EPI_BIAS_SPLIT) && d.ldc < 2LL * d.N) return cudaErrorInvalidValue;
   KArgs ka;
   ka.M = d.M; ka.N = d.N; ka.K = d.K; ka.batch = d.batch;
   ka.a_row_stride = d.a_row_stride; ka.b_row_stride = d.b_row_stride;
@@ -349,6 +363,14 @@ cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t st) {
       if (d.N == 64) return run<64, 8, EPI_ROPE_F32>(d, ka, num_sms, st);
       if (d.N == 128) return run<128, 6, EPI_ROPE_F32>(d, ka, num_sms, st);
       if (d.N == 256) return run<256, 4, EPI_ROPE_F32>(d, ka, num_sms, st);
+      return cudaErrorInvalidValue;
+    case EPI_GELU_SPLIT:
+      if (d.N % 256 == 0) return run<256, 4, EPI_GELU_SPLIT>(d, ka, num_sms, st);
+      if (d.N % 64 == 0) return run<64, 8, EPI_GELU_SPLIT>(d, ka, num_sms, st);
+      return cudaErrorInvalidValue;
+    case EPI_BIAS_SPLIT:
+      if (d.N % 256 == 0) return run<256, 4, EPI_BIAS_SPLIT>(d, ka, num_sms, st);
+      if (d.N % 64 == 0) return run<64, 8, EPI_BIAS_SPLIT>(d, ka, num_sms, st);
       return cudaErrorInvalidValue;
     case EPI_F32:
       return run<128, 6, EPI_F32>(d, ka, num_sms, st);

@@ -5,7 +5,11 @@
 
 namespace mapk {
 
-enum Epi { EPI_GELU_BF16 = 0, EPI_BIAS_BF16 = 1, EPI_ROPE_F32 = 2, EPI_F32 = 3 };
+// *_SPLIT epilogues store an fp32 activation x as two bf16 halves, hi = bf16(x) at
+// column c and lo = bf16(x - hi) at column N + c of a [rows, 2N] buffer, so that the next
+// layer can consume ~16 significant bits through a bf16 GEMM: [hi | lo] @ [W | W]^T.
+enum Epi { EPI_GELU_BF16 = 0, EPI_BIAS_BF16 = 1, EPI_ROPE_F32 = 2, EPI_F32 = 3, EPI_GELU_SPLIT = 4,
+           EPI_BIAS_SPLIT = 5 };
 
 // Batched C = epi(A @ B^T): A rows [batch][a_row_stride] x K, B rows [batch][b_row_stride] x K
 // (both bf16, K contiguous, tightly packed 2D arrays of a_rows_total / b_rows_total rows).

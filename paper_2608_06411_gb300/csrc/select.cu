@@ -165,7 +165,7 @@ __global__ void sel_choose_kernel(SelState s) {
   __shared__ uint64_t sh_theta;
   const int b = blockIdx.x;
   const long long base = static_cast<long long>(b) * s.N;
-  const int S = s.S, R = s.S + s.K;          // rows per image in Vg
+  const int S = s.S, R = s.R;                // rows per image in Vg
   int32_t* aslot = s.aslot + static_cast<long long>(b) * S;
   if (s.done[b]) {
     if (threadIdx.x == 0) s.nlimit[b] = 0;
@@ -238,7 +238,7 @@ __global__ void sel_greedy_kernel(SelState s) {
   __shared__ float sh_r2;
   const int b = blockIdx.x;
   if (s.done[b]) return;
-  const int S = s.S, R = s.S + s.K;
+  const int S = s.S, R = s.R;
   const long long base = static_cast<long long>(b) * s.N;
   const int slot = threadIdx.x;
   const int tok = s.aslot[static_cast<long long>(b) * S + slot];

@@ -8,6 +8,7 @@ namespace mapk {
 
 struct SelState {
   int B, N, D, K, K0, S;          // S = active-set size (Gram block rows)
+  int R;                          // rows per image in Vg = row stride of G (>= S + K, multiple of 16)
   float lambda, tau;
   const float* scores;            // [B, N] p_hat
   const void* V;                  // [B, N, D] bf16
@@ -25,8 +26,8 @@ struct SelState {
   int32_t* nlimit;                // [B] Gram block columns (S + nbasis), 0 when done
   uint64_t* theta;                // [B] key of the best candidate outside A (0: none)
   int32_t* aslot;                 // [B, S] active tokens (-1 empty)
-  void* Vg;                       // [B, S + K, D] bf16 gathered rows
-  float* G;                       // [B, S, S + K] Gram block
+  void* Vg;                       // [B, R, D] bf16 gathered rows
+  float* G;                       // [B, S, R] Gram block
   int32_t* done_count;            // images finished
   int* status;
 };

@@ -115,7 +115,8 @@ def test_scores_without_rope_are_permutation_equivariant():
     p1 = ctx.score(dev_bits(text), dev_bits(vis[None]), [7]).cpu().numpy()[0]
     p2 = ctx.score(dev_bits(text), dev_bits(vis[perm][None]), [7]).cpu().numpy()[0]
     ctx.check()
-    np.testing.assert_array_equal(p2, p1[perm])
+    # each token's key is computed alone; only the softmax sums see a different order
+    np.testing.assert_allclose(p2, p1[perm], rtol=1e-6)
     p_ref = O.map_score(text, vis[None], [7], w, rope_on=False)[0]
     assert P.score_rel_err(p1, p_ref) <= 1e-3
 
