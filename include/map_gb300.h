@@ -112,7 +112,8 @@ int map_score(map_ctx *ctx, const void *text_feats, const void *vis_feats,
  *   pick_order  int32 [B, k] output (device) or NULL: the same tokens in the order they
  *               were retained (R0 in p_hat order first).
  * k == N keeps every token (keep_idx = pick_order = 0..N-1); k == 0 is a no-op;
- * k > N is MAP_EINVAL.  Supported: k <= 4096, N <= 16384 (MAP_EUNSUPPORTED beyond).
+ * k > N is MAP_EINVAL.  Supported: N <= 16384; k <= 4096 for plain top-k (lambda = 0 or
+ * K0 = k), k <= 1024 with the diversity term (MAP_EUNSUPPORTED beyond).
  * Runs a few selection rounds per host synchronisation: the call returns after the
  * selection has finished on the device (the final gather of indices is still queued).
  */

@@ -16,7 +16,8 @@ using mapk::GemmDesc;
 
 namespace {
 
-constexpr int kSelS = 128;          // active-set size of the selection (Gram block rows)
+constexpr int kSelS = 256;          // active-set size of the selection (Gram block rows)
+constexpr int kMaxKDiverse = 1024;  // k limit when the diversity term is on (shared-memory staging)
 constexpr int kMaxK = 4096;
 constexpr int kMaxN = 16384;
 
@@ -312,11 +313,13 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, 
   const map_config& g = c->cfg;
   int K0 = resolve_k0(g, K);
   if (g.lambda == 0.f) K0 = K;        // values are p_hat alone: plain top-K
+  if (K0 < K && K > kMaxKDiverse) return MAP_EUNSUPPORTED;
   const long long BN = static_cast<long long>(B) * N;
   const int S = kSelS, R = ((kSelS + K + 15) / 16) * 16;   // row stride of Vg and G (16-byte rows)
 
   mapk::SelState s{};
-  s.B = B; s.N = N; s.D = g.D; s.K = K; s.K0 = K0; s.S = S; s.R = R;
+  const int KP = ((K + 3) / 4) * 4;
+  s.B = B; s.N = N; s.D = g.D; s.K = K; s.K0 = K0; s.S = S; s.R = R; s.KP = KP;
   s.lambda = g.lambda; s.tau = g.tau;
   s.scores = scores; s.V = vis; s.status = c->status;
   // per-token arrays
@@ -329,7 +332,7 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, 
   MAP_TRY(ensure(c->sr0, static_cast<size_t>(B) * K * 4));
   MAP_TRY(ensure(c->sbt, static_cast<size_t>(B) * K * 4));
   MAP_TRY(ensure(c->srn, static_cast<size_t>(B) * K * 4));
-  MAP_TRY(ensure(c->ssmall, static_cast<size_t>(B) * 8 * 256 + 256));
+  MAP_TRY(ensure(c->ssmall, static_cast<size_t>(B) * 4 * 16 + 16 * 256));
   MAP_TRY(ensure(c->stheta, static_cast<size_t>(B) * 8));
   MAP_TRY(ensure(c->saslot, static_cast<size_t>(B) * S * 4));
   s.sqn = static_cast<float*>(c->sqn.p);
@@ -348,6 +351,8 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, 
   s.done = carve<int32_t>(sm, B);
   s.mode = carve<int32_t>(sm, B);
   s.nlimit = carve<int32_t>(sm, B);
+  s.gb_lo = carve<int32_t>(sm, B);
+  s.gb_hi = carve<int32_t>(sm, B);
   s.done_count = carve<int32_t>(sm, 1);
   s.theta = static_cast<uint64_t*>(c->stheta.p);
   s.aslot = static_cast<int32_t*>(c->saslot.p);
@@ -361,7 +366,7 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, 
   ++c->counters.launches;
   CU_TRY(mapk::launch_sel_init(s, st));
   if (K0 < K) {
-    MAP_TRY(ensure(c->sEc, static_cast<size_t>(BN) * K * 4));
+    MAP_TRY(ensure(c->sEc, static_cast<size_t>(BN) * KP * 4));
     MAP_TRY(ensure(c->sVg, static_cast<size_t>(B) * R * g.D * 2));
     MAP_TRY(ensure(c->sG, static_cast<size_t>(B) * S * R * 4));
     s.Ec = static_cast<float*>(c->sEc.p);
@@ -376,10 +381,10 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, 
     d.epi = mapk::EPI_F32; d.status = c->status;
     const long long cap = 8LL * (K + N / S) + 64;
     long long rounds = 0;
-    int burst = (K0 + S - 1) / S + 2;
+    int burst = (K0 + S - 1) / S + 6;   // rounds queued per host check; finished images skip
     for (;;) {
       for (int r = 0; r < burst; ++r) {
-        c->counters.launches += 2;
+        c->counters.launches += 3;
         CU_TRY(mapk::launch_sel_choose(s, st));
         MAP_TRY(gemm(c, d, st));
         CU_TRY(mapk::launch_sel_greedy(s, st));

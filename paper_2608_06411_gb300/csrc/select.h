@@ -9,6 +9,7 @@ namespace mapk {
 struct SelState {
   int B, N, D, K, K0, S;          // S = active-set size (Gram block rows)
   int R;                          // rows per image in Vg = row stride of G (>= S + K, multiple of 16)
+  int KP;                         // row stride of Ec (>= K, multiple of 4)
   float lambda, tau;
   const float* scores;            // [B, N] p_hat
   const void* V;                  // [B, N, D] bf16
@@ -17,13 +18,14 @@ struct SelState {
   float* r2;                      // [B, N] residual^2 as of cstep
   int32_t* cstep;                 // [B, N] basis coordinates cached
   uint8_t* state;                 // [B, N] 0 candidate, 1 retained
-  float* Ec;                      // [B, N, K] cached coordinates e_beta[i]
+  float* Ec;                      // [B, N, KP] cached coordinates e_beta[i]
   int32_t* picks;                 // [B, K] pick order
   int32_t* r0;                    // [B, K] R0 in p_hat order (first K0 used)
   int32_t* basis_tok;             // [B, K] token that added basis vector beta
   float* rnorm;                   // [B, K] its residual norm at that time
   int32_t* npicks; int32_t* nbasis; int32_t* nb_gathered; int32_t* done; int32_t* mode;
   int32_t* nlimit;                // [B] Gram block columns (S + nbasis), 0 when done
+  int32_t* gb_lo; int32_t* gb_hi;  // [B] basis rows to gather this round
   uint64_t* theta;                // [B] key of the best candidate outside A (0: none)
   int32_t* aslot;                 // [B, S] active tokens (-1 empty)
   void* Vg;                       // [B, R, D] bf16 gathered rows
@@ -34,6 +36,7 @@ struct SelState {
 
 size_t sel_init_smem(int N, int K0);
 size_t sel_choose_smem(int N);
+size_t sel_greedy_smem(int KP, int S, bool* smem_coords);
 cudaError_t launch_sel_init(const SelState& s, cudaStream_t st);
 cudaError_t launch_sel_choose(const SelState& s, cudaStream_t st);
 cudaError_t launch_sel_greedy(const SelState& s, cudaStream_t st);
