@@ -35,7 +35,7 @@ struct map_ctx {
   int device = 0, num_sms = 148;
   void* w[10] = {};                 // wT1 bT1 wT2 bT2 wQ wV1 bV1 wV2 bV2 wK (device bf16)
   DevBuf rope;  int rope_rows = 0;
-  DevBuf h1, h2, kb, th1, th2, qb, stats, qoff, post, sqn;
+  DevBuf h1, h2, kb, th1, th2, qb, stats, qoff, post, sqn, pmean;
   // selection
   DevBuf sU, sr2, scstep, sstate, sEc, spicks, sr0, sbt, srn, ssmall, stheta, saslot, sVg, sG;
   // map_prune staging
@@ -194,12 +194,14 @@ GemmDesc linear_desc(map_ctx* c, const void* x, long long rows, int K, const voi
   return d;
 }
 
-// Predictor for one modality: x [rows, D] -> RoPE(W f(x)) [rows, dp] fp32.
-// The hidden activations h1, h2 are kept as bf16 hi/lo pairs [rows, 2 Dh] (about 16
-// significant bits), and the layers after them run with K = 2 Dh against [W | W].
+// Predictor for one modality: x [rows, D] -> RoPE(W f(x)) * scale [rows, dp], stored as
+// three bf16 segments [rows, 3 dp] (split_kind 0: hi|lo|hi, 1: hi|hi|lo) and, if aux is
+// given, as fp32 too.  The hidden activations h1, h2 are kept as bf16 hi/lo pairs
+// [rows, 2 Dh] (about 16 significant bits), and the layers after them run with K = 2 Dh
+// against [W | W].
 int predictor_branch(map_ctx* c, const void* x, long long rows, const void* w1, const void* b1, const void* w2,
-                     const void* b2, const void* wp, DevBuf& h1, DevBuf& h2, float* out, const int* pos, int pos_mod,
-                     cudaStream_t st, int tid_l1, int tid_l2, int tid_p) {
+                     const void* b2, const void* wp, DevBuf& h1, DevBuf& h2, void* out3, int split_kind, float scale,
+                     float* aux, const int* pos, int pos_mod, cudaStream_t st, int tid_l1, int tid_l2, int tid_p) {
   const map_config& g = c->cfg;
   MAP_TRY(ensure(h1, static_cast<size_t>(rows) * g.Dh * 4));
   MAP_TRY(ensure(h2, static_cast<size_t>(rows) * g.Dh * 4));
@@ -217,11 +219,14 @@ int predictor_branch(map_ctx* c, const void* x, long long rows, const void* w1, 
   }
   {
     Timed t(c, st, tid_p);
-    GemmDesc d = linear_desc(c, h2.p, rows, 2 * g.Dh, wp, g.dp, nullptr, out,
-                             g.rope_on ? mapk::EPI_ROPE_F32 : mapk::EPI_F32);
+    GemmDesc d = linear_desc(c, h2.p, rows, 2 * g.Dh, wp, g.dp, nullptr, out3, mapk::EPI_ROPE_SPLIT3);
+    d.ldc = 3LL * g.dp;
     d.rope = static_cast<const float2*>(c->rope.p);
-    d.pos = pos;
-    d.pos_mod = pos_mod;
+    d.pos = g.rope_on ? pos : nullptr;      // without RoPE every position is 0: cos 1, sin 0
+    d.pos_mod = g.rope_on ? pos_mod : 1;
+    d.split_kind = split_kind;
+    d.scale = scale;
+    d.aux = aux;
     MAP_TRY(gemm(c, d, st));
   }
   return MAP_OK;
@@ -242,49 +247,72 @@ int score_impl(map_ctx* c, const void* text, const void* vis, const int32_t* len
   if (total_m > (1ll << 30) || static_cast<long long>(B) * N > (1ll << 30)) return MAP_EUNSUPPORTED;
   const map_config& g = c->cfg;
   CU_TRY(cudaSetDevice(c->device));
-  if (g.rope_on) MAP_TRY(ensure_rope(c, N + max_m + 1));
-  // per-image query offsets and question-token positions N + m
-  const size_t off_bytes = static_cast<size_t>(B + 1) * 4, pos_bytes = static_cast<size_t>(total_m) * 4;
+  MAP_TRY(ensure_rope(c, g.rope_on ? N + max_m + 1 : 1));
+  // per-image query offsets, lengths and question-token positions N + m
+  const size_t off_bytes = static_cast<size_t>(B + 1) * 4, len_bytes = static_cast<size_t>(B) * 4;
+  const size_t pos_bytes = static_cast<size_t>(total_m) * 4;
   void* hs = nullptr;
-  MAP_TRY(stage_host(c, off_bytes + pos_bytes, &hs));
+  MAP_TRY(stage_host(c, off_bytes + len_bytes + pos_bytes, &hs));
   int32_t* hoff = static_cast<int32_t*>(hs);
-  int32_t* hpos = hoff + (B + 1);
+  int32_t* hlen = hoff + (B + 1);
+  int32_t* hpos = hlen + B;
   hoff[0] = 0;
   for (int b = 0; b < B; ++b) {
     hoff[b + 1] = hoff[b] + lens[b];
+    hlen[b] = lens[b];
     for (int m = 0; m < lens[b]; ++m) hpos[hoff[b] + m] = N + m;
   }
-  MAP_TRY(ensure(c->qoff, off_bytes));
+  MAP_TRY(ensure(c->qoff, off_bytes + len_bytes));
   MAP_TRY(ensure(c->post, pos_bytes));
-  CU_TRY(cudaMemcpyAsync(c->qoff.p, hoff, off_bytes, cudaMemcpyHostToDevice, st));
+  CU_TRY(cudaMemcpyAsync(c->qoff.p, hoff, off_bytes + len_bytes, cudaMemcpyHostToDevice, st));
   CU_TRY(cudaMemcpyAsync(c->post.p, hpos, pos_bytes, cudaMemcpyHostToDevice, st));
   CU_TRY(cudaEventRecord(c->stage_ev, st));
   c->stage_pending = true;
+  const int* d_off = static_cast<const int*>(c->qoff.p);
+  const int* d_len = d_off + (B + 1);
 
   const long long vrows = static_cast<long long>(B) * N;
-  MAP_TRY(ensure(c->kb, static_cast<size_t>(vrows) * g.dp * 4));
-  MAP_TRY(ensure(c->qb, static_cast<size_t>(total_m) * g.dp * 4));
-  MAP_TRY(predictor_branch(c, vis, vrows, c->w[5], c->w[6], c->w[7], c->w[8], c->w[9], c->h1, c->h2,
-                           static_cast<float*>(c->kb.p), nullptr, N, st, MAP_K_GEMM_FV1, MAP_K_GEMM_FV2, MAP_K_GEMM_WK));
-  MAP_TRY(predictor_branch(c, text, total_m, c->w[0], c->w[1], c->w[2], c->w[3], c->w[4], c->th1, c->th2,
-                           static_cast<float*>(c->qb.p), static_cast<const int*>(c->post.p), 1, st, MAP_K_GEMM_TEXT,
-                           MAP_K_GEMM_TEXT, MAP_K_GEMM_TEXT));
-  // Eq. 3: split the keys so that the statistics pass fills the GPU
-  int nsplit = 1;
-  const long long mblocks = static_cast<long long>(B) * ((max_m + 127) / 128);
-  while (nsplit < 64 && mblocks * nsplit < 4LL * c->num_sms && N / (nsplit * 2) >= 64) nsplit *= 2;
-  MAP_TRY(ensure(c->stats, static_cast<size_t>(total_m) * nsplit * 8));
-  mapk::ScoreDesc sd{};
-  sd.q = static_cast<const float*>(c->qb.p); sd.k = static_cast<const float*>(c->kb.p);
-  sd.q_off = static_cast<const int*>(c->qoff.p); sd.B = B; sd.N = N; sd.dp = g.dp; sd.max_m = max_m;
-  sd.stats = static_cast<float*>(c->stats.p); sd.nsplit = nsplit; sd.scores = scores; sd.status = c->status;
+  const int dp3 = 3 * g.dp;
+  MAP_TRY(ensure(c->kb, static_cast<size_t>(vrows) * dp3 * 2));
+  MAP_TRY(ensure(c->qb, static_cast<size_t>(total_m) * dp3 * 2));
+  MAP_TRY(predictor_branch(c, vis, vrows, c->w[5], c->w[6], c->w[7], c->w[8], c->w[9], c->h1, c->h2, c->kb.p, 0,
+                           1.0f, k_out, nullptr, N, st, MAP_K_GEMM_FV1, MAP_K_GEMM_FV2, MAP_K_GEMM_WK));
+  MAP_TRY(predictor_branch(c, text, total_m, c->w[0], c->w[1], c->w[2], c->w[3], c->w[4], c->th1, c->th2, c->qb.p, 1,
+                           1.0f / std::sqrt(static_cast<float>(g.dp)), q_out, static_cast<const int*>(c->post.p), 1,
+                           st, MAP_K_GEMM_TEXT, MAP_K_GEMM_TEXT, MAP_K_GEMM_TEXT));
+  // Eq. 3 on the tensor cores: logits tile [visual tokens x question tokens] of one image,
+  // pass 1 -> per-slab column (max, sum exp), combine -> (max, 1/sum), pass 2 -> mean.
+  const int m_tiles = (N + 127) / 128, nparts = 4 * m_tiles;
+  const int ld = ((max_m + 3) / 4) * 4;
+  const int n_tiles = (max_m + 255) / 256;
+  MAP_TRY(ensure(c->stats, static_cast<size_t>(B) * (nparts + 1) * ld * 8));
+  float2* part = static_cast<float2*>(c->stats.p);
+  float2* fin = part + static_cast<size_t>(B) * nparts * ld;
+  GemmDesc d{};
+  d.A = c->kb.p; d.a_rows_total = vrows; d.a_row_stride = N;
+  d.B = c->qb.p; d.b_rows_total = total_m; d.b_row_stride = 0; d.b_off = d_off;
+  d.M = N; d.N = max_m; d.K = dp3; d.batch = B; d.n_limit = d_len; d.col_count = d_len;
+  d.status = c->status;
+  float* mean_out = scores;
+  if (n_tiles > 1) {
+    MAP_TRY(ensure(c->pmean, static_cast<size_t>(vrows) * n_tiles * 4));
+    mean_out = static_cast<float*>(c->pmean.p);
+  }
   {
     Timed t(c, st, MAP_K_SCORES);
-    c->counters.launches += 2;
-    CU_TRY(mapk::launch_scores(sd, st));
+    d.epi = mapk::EPI_SM_STATS; d.stats = part; d.stat_ld = ld;
+    d.C = part; d.ldc = 4; d.c_batch_stride = 0;
+    MAP_TRY(gemm(c, d, st));
+    ++c->counters.launches;
+    CU_TRY(mapk::launch_stats_combine(part, B, nparts, ld, d_len, fin, st));
+    d.epi = mapk::EPI_SM_MEAN; d.stats = fin;
+    d.C = mean_out; d.ldc = 4; d.c_batch_stride = static_cast<long long>(N) * n_tiles;
+    MAP_TRY(gemm(c, d, st));
+    if (n_tiles > 1) {
+      ++c->counters.launches;
+      CU_TRY(mapk::launch_sum_tiles(mean_out, B, N, n_tiles, scores, st));
+    }
   }
-  if (q_out) CU_TRY(cudaMemcpyAsync(q_out, c->qb.p, static_cast<size_t>(total_m) * g.dp * 4, cudaMemcpyDeviceToDevice, st));
-  if (k_out) CU_TRY(cudaMemcpyAsync(k_out, c->kb.p, static_cast<size_t>(vrows) * g.dp * 4, cudaMemcpyDeviceToDevice, st));
   return MAP_OK;
 }
 
@@ -569,7 +597,7 @@ void map_destroy(map_ctx* ctx) {
   for (void*& p : ctx->w)
     if (p) cudaFree(p);
   DevBuf* bufs[] = {&ctx->rope, &ctx->h1, &ctx->h2, &ctx->kb, &ctx->th1, &ctx->th2, &ctx->qb, &ctx->stats,
-                    &ctx->qoff, &ctx->post, &ctx->sqn, &ctx->sU, &ctx->sr2, &ctx->scstep, &ctx->sstate,
+                    &ctx->qoff, &ctx->post, &ctx->sqn, &ctx->pmean, &ctx->sU, &ctx->sr2, &ctx->scstep, &ctx->sstate,
                     &ctx->sEc, &ctx->spicks, &ctx->sr0, &ctx->sbt, &ctx->srn, &ctx->ssmall, &ctx->stheta,
                     &ctx->saslot, &ctx->sVg, &ctx->sG, &ctx->pvis, &ctx->ptext, &ctx->pout, &ctx->pkeep,
                     &ctx->pscores};

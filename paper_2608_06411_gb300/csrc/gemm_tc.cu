@@ -38,6 +38,10 @@ struct KArgs {
   const float2* rope; int rope_half;
   const int* pos; int pos_mod;
   int* status;
+  int split_kind; float scale; float* aux;
+  const int* b_off;
+  float2* stats; int stat_ld;
+  const int* col_count;
 };
 
 __device__ __forceinline__ float gelu_erf(float x) {
@@ -56,7 +60,8 @@ struct Smem {
   static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr uint32_t TILES = STAGES * STAGE_BYTES;
   static constexpr uint32_t BARS = (2 * STAGES + 5) * 8;
-  static constexpr uint32_t TOTAL = 1024 + TILES + BARS + 16;
+  static constexpr uint32_t XPOSE = 4 * 32 * 33 * 4;          // per-warp 32x32 transpose tiles (softmax stats)
+  static constexpr uint32_t TOTAL = 1024 + TILES + BARS + 16 + XPOSE;
   static constexpr uint32_t TMEM_COLS = 2 * BN;
 };
 
@@ -90,6 +95,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   uint64_t* drain = tempty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  float* xpose = reinterpret_cast<float*>(smem + S::TILES + S::BARS + 16);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -122,7 +128,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         TileCoord c = tile_coord(a, t, m_tiles, n_tiles, BN);
         if (c.skip) continue;
         const int arow = c.b * a.a_row_stride + c.m_blk * kBM;
-        const int brow = c.b * a.b_row_stride + c.n_blk * BN;
+        const int brow = (a.b_off ? __ldg(a.b_off + c.b) : c.b * a.b_row_stride) + c.n_blk * BN;
         for (int kb = 0; kb < KB; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1, a.status, abort_flag)) { ok = false; break; }
           mbar_arrive_expect_tx(&full[stage], S::STAGE_BYTES);
@@ -216,6 +222,112 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
               *reinterpret_cast<float4*>(out + HALF + ch * 32 + j) = make_float4(o2[0], o2[1], o2[2], o2[3]);
             }
           }
+        }
+      } else if constexpr (EPI == EPI_ROPE_SPLIT3) {
+        // BN == dp; x = RoPE(acc) * scale, stored as bf16 (hi, lo) segments
+        constexpr int HALF = BN / 2;
+        __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(a.C) + crow;
+        float* aux = a.aux ? a.aux + static_cast<long long>(row) * BN : nullptr;
+        int pos = 0;
+        if (row_ok) pos = a.pos ? __ldg(a.pos + row) : row % a.pos_mod;
+        const float2* rt = a.rope + static_cast<long long>(pos) * a.rope_half;
+        // segment order: keys [hi, lo, hi], queries [hi, hi, lo]
+        const int seg_lo = a.split_kind == 0 ? 1 : 2;
+#pragma unroll 1
+        for (int ch = 0; ch < HALF / 32; ++ch) {
+          uint32_t r1[32], r2[32];
+          tmem_ld32(tbase + ch * 32, r1);
+          tmem_ld32(tbase + HALF + ch * 32, r2);
+          if (row_ok) {
+#pragma unroll
+            for (int j = 0; j < 32; j += 8) {
+              float o1[8], o2[8];
+#pragma unroll
+              for (int u = 0; u < 8; ++u) {
+                const float2 cs = __ldg(rt + ch * 32 + j + u);
+                const float x1 = __uint_as_float(r1[j + u]), x2 = __uint_as_float(r2[j + u]);
+                o1[u] = x1 * cs.x - x2 * cs.y;
+                o2[u] = x2 * cs.x + x1 * cs.y;
+              }
+              if (aux) {
+#pragma unroll
+                for (int u = 0; u < 8; u += 4) {
+                  *reinterpret_cast<float4*>(aux + ch * 32 + j + u) = make_float4(o1[u], o1[u + 1], o1[u + 2], o1[u + 3]);
+                  *reinterpret_cast<float4*>(aux + HALF + ch * 32 + j + u) =
+                      make_float4(o2[u], o2[u + 1], o2[u + 2], o2[u + 3]);
+                }
+              }
+#pragma unroll
+              for (int u = 0; u < 8; ++u) { o1[u] *= a.scale; o2[u] *= a.scale; }
+              uint32_t h1[4], l1[4], h2[4], l2[4];
+#pragma unroll
+              for (int u = 0; u < 8; u += 2) {
+                const __nv_bfloat162 a1 = __floats2bfloat162_rn(o1[u], o1[u + 1]);
+                const __nv_bfloat162 a2 = __floats2bfloat162_rn(o2[u], o2[u + 1]);
+                h1[u / 2] = *reinterpret_cast<const uint32_t*>(&a1);
+                h2[u / 2] = *reinterpret_cast<const uint32_t*>(&a2);
+                l1[u / 2] = pack_bf16(o1[u] - __bfloat162float(a1.x), o1[u + 1] - __bfloat162float(a1.y));
+                l2[u / 2] = pack_bf16(o2[u] - __bfloat162float(a2.x), o2[u + 1] - __bfloat162float(a2.y));
+              }
+              const uint4 H1 = make_uint4(h1[0], h1[1], h1[2], h1[3]), L1 = make_uint4(l1[0], l1[1], l1[2], l1[3]);
+              const uint4 H2 = make_uint4(h2[0], h2[1], h2[2], h2[3]), L2 = make_uint4(l2[0], l2[1], l2[2], l2[3]);
+#pragma unroll
+              for (int sg = 0; sg < 3; ++sg) {
+                __nv_bfloat16* o = out + sg * BN + ch * 32 + j;
+                *reinterpret_cast<uint4*>(o) = sg == seg_lo ? L1 : H1;
+                *reinterpret_cast<uint4*>(o + HALF) = sg == seg_lo ? L2 : H2;
+              }
+            }
+          }
+        }
+      } else if constexpr (EPI == EPI_SM_STATS) {
+        // column max / sum of exp over this warp's 32 rows (rows past M count as -inf):
+        // the 32x32 chunk is transposed through shared memory, lane j reduces column j.
+        float2* part = a.stats + (static_cast<long long>(c.b) * m_tiles * 4 + c.m_blk * 4 + lane_grp) * a.stat_ld;
+        const int ncol = a.col_count ? min(lim, __ldg(a.col_count + c.b)) : lim;
+        float* tr = xpose + (warp - 2) * 32 * 33;
+#pragma unroll 1
+        for (int ch = 0; ch < BN / 32; ++ch) {
+          uint32_t r[32];
+          tmem_ld32(tbase + ch * 32, r);
+          const int cbase = col0 + ch * 32;
+          if (cbase >= ncol) continue;                    // uniform in the warp
+#pragma unroll
+          for (int j = 0; j < 32; ++j) tr[lane * 33 + j] = row_ok ? __uint_as_float(r[j]) : -INFINITY;
+          __syncwarp();
+          float m = -INFINITY;
+#pragma unroll
+          for (int i = 0; i < 32; ++i) m = fmaxf(m, tr[i * 33 + lane]);
+          float sum = 0.f;
+          if (m != -INFINITY) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) sum += expf(tr[i * 33 + lane] - m);
+          }
+          __syncwarp();
+          if (cbase + lane < ncol) part[cbase + lane] = make_float2(m, sum);
+        }
+      } else if constexpr (EPI == EPI_SM_MEAN) {
+        // p_hat[row] = (1/M_b) sum_col exp(l - max_col) / sum_col
+        const int ncol = a.col_count ? min(lim, __ldg(a.col_count + c.b)) : lim;
+        const float2* fin = a.stats + static_cast<long long>(c.b) * a.stat_ld;
+        float acc_p = 0.f;
+#pragma unroll 1
+        for (int ch = 0; ch < BN / 32; ++ch) {
+          uint32_t r[32];
+          tmem_ld32(tbase + ch * 32, r);
+          const int cbase = col0 + ch * 32;
+          if (cbase >= ncol) continue;
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            if (cbase + j < ncol) {
+              const float2 st = __ldg(fin + cbase + j);
+              acc_p += expf(__uint_as_float(r[j]) - st.x) * st.y;
+            }
+          }
+        }
+        if (row_ok) {
+          float* out = reinterpret_cast<float*>(a.C) + static_cast<long long>(c.b) * a.c_batch_stride;
+          out[static_cast<long long>(c.n_blk) * a.M + row] = acc_p / static_cast<float>(ncol > 0 ? ncol : 1);
         }
       } else if constexpr (EPI == EPI_F32) {
         float* out = reinterpret_cast<float*>(a.C) + crow + col0;
@@ -339,9 +451,13 @@ cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t st) {
   if ((reinterpret_cast<uintptr_t>(d.A) | reinterpret_cast<uintptr_t>(d.B)) & 15) return cudaErrorInvalidValue;
   if (d.M == 0) return cudaSuccess;
   // every output row and column block is written with 16-byte vector stores
+  const bool scalar_out = d.epi == EPI_SM_STATS || d.epi == EPI_SM_MEAN;   // float / float2 stores
   const bool f32 = d.epi == EPI_F32 || d.epi == EPI_ROPE_F32;
   const long long vec = f32 ? 4 : 8;
-  if (d.ldc % vec != 0 || d.c_batch_stride % vec != 0 || (reinterpret_cast<uintptr_t>(d.C) & 15)) return cudaErrorInvalidValue;
+  if (!scalar_out && (d.ldc % vec != 0 || d.c_batch_stride % vec != 0 || (reinterpret_cast<uintptr_t>(d.C) & 15)))
+    return cudaErrorInvalidValue;
+  if (scalar_out && (!d.stats || (reinterpret_cast<uintptr_t>(d.stats) & 7) || (reinterpret_cast<uintptr_t>(d.C) & 3)))
+    return cudaErrorInvalidValue;
   if ((d.epi == EPI_GELU_SPLIT || d.epi == EPI_BIAS_SPLIT) && d.ldc < 2LL * d.N) return cudaErrorInvalidValue;
   KArgs ka;
   ka.M = d.M; ka.N = d.N; ka.K = d.K; ka.batch = d.batch;
@@ -350,6 +466,8 @@ cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t st) {
   ka.bias = static_cast<const __nv_bfloat16*>(d.bias);
   ka.rope = d.rope; ka.rope_half = d.rope_half; ka.pos = d.pos; ka.pos_mod = d.pos_mod > 0 ? d.pos_mod : 1;
   ka.status = d.status;
+  ka.split_kind = d.split_kind; ka.scale = d.scale; ka.aux = d.aux; ka.b_off = d.b_off;
+  ka.stats = d.stats; ka.stat_ld = d.stat_ld; ka.col_count = d.col_count;
   switch (d.epi) {
     case EPI_GELU_BF16:
       if (d.N % 256 == 0) return run<256, 4, EPI_GELU_BF16>(d, ka, num_sms, st);
@@ -372,6 +490,14 @@ cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t st) {
       if (d.N % 256 == 0) return run<256, 4, EPI_BIAS_SPLIT>(d, ka, num_sms, st);
       if (d.N % 64 == 0) return run<64, 8, EPI_BIAS_SPLIT>(d, ka, num_sms, st);
       return cudaErrorInvalidValue;
+    case EPI_ROPE_SPLIT3:
+      if (d.N == 64) return run<64, 8, EPI_ROPE_SPLIT3>(d, ka, num_sms, st);
+      if (d.N == 128) return run<128, 6, EPI_ROPE_SPLIT3>(d, ka, num_sms, st);
+      return cudaErrorInvalidValue;
+    case EPI_SM_STATS:
+      return run<256, 4, EPI_SM_STATS>(d, ka, num_sms, st);
+    case EPI_SM_MEAN:
+      return run<256, 4, EPI_SM_MEAN>(d, ka, num_sms, st);
     case EPI_F32:
       return run<128, 6, EPI_F32>(d, ka, num_sms, st);
     default:

@@ -8,8 +8,15 @@ namespace mapk {
 // *_SPLIT epilogues store an fp32 activation x as two bf16 halves, hi = bf16(x) at
 // column c and lo = bf16(x - hi) at column N + c of a [rows, 2N] buffer, so that the next
 // layer can consume ~16 significant bits through a bf16 GEMM: [hi | lo] @ [W | W]^T.
+// EPI_ROPE_SPLIT3 applies RoPE (and `scale`) and stores the vector as three bf16
+// segments, [hi | lo | hi] (split_kind 0, keys) or [hi | hi | lo] (split_kind 1, queries),
+// so that one bf16 GEMM with K = 3 dp gives q.k to about 16 significant bits; it can also
+// store the fp32 vector to `aux`.
+// EPI_SM_STATS / EPI_SM_MEAN are the two passes of Eq. 3 over a logits tile (rows =
+// visual tokens, columns = question tokens): per-column max / sum of exp over each
+// 32-row slab, then per-row mean over columns of exp(l - max) / sum.
 enum Epi { EPI_GELU_BF16 = 0, EPI_BIAS_BF16 = 1, EPI_ROPE_F32 = 2, EPI_F32 = 3, EPI_GELU_SPLIT = 4,
-           EPI_BIAS_SPLIT = 5 };
+           EPI_BIAS_SPLIT = 5, EPI_ROPE_SPLIT3 = 6, EPI_SM_STATS = 7, EPI_SM_MEAN = 8 };
 
 // Batched C = epi(A @ B^T): A rows [batch][a_row_stride] x K, B rows [batch][b_row_stride] x K
 // (both bf16, K contiguous, tightly packed 2D arrays of a_rows_total / b_rows_total rows).
@@ -24,6 +31,15 @@ struct GemmDesc {
   const int* pos; int pos_mod;          // per-row positions (device) or row % pos_mod
   int epi;
   int* status;
+  // EPI_ROPE_SPLIT3
+  int split_kind = 0; float scale = 1.f; float* aux = nullptr;
+  // batched B rows at per-batch offsets (device) instead of b * b_row_stride
+  const int* b_off = nullptr;
+  // EPI_SM_STATS: partial (max, sum) per 32-row slab [batch][m_tiles * 4][stat_ld] (float2)
+  // EPI_SM_MEAN:  final (max, 1/sum) per column [batch][stat_ld]; output C = scores
+  //               [batch][M] when one column tile covers all columns
+  float2* stats = nullptr; int stat_ld = 0;
+  const int* col_count = nullptr;       // per-batch number of valid columns (M_b)
 };
 
 // Returns cudaSuccess, or an error for an unsupported shape (cudaErrorInvalidValue).
@@ -32,17 +48,13 @@ cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t st);
 // Squared row norms of bf16 rows: out[r] = sum_d x[r, d]^2 (fp32).
 cudaError_t launch_row_sqnorm(const void* x, long long rows, int D, float* out, cudaStream_t st);
 
-// Eq. 3 softmax statistics and mean (q [sum M, dp], k [B*N, dp] fp32).
-struct ScoreDesc {
-  const float* q; const float* k;
-  const int* q_off;       // [B+1] device row offsets of each image's queries
-  int B, N, dp, max_m;
-  float* stats;           // workspace [sum M][nsplit][2]
-  int nsplit;
-  float* scores;          // [B, N]
-  int* status;
-};
-cudaError_t launch_scores(const ScoreDesc& d, cudaStream_t st);
+// scores[b, n] = sum_t part[b, t, n] over n_tiles column-tile partial means.
+cudaError_t launch_sum_tiles(const float* part, int B, int N, int n_tiles, float* scores, cudaStream_t st);
+
+// Combines the per-slab softmax statistics into (max, 1/sum) per question token:
+// part [B][nparts][ld] -> fin [B][ld], columns < lens[b].
+cudaError_t launch_stats_combine(const float2* part, int B, int nparts, int ld, const int* lens, float2* fin,
+                                 cudaStream_t st);
 
 // Gather rows: out[b, j, :] = V[b, idx[b, j], :].
 cudaError_t launch_gather(const void* V, const int32_t* idx, int B, int N, int k, int D, void* out,

@@ -1,4 +1,4 @@
-// Eq. 3 softmax-mean scores, squared row norms, and the compaction gather.
+// Eq. 3 softmax statistics combine, squared row norms, and the compaction gather.
 #include <algorithm>
 
 #include "kernels.h"
@@ -48,120 +48,40 @@ __global__ void gather_rows_kernel(const uint4* __restrict__ V, const int32_t* _
   for (int v = threadIdx.x; v < vec_per_row; v += blockDim.x) d[v] = __ldg(s + v);
 }
 
-// ------------------------------------------------------------------ Eq. 3
-// Pass 1: per query m and key split, running max / sum of exp over the split's keys.
-// Thread = one query (q_m in registers); keys staged through shared memory in tiles.
-template <int DP>
-__global__ void __launch_bounds__(128) score_stats_kernel(const float* __restrict__ q, const float* __restrict__ k,
-                                                          const int* __restrict__ q_off, int N, int nsplit,
-                                                          float scale, float2* __restrict__ stats) {
-  constexpr int KT = 32;
-  __shared__ float4 ks[KT * DP / 4];
-  const int b = blockIdx.z, split = blockIdx.y;
-  const int m0 = q_off[b], M = q_off[b + 1] - m0;
-  const int m = blockIdx.x * 128 + threadIdx.x;
-  if (blockIdx.x * 128 >= M) return;
-  const bool active = m < M;
-  float qr[DP];
-  {
-    const float4* qp = reinterpret_cast<const float4*>(q + static_cast<long long>(m0 + (active ? m : 0)) * DP);
-#pragma unroll
-    for (int i = 0; i < DP / 4; ++i) {
-      const float4 v = __ldg(qp + i);
-      qr[4 * i] = v.x * scale; qr[4 * i + 1] = v.y * scale; qr[4 * i + 2] = v.z * scale; qr[4 * i + 3] = v.w * scale;
-    }
+// (max, sum) partials of one column over all slabs -> (max, 1/sum); thread = column.
+__global__ void stats_combine_kernel(const float2* __restrict__ part, int nparts, int ld, const int* __restrict__ lens,
+                                     float2* __restrict__ fin) {
+  const int b = blockIdx.y, col = blockIdx.x * blockDim.x + threadIdx.x;
+  if (col >= lens[b]) return;
+  const float2* p = part + static_cast<long long>(b) * nparts * ld + col;
+  float m = -INFINITY;
+  for (int i = 0; i < nparts; ++i) m = fmaxf(m, p[static_cast<long long>(i) * ld].x);
+  float sum = 0.f;
+  for (int i = 0; i < nparts; ++i) {
+    const float2 v = p[static_cast<long long>(i) * ld];
+    if (v.y > 0.f) sum += v.y * expf(v.x - m);
   }
-  const int per = (N + nsplit - 1) / nsplit;
-  const int n_beg = split * per, n_end = min(N, n_beg + per);
-  float mx = -INFINITY, sm = 0.f;
-  const float4* kb = reinterpret_cast<const float4*>(k + static_cast<long long>(b) * N * DP);
-  for (int t0 = n_beg; t0 < n_end; t0 += KT) {
-    const int cnt = min(KT, n_end - t0);
-    __syncthreads();
-    for (int i = threadIdx.x; i < cnt * DP / 4; i += 128) ks[i] = __ldg(kb + static_cast<long long>(t0) * (DP / 4) + i);
-    __syncthreads();
-    for (int j = 0; j < cnt; ++j) {
-      float l0 = 0.f, l1 = 0.f, l2 = 0.f, l3 = 0.f;
-#pragma unroll
-      for (int i = 0; i < DP / 4; ++i) {
-        const float4 kv = ks[j * (DP / 4) + i];
-        l0 = fmaf(qr[4 * i], kv.x, l0);
-        l1 = fmaf(qr[4 * i + 1], kv.y, l1);
-        l2 = fmaf(qr[4 * i + 2], kv.z, l2);
-        l3 = fmaf(qr[4 * i + 3], kv.w, l3);
-      }
-      const float l = (l0 + l1) + (l2 + l3);
-      if (l > mx) { sm = sm * expf(mx - l) + 1.f; mx = l; }
-      else sm += expf(l - mx);
-    }
-  }
-  if (active) stats[static_cast<long long>(m0 + m) * nsplit + split] = make_float2(mx, sm);
+  fin[static_cast<long long>(b) * ld + col] = make_float2(m, 1.0f / sum);
 }
 
-// Pass 2: thread = one key n (k_n in registers); loops over the image's queries with
-// their combined (max, 1/sum) and accumulates p_hat_n = (1/M) sum_m exp(l_mn - max_m) / sum_m.
-template <int DP>
-__global__ void __launch_bounds__(128) score_mean_kernel(const float* __restrict__ q, const float* __restrict__ k,
-                                                         const int* __restrict__ q_off, int N, int nsplit,
-                                                         float scale, const float2* __restrict__ stats,
-                                                         float* __restrict__ scores) {
-  constexpr int QT = 32;
-  __shared__ float4 qs[QT * DP / 4];
-  __shared__ float2 qn[QT];          // (max_m, 1 / sum_m)
-  const int b = blockIdx.y;
-  const int n = blockIdx.x * 128 + threadIdx.x;
-  const bool active = n < N;
-  const int m0 = q_off[b], M = q_off[b + 1] - m0;
-  float kr[DP];
-  {
-    const float4* kp = reinterpret_cast<const float4*>(k + (static_cast<long long>(b) * N + (active ? n : 0)) * DP);
-#pragma unroll
-    for (int i = 0; i < DP / 4; ++i) {
-      const float4 v = __ldg(kp + i);
-      kr[4 * i] = v.x; kr[4 * i + 1] = v.y; kr[4 * i + 2] = v.z; kr[4 * i + 3] = v.w;
-    }
-  }
-  float acc = 0.f;
-  for (int t0 = 0; t0 < M; t0 += QT) {
-    const int cnt = min(QT, M - t0);
-    __syncthreads();
-    const float4* qp = reinterpret_cast<const float4*>(q + static_cast<long long>(m0 + t0) * DP);
-    for (int i = threadIdx.x; i < cnt * DP / 4; i += 128) {
-      float4 v = __ldg(qp + i);
-      v.x *= scale; v.y *= scale; v.z *= scale; v.w *= scale;
-      qs[i] = v;
-    }
-    if (threadIdx.x < cnt) {
-      const float2* st = stats + static_cast<long long>(m0 + t0 + threadIdx.x) * nsplit;
-      float mx = -INFINITY;
-      for (int s = 0; s < nsplit; ++s) mx = fmaxf(mx, st[s].x);
-      float sm = 0.f;
-      for (int s = 0; s < nsplit; ++s) {
-        const float2 v = st[s];
-        if (v.y > 0.f) sm += v.y * expf(v.x - mx);
-      }
-      qn[threadIdx.x] = make_float2(mx, 1.f / sm);
-    }
-    __syncthreads();
-    for (int j = 0; j < cnt; ++j) {
-      float l0 = 0.f, l1 = 0.f, l2 = 0.f, l3 = 0.f;
-#pragma unroll
-      for (int i = 0; i < DP / 4; ++i) {
-        const float4 qv = qs[j * (DP / 4) + i];
-        l0 = fmaf(qv.x, kr[4 * i], l0);
-        l1 = fmaf(qv.y, kr[4 * i + 1], l1);
-        l2 = fmaf(qv.z, kr[4 * i + 2], l2);
-        l3 = fmaf(qv.w, kr[4 * i + 3], l3);
-      }
-      const float l = (l0 + l1) + (l2 + l3);
-      const float2 st = qn[j];
-      acc += expf(l - st.x) * st.y;
-    }
-  }
-  if (active) scores[static_cast<long long>(b) * N + n] = acc / static_cast<float>(M);
+__global__ void sum_tiles_kernel(const float* __restrict__ part, int N, int n_tiles, long long total,
+                                 float* __restrict__ scores) {
+  const long long i = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (i >= total) return;
+  const long long b = i / N, n = i - b * N;
+  float s = 0.f;
+  for (int t = 0; t < n_tiles; ++t) s += part[(b * n_tiles + t) * N + n];
+  scores[i] = s;
 }
 
 }  // namespace
+
+cudaError_t launch_stats_combine(const float2* part, int B, int nparts, int ld, const int* lens, float2* fin,
+                                 cudaStream_t st) {
+  dim3 g((ld + 127) / 128, B);
+  stats_combine_kernel<<<g, 128, 0, st>>>(part, nparts, ld, lens, fin);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_row_sqnorm(const void* x, long long rows, int D, float* out, cudaStream_t st) {
   if (rows <= 0) return cudaSuccess;
@@ -183,22 +103,9 @@ cudaError_t launch_gather(const void* V, const int32_t* idx, int B, int N, int k
   return cudaGetLastError();
 }
 
-cudaError_t launch_scores(const ScoreDesc& d, cudaStream_t st) {
-  const float scale = 1.0f / sqrtf(static_cast<float>(d.dp));
-  dim3 g1((d.max_m + 127) / 128, d.nsplit, d.B);
-  dim3 g2((d.N + 127) / 128, d.B);
-  const float2* stats = reinterpret_cast<const float2*>(d.stats);
-  if (d.dp == 128) {
-    score_stats_kernel<128><<<g1, 128, 0, st>>>(d.q, d.k, d.q_off, d.N, d.nsplit, scale,
-                                                reinterpret_cast<float2*>(d.stats));
-    score_mean_kernel<128><<<g2, 128, 0, st>>>(d.q, d.k, d.q_off, d.N, d.nsplit, scale, stats, d.scores);
-  } else if (d.dp == 64) {
-    score_stats_kernel<64><<<g1, 128, 0, st>>>(d.q, d.k, d.q_off, d.N, d.nsplit, scale,
-                                               reinterpret_cast<float2*>(d.stats));
-    score_mean_kernel<64><<<g2, 128, 0, st>>>(d.q, d.k, d.q_off, d.N, d.nsplit, scale, stats, d.scores);
-  } else {
-    return cudaErrorInvalidValue;
-  }
+cudaError_t launch_sum_tiles(const float* part, int B, int N, int n_tiles, float* scores, cudaStream_t st) {
+  const long long total = static_cast<long long>(B) * N;
+  sum_tiles_kernel<<<static_cast<unsigned>((total + 255) / 256), 256, 0, st>>>(part, N, n_tiles, total, scores);
   return cudaGetLastError();
 }
 
