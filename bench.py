@@ -35,6 +35,7 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 from paper_2608_06411_gb300 import workloads as W  # noqa: E402
+from paper_2608_06411_gb300.sharding import image_range, max_over_ranks  # noqa: E402
 
 METRIC = "images pruned/s (score+select+gather) at N=2880,k=160; p50/p99 µs; % roofline"
 WORKLOAD = W.WORKLOADS["c3"]
@@ -213,7 +214,8 @@ def main():
         pg = dist
 
     B, N, K, D = WORKLOAD.B, WORKLOAD.N, WORKLOAD.K, WORKLOAD.D
-    vis_np, text_np, lens = W.make_batch(WORKLOAD, B=B, first_image=rank * B, threads=min(16, _CORES))
+    first, B = image_range(B * ws, ws, rank)              # weak scaling: 64 images per rank
+    vis_np, text_np, lens = W.make_batch(WORKLOAD, B=B, first_image=first, threads=min(16, _CORES))
     w = W.make_weights(DIMS)
     ctx = mb.Context({k: torch.from_numpy(v.view(np.int16)).to(dev) for k, v in w.items()}, DIMS.D, DIMS.Dh,
                      DIMS.dp)
@@ -265,10 +267,7 @@ def main():
              [("fv2", mb.K_GEMM_FV2), ("wk", mb.K_GEMM_WK), ("text", mb.K_GEMM_TEXT), ("scores", mb.K_SCORES),
               ("select", mb.K_SELECT), ("gather", mb.K_GATHER)]}
     ctx.set_timing(False)
-    if pg:
-        t = torch.tensor([total_ms], device=dev)
-        pg.all_reduce(t, op=pg.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(total_ms, dev)
 
     images = B * args.steps * ws
     value = images / (total_ms / 1000.0)
@@ -312,10 +311,7 @@ def main():
     for _ in range(args.e2e_steps):
         ctx.prune(text_h, vis_h, lens, K, out_h, keep_h)
     e2e_s = time.perf_counter() - t0
-    if pg:
-        t = torch.tensor([e2e_s], device=dev)
-        pg.all_reduce(t, op=pg.ReduceOp.MAX)
-        e2e_s = float(t.item())
+    e2e_s = max_over_ranks(e2e_s, dev)
     e2e_value = B * args.e2e_steps * ws / e2e_s
     ctx.check()
 
