@@ -131,6 +131,28 @@ int map_gather(map_ctx *ctx, const void *vis_feats, const int32_t *keep_idx, int
                int k, void *out, void *stream);
 
 /*
+ * map_select without allocating memory in the call (the paper has no counterpart; this
+ * is a deployment variant of map_select).  Same arguments, results and limits as
+ * map_select, but every scratch buffer is carved from one static device array of
+ * MAP_NOALLOC_SCRATCH_BYTES held by each GPU that loads it until the process exits, so
+ * that callers that must not allocate (during CUDA-graph stream capture, inside a fixed
+ * device-memory budget or someone else's pool, on a real-time path) can still prune.
+ * The call makes no cudaMalloc / cudaFree and allocates through no library.
+ * Workspace needed, in bytes (each array rounded up to 256): 17 B*N + 16 B*k + 4 B*256
+ * + 8 B + small per-image counters, plus, when the diversity term is on (lambda > 0 and
+ * K0 < k), 4 B*N*ceil4(k) + 2 B*R*D + 4 B*256*R with R = ceil16(256 + k).  A request
+ * that does not fit returns MAP_EUNSUPPORTED and does nothing.  One LLaVA-NeXT image
+ * (N = 2880, k = 160, D = 4096) needs about 6 MB.
+ * The first call on a device looks the array's address up (device must be current);
+ * make that call before any stream capture.  All calls share the array and it keeps the
+ * last call's contents; calls whose GPU work overlaps (other streams, other threads)
+ * race on it and must be serialised by the caller.
+ */
+#define MAP_NOALLOC_SCRATCH_BYTES (16u * 1024u * 1024u)
+int map_select_noalloc(map_ctx *ctx, const float *scores, const void *vis_feats, int B, int N,
+                       int k, int32_t *keep_idx, int32_t *pick_order, void *stream);
+
+/*
  * The whole path in one call: score, select, gather.  Pointers may be HOST or DEVICE
  * memory (detected per pointer); host inputs are copied in and host outputs copied out
  * on `stream`, and the call synchronises `stream` before returning when any pointer is

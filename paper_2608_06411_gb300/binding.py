@@ -43,6 +43,8 @@ SIGNATURES = {
     "map_init": (c_int, [POINTER(MapConfig), POINTER(MapWeights), POINTER(c_void_p)]),
     "map_score": (c_int, [c_void_p, c_void_p, c_void_p, POINTER(c_int32), c_int, c_int, c_void_p, c_void_p]),
     "map_select": (c_int, [c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_void_p, c_void_p, c_void_p]),
+    "map_select_noalloc": (c_int, [c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_void_p, c_void_p,
+                                   c_void_p]),
     "map_gather": (c_int, [c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_void_p, c_void_p]),
     "map_prune": (c_int, [c_void_p, c_void_p, c_void_p, POINTER(c_int32), c_int, c_int, c_int, c_void_p,
                           c_void_p, c_void_p, c_void_p]),
@@ -164,6 +166,14 @@ class Context:
             order = torch.empty((B, k), dtype=torch.int32, device=vis.device)
         _check(lib.map_select(self.h, _ptr(scores), _ptr(vis), B, N, k, _ptr(keep), _ptr(order), _stream(stream)),
                "map_select")
+        return keep, order
+
+    def select_noalloc(self, scores, vis, k: int, keep, order=None, stream=None):
+        """map_select_noalloc: the caller provides keep (and order) buffers; nothing is
+        allocated during the call."""
+        B, N = vis.shape[0], vis.shape[1]
+        _check(lib.map_select_noalloc(self.h, _ptr(scores), _ptr(vis), B, N, k, _ptr(keep), _ptr(order),
+                                      _stream(stream)), "map_select_noalloc")
         return keep, order
 
     def gather(self, vis, keep, out=None, stream=None):

@@ -461,6 +461,22 @@ bool is_device_ptr(const void* p) {
 
 }  // namespace
 
+// Read-only view of a context for other translation units of the library.
+namespace mapk {
+struct CtxView {
+  const map_config* cfg;
+  int device, num_sms;
+  int* status;
+  int32_t* h_done;
+  long long* launches;
+  long long* rounds;
+};
+CtxView ctx_view(map_ctx* c) {
+  return CtxView{&c->cfg, c->device, c->num_sms, c->status, c->h_done, &c->counters.launches,
+                 &c->counters.select_rounds};
+}
+}  // namespace mapk
+
 extern "C" {
 
 int map_config_default(map_config* cfg) {
