@@ -18,6 +18,7 @@ namespace {
 
 constexpr int kSelS = 256;          // active-set size of the selection (Gram block rows)
 constexpr int kMaxKDiverse = 1024;  // k limit when the diversity term is on (shared-memory staging)
+constexpr int kProjMaxBasis = 128;  // R0 size up to which the projection pass is used
 constexpr int kMaxK = 4096;
 constexpr int kMaxN = 16384;
 
@@ -385,14 +386,21 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, 
   s.theta = static_cast<uint64_t*>(c->stheta.p);
   s.aslot = static_cast<int32_t*>(c->saslot.p);
 
-  if (K0 < K) {
+  // With 0 < K0 <= 128, one tensor-core pass over V after the R0 rounds gives every
+  // candidate its exact value (and ||v||^2); otherwise values start from p_hat * ||v||^lambda.
+  const bool project = K0 > 0 && K0 < K && K0 <= kProjMaxBasis;
+  if (K0 < K && !project) {
     ++c->counters.launches;
     CU_TRY(mapk::launch_row_sqnorm(vis, BN, g.D, static_cast<float*>(c->sqn.p), st));
-  } else {
+  } else if (K0 >= K) {
     CU_TRY(cudaMemsetAsync(c->sqn.p, 0, BN * 4, st));
   }
   ++c->counters.launches;
-  CU_TRY(mapk::launch_sel_init(s, st));
+  {
+    mapk::SelState si = s;
+    if (project) si.sqn = nullptr;     // written by the projection
+    CU_TRY(mapk::launch_sel_init(si, st));
+  }
   if (K0 < K) {
     MAP_TRY(ensure(c->sEc, static_cast<size_t>(BN) * KP * 4));
     MAP_TRY(ensure(c->sVg, static_cast<size_t>(B) * R * g.D * 2));
@@ -410,6 +418,33 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, 
     const long long cap = 8LL * (K + N / S) + 64;
     long long rounds = 0;
     int burst = (K0 + S - 1) / S + 6;   // rounds queued per host check; finished images skip
+    if (project) {
+      s.diag_sq = 1;                    // R0 tokens take ||v||^2 from the Gram diagonal
+      for (int r = 0; r < (K0 + S - 1) / S; ++r) {
+        c->counters.launches += 3;
+        CU_TRY(mapk::launch_sel_choose(s, st));
+        MAP_TRY(gemm(c, d, st));
+        CU_TRY(mapk::launch_sel_greedy(s, st));
+        ++rounds;
+        ++c->counters.select_rounds;
+      }
+      s.diag_sq = 0;
+      c->counters.launches += 2;
+      CU_TRY(mapk::launch_sel_proj_prep(s, st));
+      CU_TRY(mapk::launch_sel_gather(s, st));
+      GemmDesc pd{};
+      pd.A = vis; pd.a_rows_total = BN; pd.a_row_stride = N;
+      pd.B = s.Vg; pd.b_rows_total = static_cast<long long>(B) * R; pd.b_row_stride = R; pd.b_base = S;
+      pd.M = N; pd.N = kProjMaxBasis; pd.K = g.D; pd.batch = B; pd.n_limit = nullptr;
+      pd.C = nullptr; pd.ldc = 0; pd.c_batch_stride = 0;
+      pd.epi = mapk::EPI_PROJECT; pd.status = c->status;
+      pd.proj.state = s.state; pd.proj.scores = scores; pd.proj.Ec = s.Ec; pd.proj.KP = KP;
+      pd.proj.basis_tok = s.basis_tok; pd.proj.rnorm = s.rnorm; pd.proj.nbasis = s.nbasis; pd.proj.Kcap = K;
+      pd.proj.lambda = g.lambda; pd.proj.tau = g.tau;
+      pd.proj.r2 = s.r2; pd.proj.U = s.U; pd.proj.sqn = static_cast<float*>(c->sqn.p); pd.proj.cstep = s.cstep;
+      MAP_TRY(gemm(c, pd, st));
+      burst = 6;
+    }
     for (;;) {
       for (int r = 0; r < burst; ++r) {
         c->counters.launches += 3;

@@ -5,7 +5,7 @@
 // epilogue (section "Cross-Modal Attention Distillation"), and the Gram blocks
 // <v_i, v_j> that the diversity term of Eq. 4 needs.
 //
-// Structure (one CTA per SM, 6 warps):
+// Structure (one CTA per SM, 6 warps; 8 for EPI_PROJECT):
 //   warp 0      one thread issues TMA loads of 128x64 (A) and BNx64 (B) bf16 tiles, 128-byte
 //               swizzled, into a STAGES-deep shared-memory ring (mbarrier full/empty).
 //   warp 1      allocates TMEM (2 accumulators x BN fp32 columns); one thread issues
@@ -14,6 +14,7 @@
 //               thread), apply bias / GELU / RoPE, store (bf16, bf16 hi/lo pair, or fp32);
 //               release the accumulator so the
 //               MMA warp can start the tile after next while this one drains.
+//   warps 6-7   (EPI_PROJECT only) sum ||row||^2 of every A tile from shared memory.
 // All waits are bounded (ptx.cuh); a timeout sets ST_TIMEOUT and every role drains and exits.
 #include <algorithm>
 #include <cstdio>
@@ -28,7 +29,6 @@ namespace {
 
 constexpr int kBM = 128;
 constexpr int kBK = 64;
-constexpr int kThreads = 192;
 
 struct KArgs {
   int M, N, K, batch, a_row_stride, b_row_stride;
@@ -42,6 +42,8 @@ struct KArgs {
   const int* b_off;
   float2* stats; int stat_ld;
   const int* col_count;
+  int b_base;
+  ProjArgs proj;
 };
 
 __device__ __forceinline__ float gelu_erf(float x) {
@@ -53,17 +55,30 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
   return *reinterpret_cast<uint32_t*>(&h);
 }
 
-template <int BN, int STAGES>
+constexpr int kProjMaxBasis = 128;             // EPI_PROJECT: R0 basis size supported
+
+template <int BN, int STAGES, int EPI>
 struct Smem {
+  static constexpr bool PROJ = EPI == EPI_PROJECT;
   static constexpr uint32_t A_BYTES = kBM * kBK * 2;
   static constexpr uint32_t B_BYTES = BN * kBK * 2;
   static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr uint32_t TILES = STAGES * STAGE_BYTES;
-  static constexpr uint32_t BARS = (2 * STAGES + 5) * 8;
-  static constexpr uint32_t XPOSE = 4 * 32 * 33 * 4;          // per-warp 32x32 transpose tiles (softmax stats)
-  static constexpr uint32_t TOTAL = 1024 + TILES + BARS + 16 + XPOSE;
+  static constexpr uint32_t BARS = (2 * STAGES + 5 + (PROJ ? 5 : 0)) * 8;
+  static constexpr uint32_t XPOSE = EPI == EPI_SM_STATS ? 4 * 32 * 33 * 4 : 0;   // per-warp 32x32 transposes
+  static constexpr uint32_t LSM = PROJ ? kProjMaxBasis * kProjMaxBasis * 4 : 0;  // L rows of the R0 basis
+  static constexpr uint32_t PEXTRA = PROJ ? (kProjMaxBasis + 2 * kBM) * 4 : 0;   // 1/r, ||v||^2 x 2 buffers
+  static constexpr uint32_t TOTAL = 1024 + TILES + BARS + 16 + XPOSE + LSM + PEXTRA;
   static constexpr uint32_t TMEM_COLS = 2 * BN;
+  static constexpr int THREADS = PROJ ? 256 : 192;   // + 2 warps summing ||v||^2 for EPI_PROJECT
 };
+
+__device__ __forceinline__ float proj_value(float p, float r2, float sq, float lam, float tau) {
+  if (lam == 0.f) return p > 0.f ? p : 0.f;
+  if (!(r2 > tau * sq) || !(r2 > 0.f)) return 0.f;
+  const float v = lam == 1.f ? p * sqrtf(r2) : p * powf(r2, 0.5f * lam);
+  return v > 0.f ? v : 0.f;
+}
 
 struct TileCoord { int b, m_blk, n_blk; bool skip; };
 
@@ -80,9 +95,9 @@ __device__ __forceinline__ TileCoord tile_coord(const KArgs& a, int t, int m_til
 }
 
 template <int BN, int STAGES, int EPI>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(Smem<BN, STAGES, EPI>::THREADS, 1)
 gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, KArgs a) {
-  using S = Smem<BN, STAGES>;
+  using S = Smem<BN, STAGES, EPI>;
   constexpr uint32_t IDESC = idesc_bf16(kBM, BN);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -93,15 +108,25 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   uint64_t* tfull = empty + STAGES;
   uint64_t* tempty = tfull + 2;
   uint64_t* drain = tempty + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1 + (S::PROJ ? 5 : 0));
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  uint64_t* nfull = drain + 1;                   // EPI_PROJECT: ||v||^2 of a tile ready / consumed
+  uint64_t* nempty = nfull + 2;
+  uint64_t* egsync = nempty + 2;                 // EPI_PROJECT: epilogue warps' group barrier
   float* xpose = reinterpret_cast<float*>(smem + S::TILES + S::BARS + 16);
+  float* Lsm = xpose + S::XPOSE / 4;
+  float* rinv_sm = Lsm + S::LSM / 4;
+  float* sqbuf = rinv_sm + (S::PROJ ? kProjMaxBasis : 0);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
-    for (int s = 0; s < STAGES; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
+    for (int s = 0; s < STAGES; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], S::PROJ ? 3 : 1); }
     for (int i = 0; i < 2; ++i) { mbar_init(&tfull[i], 1); mbar_init(&tempty[i], 128); }
     mbar_init(drain, 1);
+    if constexpr (S::PROJ) {
+      for (int i = 0; i < 2; ++i) { mbar_init(&nfull[i], 2); mbar_init(&nempty[i], 128); }
+      mbar_init(egsync, 128);
+    }
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -128,7 +153,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         TileCoord c = tile_coord(a, t, m_tiles, n_tiles, BN);
         if (c.skip) continue;
         const int arow = c.b * a.a_row_stride + c.m_blk * kBM;
-        const int brow = (a.b_off ? __ldg(a.b_off + c.b) : c.b * a.b_row_stride) + c.n_blk * BN;
+        const int brow = (a.b_off ? __ldg(a.b_off + c.b) : c.b * a.b_row_stride + a.b_base) + c.n_blk * BN;
         for (int kb = 0; kb < KB; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1, a.status, abort_flag)) { ok = false; break; }
           mbar_arrive_expect_tx(&full[stage], S::STAGE_BYTES);
@@ -178,14 +203,49 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       }
     }
     __syncwarp();
-  } else {
+  } else if (warp < 6) {
     // ------------------------------------------------------------------ epilogue
     const int lane_grp = warp & 3;                 // TMEM lanes this warp may access
     const int r_in_tile = lane_grp * 32 + lane;
     uint32_t acc = 0, acc_phase = 0;
-    for (int t = blockIdx.x; t < total; t += gridDim.x) {
+    int staged_b = -1;                             // EPI_PROJECT: image whose L is in shared memory
+    uint32_t eg_phase = 0;
+    bool eg_ok = true;
+    for (int t = blockIdx.x; t < total && eg_ok; t += gridDim.x) {
       TileCoord c = tile_coord(a, t, m_tiles, n_tiles, BN);
       if (c.skip) continue;
+      if constexpr (S::PROJ) {
+        if (c.b != staged_b) {                     // stage L and 1/r of this image's R0 basis
+          // group barrier of the 128 epilogue threads (bounded, unlike a named barrier)
+          mbar_arrive(egsync);
+          if (!mbar_wait(egsync, eg_phase, a.status, abort_flag)) { eg_ok = false; break; }
+          eg_phase ^= 1;
+          const ProjArgs& pj = a.proj;
+          const int nb0 = min(kProjMaxBasis, __ldg(pj.nbasis + c.b));
+          const long long ibase = static_cast<long long>(c.b) * a.M;
+          const int KV = kProjMaxBasis / 4;
+          for (int t4 = threadIdx.x - 64; t4 < nb0 * KV; t4 += 128) {
+            const int i = t4 / KV, q = (t4 - i * KV) * 4;
+            float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (q < i) {
+              const int tk = __ldg(pj.basis_tok + static_cast<long long>(c.b) * pj.Kcap + i);
+              const float* row = pj.Ec + (ibase + tk) * pj.KP + q;
+              v.x = row[0];
+              v.y = q + 1 < i ? row[1] : 0.f;
+              v.z = q + 2 < i ? row[2] : 0.f;
+              v.w = q + 3 < i ? row[3] : 0.f;
+            }
+            *reinterpret_cast<float4*>(Lsm + i * kProjMaxBasis + q) = v;
+          }
+          for (int i = threadIdx.x - 64; i < nb0; i += 128)
+            rinv_sm[i] = 1.0f / __ldg(pj.rnorm + static_cast<long long>(c.b) * pj.Kcap + i);
+          mbar_arrive(egsync);
+          if (!mbar_wait(egsync, eg_phase, a.status, abort_flag)) { eg_ok = false; break; }
+          eg_phase ^= 1;
+          staged_b = c.b;
+        }
+        if (!mbar_wait(&nfull[acc], acc_phase, a.status, abort_flag)) break;
+      }
       if (!mbar_wait(&tfull[acc], acc_phase, a.status, abort_flag)) break;
       tc_fence_after();
       const int row = c.m_blk * kBM + r_in_tile;
@@ -329,6 +389,55 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           float* out = reinterpret_cast<float*>(a.C) + static_cast<long long>(c.b) * a.c_batch_stride;
           out[static_cast<long long>(c.n_blk) * a.M + row] = acc_p / static_cast<float>(ncol > 0 ? ncol : 1);
         }
+      } else if constexpr (EPI == EPI_PROJECT) {
+        // Cholesky coordinates of token `row` on the R0 basis by forward substitution,
+        // 32 basis vectors at a time: e_beta = (g_beta - sum_{q<beta} L[beta][q] e_q) / r_beta.
+        const ProjArgs& pj = a.proj;
+        const int nb0 = min(kProjMaxBasis, __ldg(pj.nbasis + c.b));
+        const long long tok = static_cast<long long>(c.b) * a.M + row;
+        const bool alive = row_ok && __ldg(pj.state + tok) == 0;
+        float* erow = pj.Ec + tok * pj.KP;
+        const float sq = sqbuf[acc * kBM + r_in_tile];
+        float r2 = sq;
+#pragma unroll 1
+        for (int b0 = 0; b0 < nb0; b0 += 32) {
+          uint32_t g[32];
+          tmem_ld32(tbase + b0, g);
+          if (!alive) continue;
+          const int b1 = min(nb0, b0 + 32);
+          float accv[32], e[32];
+#pragma unroll
+          for (int i = 0; i < 32; ++i) accv[i] = __uint_as_float(g[i]);
+          for (int q = 0; q < b0; q += 4) {
+            const float4 eq = *reinterpret_cast<const float4*>(erow + q);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const float4 l = *reinterpret_cast<const float4*>(Lsm + (b0 + i) * kProjMaxBasis + q);
+              accv[i] = fmaf(-l.x, eq.x, accv[i]);
+              accv[i] = fmaf(-l.y, eq.y, accv[i]);
+              accv[i] = fmaf(-l.z, eq.z, accv[i]);
+              accv[i] = fmaf(-l.w, eq.w, accv[i]);
+            }
+          }
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            if (b0 + i < b1) {
+              float v = accv[i];
+#pragma unroll
+              for (int q = 0; q < i; ++q) v = fmaf(-Lsm[(b0 + i) * kProjMaxBasis + b0 + q], e[q], v);
+              e[i] = v * rinv_sm[b0 + i];
+              erow[b0 + i] = e[i];
+              r2 = fmaf(-e[i], e[i], r2);
+            }
+          }
+        }
+        if (alive) {
+          pj.r2[tok] = r2;
+          pj.sqn[tok] = sq;
+          pj.U[tok] = proj_value(__ldg(pj.scores + tok), r2, sq, pj.lambda, pj.tau);
+          pj.cstep[tok] = nb0;
+        }
+        mbar_arrive(&nempty[acc]);
       } else if constexpr (EPI == EPI_F32) {
         float* out = reinterpret_cast<float*>(a.C) + crow + col0;
 #pragma unroll 1
@@ -390,6 +499,58 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       if (acc == 0) acc_phase ^= 1;
     }
   }
+  if constexpr (S::PROJ) {
+    if (warp >= 6) {
+      // ---------------------------------------------------------------- ||v||^2 warps
+      // Warp 6 sums rows 0..63 of each A tile, warp 7 rows 64..127: 8 lanes per row, one
+      // 16-byte chunk each (the 128-byte swizzle only permutes chunks within a row).
+      const int rbase = (warp - 6) * 64;
+      uint32_t stage = 0, phase = 0, nb = 0, nb_phase = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+        TileCoord c = tile_coord(a, t, m_tiles, n_tiles, BN);
+        if (c.skip) continue;
+        float sacc[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) sacc[i] = 0.f;
+        for (int kb = 0; kb < KB; ++kb) {
+          if (!mbar_wait(&full[stage], phase, a.status, abort_flag)) { ok = false; break; }
+          const uint8_t* tileA = sA + stage * S::A_BYTES;
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            const int r = rbase + 4 * i + (lane >> 3);
+            const uint4 u = *reinterpret_cast<const uint4*>(tileA + r * 128 + (lane & 7) * 16);
+            const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+              const float lo = __uint_as_float(w[j] << 16), hi = __uint_as_float(w[j] & 0xFFFF0000u);
+              sacc[i] = fmaf(lo, lo, sacc[i]);
+              sacc[i] = fmaf(hi, hi, sacc[i]);
+            }
+          }
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&empty[stage]);
+          if (++stage == STAGES) { stage = 0; phase ^= 1; }
+        }
+        if (!ok) break;
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          sacc[i] += __shfl_xor_sync(0xffffffffu, sacc[i], 1);
+          sacc[i] += __shfl_xor_sync(0xffffffffu, sacc[i], 2);
+          sacc[i] += __shfl_xor_sync(0xffffffffu, sacc[i], 4);
+        }
+        if (!mbar_wait(&nempty[nb], nb_phase ^ 1, a.status, abort_flag)) break;
+        if ((lane & 7) == 0) {
+#pragma unroll
+          for (int i = 0; i < 16; ++i) sqbuf[nb * kBM + rbase + 4 * i + (lane >> 3)] = sacc[i];
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&nfull[nb]);
+        nb ^= 1;
+        if (nb == 0) nb_phase ^= 1;
+      }
+    }
+  }
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
@@ -426,7 +587,7 @@ bool make_map(CUtensorMap* m, const void* base, long long rows, int K, int box_r
 
 template <int BN, int STAGES, int EPI>
 cudaError_t run(const GemmDesc& d, const KArgs& ka, int num_sms, cudaStream_t st) {
-  using S = Smem<BN, STAGES>;
+  using S = Smem<BN, STAGES, EPI>;
   CUtensorMap ta, tb;
   if (!make_map(&ta, d.A, d.a_rows_total, d.K, kBM)) return cudaErrorInvalidValue;
   if (!make_map(&tb, d.B, d.b_rows_total, d.K, BN)) return cudaErrorInvalidValue;
@@ -440,7 +601,7 @@ cudaError_t run(const GemmDesc& d, const KArgs& ka, int num_sms, cudaStream_t st
   const int tiles = d.batch * ((d.M + kBM - 1) / kBM) * ((d.N + BN - 1) / BN);
   if (tiles == 0) return cudaSuccess;
   const int grid = std::max(1, std::min(tiles, num_sms));
-  kern<<<grid, kThreads, S::TOTAL, st>>>(ta, tb, ka);
+  kern<<<grid, S::THREADS, S::TOTAL, st>>>(ta, tb, ka);
   return cudaGetLastError();
 }
 
@@ -454,8 +615,12 @@ cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t st) {
   const bool scalar_out = d.epi == EPI_SM_STATS || d.epi == EPI_SM_MEAN;   // float / float2 stores
   const bool f32 = d.epi == EPI_F32 || d.epi == EPI_ROPE_F32;
   const long long vec = f32 ? 4 : 8;
-  if (!scalar_out && (d.ldc % vec != 0 || d.c_batch_stride % vec != 0 || (reinterpret_cast<uintptr_t>(d.C) & 15)))
+  if (d.epi == EPI_PROJECT) {      // writes through ProjArgs only (float4 reads of Ec rows)
+    if (d.proj.KP % 4 != 0 || !d.proj.Ec || (reinterpret_cast<uintptr_t>(d.proj.Ec) & 15)) return cudaErrorInvalidValue;
+  } else if (!scalar_out &&
+             (d.ldc % vec != 0 || d.c_batch_stride % vec != 0 || (reinterpret_cast<uintptr_t>(d.C) & 15))) {
     return cudaErrorInvalidValue;
+  }
   if (scalar_out && (!d.stats || (reinterpret_cast<uintptr_t>(d.stats) & 7) || (reinterpret_cast<uintptr_t>(d.C) & 3)))
     return cudaErrorInvalidValue;
   if ((d.epi == EPI_GELU_SPLIT || d.epi == EPI_BIAS_SPLIT) && d.ldc < 2LL * d.N) return cudaErrorInvalidValue;
@@ -468,6 +633,7 @@ cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t st) {
   ka.status = d.status;
   ka.split_kind = d.split_kind; ka.scale = d.scale; ka.aux = d.aux; ka.b_off = d.b_off;
   ka.stats = d.stats; ka.stat_ld = d.stat_ld; ka.col_count = d.col_count;
+  ka.b_base = d.b_base; ka.proj = d.proj;
   switch (d.epi) {
     case EPI_GELU_BF16:
       if (d.N % 256 == 0) return run<256, 4, EPI_GELU_BF16>(d, ka, num_sms, st);
@@ -498,6 +664,9 @@ cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t st) {
       return run<256, 4, EPI_SM_STATS>(d, ka, num_sms, st);
     case EPI_SM_MEAN:
       return run<256, 4, EPI_SM_MEAN>(d, ka, num_sms, st);
+    case EPI_PROJECT:
+      if (d.N > kProjMaxBasis || d.batch < 1) return cudaErrorInvalidValue;
+      return run<128, 4, EPI_PROJECT>(d, ka, num_sms, st);
     case EPI_F32:
       return run<128, 6, EPI_F32>(d, ka, num_sms, st);
     default:

@@ -15,8 +15,26 @@ namespace mapk {
 // EPI_SM_STATS / EPI_SM_MEAN are the two passes of Eq. 3 over a logits tile (rows =
 // visual tokens, columns = question tokens): per-column max / sum of exp over each
 // 32-row slab, then per-row mean over columns of exp(l - max) / sum.
+// EPI_PROJECT: rows = visual tokens, columns = the R0 basis tokens' rows (Gram entries
+// <v_n, v_r>); the epilogue solves for the tokens' Cholesky coordinates against the R0
+// basis (L staged in shared memory), and two extra warps sum ||v_n||^2 from the same
+// shared-memory tiles.  It writes the exact residual, value and coordinate cache of every
+// candidate token (see select.cu).
 enum Epi { EPI_GELU_BF16 = 0, EPI_BIAS_BF16 = 1, EPI_ROPE_F32 = 2, EPI_F32 = 3, EPI_GELU_SPLIT = 4,
-           EPI_BIAS_SPLIT = 5, EPI_ROPE_SPLIT3 = 6, EPI_SM_STATS = 7, EPI_SM_MEAN = 8 };
+           EPI_BIAS_SPLIT = 5, EPI_ROPE_SPLIT3 = 6, EPI_SM_STATS = 7, EPI_SM_MEAN = 8, EPI_PROJECT = 9 };
+
+// Inputs and outputs of the EPI_PROJECT epilogue (device pointers).
+struct ProjArgs {
+  const uint8_t* state;        // [B, N] 0 = candidate
+  const float* scores;         // [B, N] p_hat
+  float* Ec; int KP;           // coordinate cache rows [B, N, KP]
+  const int32_t* basis_tok;    // [B, Kcap]
+  const float* rnorm;          // [B, Kcap]
+  const int32_t* nbasis;       // [B] basis size after R0 (<= 128)
+  int Kcap;
+  float lambda, tau;
+  float* r2; float* U; float* sqn; int32_t* cstep;   // [B, N] outputs
+};
 
 // Batched C = epi(A @ B^T): A rows [batch][a_row_stride] x K, B rows [batch][b_row_stride] x K
 // (both bf16, K contiguous, tightly packed 2D arrays of a_rows_total / b_rows_total rows).
@@ -40,6 +58,9 @@ struct GemmDesc {
   //               [batch][M] when one column tile covers all columns
   float2* stats = nullptr; int stat_ld = 0;
   const int* col_count = nullptr;       // per-batch number of valid columns (M_b)
+  // B rows at b * b_row_stride + b_base
+  int b_base = 0;
+  ProjArgs proj{};
 };
 
 // Returns cudaSuccess, or an error for an unsupported shape (cudaErrorInvalidValue).

@@ -147,7 +147,7 @@ __global__ void __launch_bounds__(1024) sel_init_kernel(SelState s) {
   __shared__ uint32_t hist[256], bc[2];
   __shared__ int cnt;
   for (int i = threadIdx.x; i < s.N; i += blockDim.x) {
-    const float p = s.scores[base + i], sq = s.sqn[base + i];
+    const float p = s.scores[base + i], sq = s.sqn ? s.sqn[base + i] : 0.f;
     s.U[base + i] = sel_value(p, sq, sq, s.lambda, s.tau);
     s.r2[base + i] = sq;
     s.cstep[base + i] = 0;
@@ -313,11 +313,15 @@ __global__ void __launch_bounds__(256, 1) sel_greedy_kernel(SelState s) {
   int c0 = nb, mine = nb;                            // cached coordinates; valid coordinates at the end
   bool alive = false;
   if (tok >= 0) {
-    r2 = s.r2[base + tok];
-    sq = s.sqn[base + tok];
     p = s.scores[base + tok];
     alive = s.state[base + tok] == 0;
     c0 = min(s.cstep[base + tok], nb);
+    if (s.diag_sq && c0 == 0) {
+      sq = r2 = Gr[slot];                            // <v, v> from the Gram block
+    } else {
+      r2 = s.r2[base + tok];
+      sq = s.sqn[base + tok];
+    }
     if constexpr (SMEM) {
       const float4* g = reinterpret_cast<const float4*>(s.Ec + (base + tok) * KP);
       int q = 0;
@@ -487,6 +491,18 @@ __global__ void __launch_bounds__(256, 1) sel_greedy_kernel(SelState s) {
   }
 }
 
+// ------------------------------------------------------------------ projection set-up
+// After the R0 rounds: gather every R0 basis row (no active tokens) for the projection.
+__global__ void sel_proj_prep_kernel(SelState s) {
+  const int b = blockIdx.x;
+  for (int i = threadIdx.x; i < s.S; i += blockDim.x) s.aslot[static_cast<long long>(b) * s.S + i] = -1;
+  if (threadIdx.x == 0) {
+    s.gb_lo[b] = s.nb_gathered[b];
+    s.gb_hi[b] = s.nbasis[b];
+    s.nb_gathered[b] = s.nbasis[b];
+  }
+}
+
 // ------------------------------------------------------------------ outputs
 // keep = picks sorted ascending; pick_order = picks.
 __global__ void sel_finalize_kernel(const int32_t* picks, int K, int32_t* keep, int32_t* order) {
@@ -570,6 +586,16 @@ cudaError_t launch_sel_finalize(const int32_t* picks, int B, int K, int32_t* kee
 
 cudaError_t launch_sel_copy_r0(const int32_t* r0, int B, int K, int32_t* picks, cudaStream_t st) {
   sel_copy_r0_kernel<<<B, 256, 0, st>>>(r0, K, picks);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_sel_proj_prep(const SelState& s, cudaStream_t st) {
+  sel_proj_prep_kernel<<<s.B, 256, 0, st>>>(s);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_sel_gather(const SelState& s, cudaStream_t st) {
+  sel_gather_kernel<<<dim3(s.S + s.K, s.B), 128, 0, st>>>(s);
   return cudaGetLastError();
 }
 

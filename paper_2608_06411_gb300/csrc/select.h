@@ -31,6 +31,8 @@ struct SelState {
   void* Vg;                       // [B, R, D] bf16 gathered rows
   float* G;                       // [B, S, R] Gram block
   int32_t* done_count;            // images finished
+  int diag_sq;                    // 1: a token evaluated for the first time takes ||v||^2 from
+                                  // the Gram block's diagonal (before the R0 projection)
   int* status;
 };
 
@@ -43,5 +45,8 @@ cudaError_t launch_sel_greedy(const SelState& s, cudaStream_t st);
 cudaError_t launch_sel_finalize(const int32_t* picks, int B, int K, int32_t* keep, int32_t* order, cudaStream_t st);
 cudaError_t launch_sel_copy_r0(const int32_t* r0, int B, int K, int32_t* picks, cudaStream_t st);
 cudaError_t launch_sel_identity(int B, int N, int32_t* keep, int32_t* order, cudaStream_t st);
+// Queues the R0 basis rows for gathering into Vg (rows S + beta) ahead of the projection.
+cudaError_t launch_sel_proj_prep(const SelState& s, cudaStream_t st);
+cudaError_t launch_sel_gather(const SelState& s, cudaStream_t st);
 
 }  // namespace mapk
