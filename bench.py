@@ -196,6 +196,9 @@ def main():
     ap.add_argument("--cpu-images", type=int, default=1, help="oracle images timed for cpu_baseline")
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--batch", type=int, default=WORKLOAD.B, help="images per GPU (profiling on a smaller case)")
+    ap.add_argument("--minimal", action="store_true",
+                    help="time the steps only (no clock sampling, latency, e2e or CPU baseline): for ncu runs")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)
@@ -213,7 +216,7 @@ def main():
         dist.init_process_group("nccl", device_id=dev)
         pg = dist
 
-    B, N, K, D = WORKLOAD.B, WORKLOAD.N, WORKLOAD.K, WORKLOAD.D
+    B, N, K, D = args.batch, WORKLOAD.N, WORKLOAD.K, WORKLOAD.D
     first, B = image_range(B * ws, ws, rank)              # weak scaling: 64 images per rank
     vis_np, text_np, lens = W.make_batch(WORKLOAD, B=B, first_image=first, threads=min(16, _CORES))
     w = W.make_weights(DIMS)
@@ -230,16 +233,18 @@ def main():
         ctx.prune(text, vis, lens, K, out, keep, scores)
 
     sampler = ClockSampler(local)          # started early: nvidia-smi start-up stalls the device briefly
-    sampler.start()
+    if not args.minimal:
+        sampler.start()
     for _ in range(args.warmup):
         step()
     torch.cuda.synchronize()
     ctx.check()
-    time.sleep(1.0)
-    for _ in range(2):
-        step()
-    torch.cuda.synchronize()
-    sampler.lines.clear()
+    if not args.minimal:
+        time.sleep(1.0)
+        for _ in range(2):
+            step()
+        torch.cuda.synchronize()
+        sampler.lines.clear()
 
     # ---------------------------------------------------------------- timed region
     ctx.set_timing(True)
@@ -281,6 +286,19 @@ def main():
     flops, bytes_ = algorithmic(DIMS, N, K, lens)
     t_roof = max(flops / (bf16_burst * 1e12), bytes_ / (hbm * 1e9))
     step_s = total_ms / 1000.0 / args.steps
+
+    if args.minimal:
+        if rank == 0:
+            print(json.dumps({"metric": METRIC, "value": B * args.steps * ws / (total_ms / 1000.0), "unit": "images/s",
+                              "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
+                              "ms_per_step": total_ms / args.steps, "higher_is_better": True, "scaling": "weak",
+                              "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+                              "config": {"workload": WORKLOAD.name, "B": B, "minimal": True},
+                              "gpu_launches": int(launches)}))
+        ctx.close()
+        if pg:
+            pg.destroy_process_group()
+        return 0
 
     # ---------------------------------------------------------------- single-image latency (N=2880, k=160)
     w1 = W.WORKLOADS["c1"]

@@ -265,3 +265,75 @@ def test_llava_next_shape_end_to_end():
     out = ctx.gather(dev_bits(vis), torch.from_numpy(keep).to(DEV))
     torch.cuda.synchronize()
     np.testing.assert_array_equal(out.cpu().numpy().view(np.uint16), O.gather(vis, keep))
+
+
+# ------------------------------------------------------------------ remaining workload configs
+
+def _batch_parity(wl, sample, K, K0=None, **ctxkw):
+    """GPU scores for the whole batch against the oracle on `sample` images; then GPU
+    selection on the batch with the oracle's scores on the sampled images."""
+    dims = W.PredictorDims(D=wl.D)
+    ctx, w = make_ctx(dims, **ctxkw)
+    vis, text, lens = W.make_batch(wl, threads=8)
+    vis_t, text_t = dev_bits(vis), dev_bits(text)
+    p = ctx.score(text_t, vis_t, lens)
+    torch.cuda.synchronize()
+    ctx.check()
+    p_all = p.cpu().numpy().copy()
+    off = np.concatenate([[0], np.cumsum(lens)])
+    for b in sample:
+        p_ref = O.map_score(text[off[b]:off[b + 1]], vis[b:b + 1], [lens[b]], w)[0]
+        assert P.score_rel_err(p_all[b], p_ref) <= 1e-3, f"image {b}"
+        p_all[b] = p_ref.astype(np.float32)           # both sides select on the oracle's scores
+    keep, order = run_select(ctx, p_all, vis, K)
+    K0 = O.resolve_k0(K) if K0 is None else K0
+    for b in sample:
+        rep = P.check_selection(p_all[b].astype(np.float64), O.bf16_bits_to_f64(vis[b]), K, K0, order[b], keep[b])
+        assert rep["ok"], f"image {b}: {rep['reason']}"
+    out = ctx.gather(vis_t, torch.from_numpy(keep).to(DEV))
+    torch.cuda.synchronize()
+    for b in sample:
+        np.testing.assert_array_equal(out[b].cpu().numpy().view(np.uint16), vis[b][keep[b]])
+    return lens
+
+
+def test_batched_serving_config_sampled():
+    """64 images, N = 2880, k = 160, ragged questions, near-duplicate images (b % 10 == 0)."""
+    wl = W.WORKLOADS["c3"]
+    _batch_parity(wl, sample=[0, 7, 63], K=wl.K)
+
+
+def test_high_token_config_sampled():
+    """16 images, N = 7290, D = 3584, k = 405, questions up to 512 tokens (two column tiles
+    in Eq. 3) and K0 = 202 (no projection pass; coordinates in global memory)."""
+    wl = W.WORKLOADS["c4"]
+    lens = W.make_lens(wl)
+    long_q = int(np.argmax(lens))
+    assert lens[long_q] > 256
+    _batch_parity(wl, sample=sorted({0, long_q}), K=wl.K)
+
+
+_SWEEP = {}
+
+
+def _sweep_inputs():
+    if not _SWEEP:
+        wl = W.WORKLOADS["c2"]
+        w = W.make_weights(W.PredictorDims())
+        vis = W.make_image(wl, 0)[None]
+        text = W.make_text(wl, 0, wl.m_lo)
+        _SWEEP["v"] = (vis, O.map_score(text, vis, [wl.m_lo], w).astype(np.float32))
+    return _SWEEP["v"]
+
+
+@pytest.mark.parametrize("K,lam,k0_frac", [(64, 1.0, 0.5), (128, 1.0, 0.5), (320, 1.0, 0.5), (640, 1.0, 0.5),
+                                           (160, 0.0, 0.5), (160, 0.5, 0.5), (160, 2.0, 0.5),
+                                           (160, 1.0, 0.0), (160, 1.0, 0.25), (160, 1.0, 1.0)])
+def test_retention_sweep_config(K, lam, k0_frac):
+    """N = 2880 LLaVA-NeXT image: retained budgets and diversity weights of the sweep."""
+    wl = W.WORKLOADS["c2"]
+    dims = W.PredictorDims()
+    ctx, w = make_ctx(dims, lam=lam, k0_frac=k0_frac)
+    vis, p32 = _sweep_inputs()
+    keep, order = run_select(ctx, p32, vis, K)
+    assert_selection(p32, vis, K, O.resolve_k0(K, k0_frac), keep, order, lam=lam)
