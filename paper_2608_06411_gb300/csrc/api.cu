@@ -361,7 +361,7 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, 
   MAP_TRY(ensure(c->sr0, static_cast<size_t>(B) * K * 4));
   MAP_TRY(ensure(c->sbt, static_cast<size_t>(B) * K * 4));
   MAP_TRY(ensure(c->srn, static_cast<size_t>(B) * K * 4));
-  MAP_TRY(ensure(c->ssmall, static_cast<size_t>(B) * 4 * 16 + 16 * 256));
+  MAP_TRY(ensure(c->ssmall, static_cast<size_t>(B) * 4 * 16 + 20 * 256));
   MAP_TRY(ensure(c->stheta, static_cast<size_t>(B) * 8));
   MAP_TRY(ensure(c->saslot, static_cast<size_t>(B) * S * 4));
   s.sqn = static_cast<float*>(c->sqn.p);
@@ -382,6 +382,7 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, 
   s.nlimit = carve<int32_t>(sm, B);
   s.gb_lo = carve<int32_t>(sm, B);
   s.gb_hi = carve<int32_t>(sm, B);
+  s.gbase = carve<int32_t>(sm, B);
   s.done_count = carve<int32_t>(sm, 1);
   s.theta = static_cast<uint64_t*>(c->stheta.p);
   s.aslot = static_cast<int32_t*>(c->saslot.p);
@@ -443,6 +444,8 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, 
       pd.proj.lambda = g.lambda; pd.proj.tau = g.tau;
       pd.proj.r2 = s.r2; pd.proj.U = s.U; pd.proj.sqn = static_cast<float*>(c->sqn.p); pd.proj.cstep = s.cstep;
       MAP_TRY(gemm(c, pd, st));
+      ++c->counters.launches;
+      CU_TRY(mapk::launch_sel_proj_done(s, st));
       burst = 6;
     }
     for (;;) {

@@ -5,7 +5,8 @@
 // epilogue (section "Cross-Modal Attention Distillation"), and the Gram blocks
 // <v_i, v_j> that the diversity term of Eq. 4 needs.
 //
-// Structure (one CTA per SM, 6 warps; 8 for EPI_PROJECT):
+// Structure (one CTA per SM, 6 warps; 8 for EPI_PROJECT; the BN = 256 predictor layers run
+// as 2-CTA clusters on vertically adjacent tiles that share one multicast B tile):
 //   warp 0      one thread issues TMA loads of 128x64 (A) and BNx64 (B) bf16 tiles, 128-byte
 //               swizzled, into a STAGES-deep shared-memory ring (mbarrier full/empty).
 //   warp 1      allocates TMEM (2 accumulators x BN fp32 columns); one thread issues
@@ -82,23 +83,33 @@ __device__ __forceinline__ float proj_value(float p, float r2, float sq, float l
 
 struct TileCoord { int b, m_blk, n_blk; bool skip; };
 
-__device__ __forceinline__ TileCoord tile_coord(const KArgs& a, int t, int m_tiles, int n_tiles, int BN) {
+// Work unit t -> tile.  With PAIR the unit is a pair of vertically adjacent M tiles with the
+// same N tile, processed by the two CTAs of a cluster (rank 0 the upper, rank 1 the lower).
+template <bool PAIR>
+__device__ __forceinline__ TileCoord tile_coord(const KArgs& a, int t, int m_units, int n_tiles, int BN,
+                                                uint32_t crank) {
   TileCoord c;
-  int per = m_tiles * n_tiles;
+  int per = m_units * n_tiles;
   c.b = t / per;
   int rem = t - c.b * per;
-  c.m_blk = rem / n_tiles;
-  c.n_blk = rem - c.m_blk * n_tiles;
+  const int mu = rem / n_tiles;
+  c.n_blk = rem - mu * n_tiles;
+  c.m_blk = PAIR ? 2 * mu + static_cast<int>(crank) : mu;
   int lim = a.n_limit ? min(a.N, __ldg(a.n_limit + c.b)) : a.N;
   c.skip = c.n_blk * BN >= lim;
   return c;
 }
 
-template <int BN, int STAGES, int EPI>
+template <int BN, int STAGES, int EPI, bool PAIR>
 __global__ void __launch_bounds__(Smem<BN, STAGES, EPI>::THREADS, 1)
 gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, KArgs a) {
   using S = Smem<BN, STAGES, EPI>;
   constexpr uint32_t IDESC = idesc_bf16(kBM, BN);
+  // PAIR: launched as 2-CTA clusters; each CTA loads half of the shared B tile and multicasts
+  // it to both, and every MMA commit releases the stage in both CTAs.
+  const uint32_t crank = PAIR ? cluster_ctarank() : 0u;
+  const int unit0 = PAIR ? static_cast<int>(blockIdx.x >> 1) : static_cast<int>(blockIdx.x);
+  const int units_step = PAIR ? static_cast<int>(gridDim.x >> 1) : static_cast<int>(gridDim.x);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
@@ -120,7 +131,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
-    for (int s = 0; s < STAGES; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], S::PROJ ? 3 : 1); }
+    for (int s = 0; s < STAGES; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], S::PROJ ? 3 : (PAIR ? 2 : 1)); }
     for (int i = 0; i < 2; ++i) { mbar_init(&tfull[i], 1); mbar_init(&tempty[i], 128); }
     mbar_init(drain, 1);
     if constexpr (S::PROJ) {
@@ -132,13 +143,15 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   }
   if (warp == 0 && lane == 0) { tma_prefetch_desc(&tmA); tma_prefetch_desc(&tmB); }
   if (warp == 1) { tmem_alloc(tmem_slot, S::TMEM_COLS); tmem_relinquish(); }
-  __syncthreads();
+  if constexpr (PAIR) cluster_sync();             // peer barriers initialised before any multicast
+  else __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
   const int m_tiles = (a.M + kBM - 1) / kBM;
+  const int m_units = PAIR ? (m_tiles + 1) / 2 : m_tiles;
   const int n_tiles = (a.N + BN - 1) / BN;
-  const int total = a.batch * m_tiles * n_tiles;
+  const int total = a.batch * m_units * n_tiles;
   const int KB = a.K / kBK;
 
   if (warp == 0) {
@@ -149,8 +162,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
 #pragma unroll
       for (int s = 0; s < STAGES; ++s) last_par[s] = -1;
       bool ok = true;
-      for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
-        TileCoord c = tile_coord(a, t, m_tiles, n_tiles, BN);
+      for (int t = unit0; t < total && ok; t += units_step) {
+        TileCoord c = tile_coord<PAIR>(a, t, m_units, n_tiles, BN, crank);
         if (c.skip) continue;
         const int arow = c.b * a.a_row_stride + c.m_blk * kBM;
         const int brow = (a.b_off ? __ldg(a.b_off + c.b) : c.b * a.b_row_stride + a.b_base) + c.n_blk * BN;
@@ -158,7 +171,12 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           if (!mbar_wait(&empty[stage], phase ^ 1, a.status, abort_flag)) { ok = false; break; }
           mbar_arrive_expect_tx(&full[stage], S::STAGE_BYTES);
           tma_load_2d(sA + stage * S::A_BYTES, &tmA, &full[stage], kb * kBK, arow);
-          tma_load_2d(sB + stage * S::B_BYTES, &tmB, &full[stage], kb * kBK, brow);
+          if constexpr (PAIR) {
+            tma_load_2d_mc(sB + stage * S::B_BYTES + crank * (S::B_BYTES / 2), &tmB, &full[stage], kb * kBK,
+                           brow + static_cast<int>(crank) * (BN / 2), static_cast<uint16_t>(3));
+          } else {
+            tma_load_2d(sB + stage * S::B_BYTES, &tmB, &full[stage], kb * kBK, brow);
+          }
           last_par[stage] = static_cast<int>(phase);
           if (++stage == STAGES) { stage = 0; phase ^= 1; }
         }
@@ -174,8 +192,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       // ---------------------------------------------------------------- MMA issuer
       uint32_t stage = 0, phase = 0, acc = 0, acc_phase = 0;
       bool issued = false, ok = true;
-      for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
-        TileCoord c = tile_coord(a, t, m_tiles, n_tiles, BN);
+      for (int t = unit0; t < total && ok; t += units_step) {
+        TileCoord c = tile_coord<PAIR>(a, t, m_units, n_tiles, BN, crank);
         if (c.skip) continue;
         if (!mbar_wait(&tempty[acc], acc_phase ^ 1, a.status, abort_flag)) break;
         tc_fence_after();
@@ -188,7 +206,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
 #pragma unroll
           for (int k = 0; k < kBK / 16; ++k)
             umma_bf16(d_tmem, desc_sw128(a0 + k * 32), desc_sw128(b0 + k * 32), IDESC, (kb | k) != 0);
-          umma_commit(&empty[stage]);
+          if constexpr (PAIR) umma_commit_mc(&empty[stage], static_cast<uint16_t>(3));
+          else umma_commit(&empty[stage]);
           issued = true;
           if (++stage == STAGES) { stage = 0; phase ^= 1; }
         }
@@ -211,8 +230,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     int staged_b = -1;                             // EPI_PROJECT: image whose L is in shared memory
     uint32_t eg_phase = 0;
     bool eg_ok = true;
-    for (int t = blockIdx.x; t < total && eg_ok; t += gridDim.x) {
-      TileCoord c = tile_coord(a, t, m_tiles, n_tiles, BN);
+    for (int t = unit0; t < total && eg_ok; t += units_step) {
+      TileCoord c = tile_coord<PAIR>(a, t, m_units, n_tiles, BN, crank);
       if (c.skip) continue;
       if constexpr (S::PROJ) {
         if (c.b != staged_b) {                     // stage L and 1/r of this image's R0 basis
@@ -507,8 +526,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       const int rbase = (warp - 6) * 64;
       uint32_t stage = 0, phase = 0, nb = 0, nb_phase = 0;
       bool ok = true;
-      for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
-        TileCoord c = tile_coord(a, t, m_tiles, n_tiles, BN);
+      for (int t = unit0; t < total && ok; t += units_step) {
+        TileCoord c = tile_coord<PAIR>(a, t, m_units, n_tiles, BN, crank);
         if (c.skip) continue;
         float sacc[16];
 #pragma unroll
@@ -551,7 +570,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       }
     }
   }
-  __syncthreads();
+  if constexpr (PAIR) cluster_sync();             // no multicast or remote arrive still in flight
+  else __syncthreads();
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem_base, S::TMEM_COLS);
@@ -585,20 +605,39 @@ bool make_map(CUtensorMap* m, const void* base, long long rows, int K, int box_r
   return r == CUDA_SUCCESS;
 }
 
-template <int BN, int STAGES, int EPI>
+template <int BN, int STAGES, int EPI, bool PAIR = false>
 cudaError_t run(const GemmDesc& d, const KArgs& ka, int num_sms, cudaStream_t st) {
   using S = Smem<BN, STAGES, EPI>;
   CUtensorMap ta, tb;
   if (!make_map(&ta, d.A, d.a_rows_total, d.K, kBM)) return cudaErrorInvalidValue;
-  if (!make_map(&tb, d.B, d.b_rows_total, d.K, BN)) return cudaErrorInvalidValue;
-  auto kern = gemm_tc_kernel<BN, STAGES, EPI>;
+  if (!make_map(&tb, d.B, d.b_rows_total, d.K, PAIR ? BN / 2 : BN)) return cudaErrorInvalidValue;
+  auto kern = gemm_tc_kernel<BN, STAGES, EPI, PAIR>;
   static bool attr_set = false;
   if (!attr_set) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, S::TOTAL);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  const int tiles = d.batch * ((d.M + kBM - 1) / kBM) * ((d.N + BN - 1) / BN);
+  const int m_tiles = (d.M + kBM - 1) / kBM, n_tiles = (d.N + BN - 1) / BN;
+  if (PAIR) {
+    const int units = d.batch * ((m_tiles + 1) / 2) * n_tiles;
+    if (units == 0) return cudaSuccess;
+    const int grid = 2 * std::max(1, std::min(units, num_sms / 2));
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(S::THREADS);
+    cfg.dynamicSmemBytes = S::TOTAL;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, ta, tb, ka);
+  }
+  const int tiles = d.batch * m_tiles * n_tiles;
   if (tiles == 0) return cudaSuccess;
   const int grid = std::max(1, std::min(tiles, num_sms));
   kern<<<grid, S::THREADS, S::TOTAL, st>>>(ta, tb, ka);
@@ -649,11 +688,11 @@ cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t st) {
       if (d.N == 256) return run<256, 4, EPI_ROPE_F32>(d, ka, num_sms, st);
       return cudaErrorInvalidValue;
     case EPI_GELU_SPLIT:
-      if (d.N % 256 == 0) return run<256, 4, EPI_GELU_SPLIT>(d, ka, num_sms, st);
+      if (d.N % 256 == 0) return run<256, 4, EPI_GELU_SPLIT, true>(d, ka, num_sms, st);
       if (d.N % 64 == 0) return run<64, 8, EPI_GELU_SPLIT>(d, ka, num_sms, st);
       return cudaErrorInvalidValue;
     case EPI_BIAS_SPLIT:
-      if (d.N % 256 == 0) return run<256, 4, EPI_BIAS_SPLIT>(d, ka, num_sms, st);
+      if (d.N % 256 == 0) return run<256, 4, EPI_BIAS_SPLIT, true>(d, ka, num_sms, st);
       if (d.N % 64 == 0) return run<64, 8, EPI_BIAS_SPLIT>(d, ka, num_sms, st);
       return cudaErrorInvalidValue;
     case EPI_ROPE_SPLIT3:

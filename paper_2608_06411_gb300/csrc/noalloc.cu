@@ -131,6 +131,7 @@ extern "C" int map_select_noalloc(map_ctx* ctx, const float* scores, const void*
   s.nlimit = cv.take<int32_t>(B);
   s.gb_lo = cv.take<int32_t>(B);
   s.gb_hi = cv.take<int32_t>(B);
+  s.gbase = cv.take<int32_t>(B);
   s.done_count = cv.take<int32_t>(1);
   s.theta = cv.take<uint64_t>(B);
   s.aslot = cv.take<int32_t>(static_cast<size_t>(B) * S);

@@ -156,7 +156,7 @@ __global__ void __launch_bounds__(1024) sel_init_kernel(SelState s) {
   }
   if (threadIdx.x == 0) {
     s.npicks[b] = 0; s.nbasis[b] = 0; s.nb_gathered[b] = 0; s.done[b] = 0; s.nlimit[b] = 0;
-    s.gb_lo[b] = 0; s.gb_hi[b] = 0;
+    s.gb_lo[b] = 0; s.gb_hi[b] = 0; s.gbase[b] = 0;
     cnt = 0;
   }
   __syncthreads();
@@ -220,7 +220,7 @@ __global__ void __launch_bounds__(1024) sel_choose_kernel(SelState s) {
   if (threadIdx.x == 0) {
     s.mode[b] = mode;
     s.theta[b] = theta;
-    s.nlimit[b] = S + nb;
+    s.nlimit[b] = S + nb - s.gbase[b];
     s.gb_lo[b] = s.nb_gathered[b];
     s.gb_hi[b] = nb;
     s.nb_gathered[b] = nb;
@@ -228,22 +228,28 @@ __global__ void __launch_bounds__(1024) sel_choose_kernel(SelState s) {
 }
 
 // Copies the rows the Gram block needs into Vg: row r < S <- token aslot[r];
-// row S + beta <- basis token beta for the basis vectors added since the last round.
+// row S + beta - gbase <- basis token beta for the basis vectors added since the last round.
+// kGatherCtas CTAs per image, each walking every kGatherCtas-th row; finished images exit.
+constexpr int kGatherCtas = 64;
+
 __global__ void __launch_bounds__(128) sel_gather_kernel(SelState s) {
-  const int b = blockIdx.y, r = blockIdx.x;
+  const int b = blockIdx.y;
   if (s.done[b]) return;
-  int src = -1;
-  if (r < s.S) {
-    src = s.aslot[static_cast<long long>(b) * s.S + r];
-  } else {
-    const int beta = r - s.S;
-    if (beta >= s.gb_lo[b] && beta < s.gb_hi[b]) src = s.basis_tok[static_cast<long long>(b) * s.K + beta];
-  }
-  if (src < 0) return;
+  const int gb = s.gbase[b], lo = s.gb_lo[b], hi = s.gb_hi[b];
   const int vec = s.D / 8;
-  const uint4* V = reinterpret_cast<const uint4*>(s.V) + (static_cast<long long>(b) * s.N + src) * vec;
-  uint4* dst = reinterpret_cast<uint4*>(s.Vg) + (static_cast<long long>(b) * s.R + r) * vec;
-  for (int c = threadIdx.x; c < vec; c += blockDim.x) dst[c] = __ldg(V + c);
+  for (int r = blockIdx.x; r < s.S + (hi - gb); r += kGatherCtas) {
+    int src = -1;
+    if (r < s.S) {
+      src = s.aslot[static_cast<long long>(b) * s.S + r];
+    } else {
+      const int beta = r - s.S + gb;
+      if (beta >= lo && beta < hi) src = s.basis_tok[static_cast<long long>(b) * s.K + beta];
+    }
+    if (src < 0) continue;                               // uniform in the CTA
+    const uint4* V = reinterpret_cast<const uint4*>(s.V) + (static_cast<long long>(b) * s.N + src) * vec;
+    uint4* dst = reinterpret_cast<uint4*>(s.Vg) + (static_cast<long long>(b) * s.R + r) * vec;
+    for (int c = threadIdx.x; c < vec; c += blockDim.x) dst[c] = __ldg(V + c);
+  }
 }
 
 // ------------------------------------------------------------------ greedy
@@ -306,6 +312,7 @@ __global__ void __launch_bounds__(256, 1) sel_greedy_kernel(SelState s) {
   const float* Gb = s.G + static_cast<long long>(b) * S * R;
   const float* Gr = Gb + static_cast<long long>(slot) * R;
   int nb = s.nbasis[b], np = s.npicks[b];
+  const int gbase = s.gbase[b];
   const bool forced = s.mode[b] == 1;
   const uint64_t th48 = theta48(s.theta[b]);
 
@@ -376,7 +383,7 @@ __global__ void __launch_bounds__(256, 1) sel_greedy_kernel(SelState s) {
     if (tok < 0 || b1 <= c0) continue;
     float acc[kChunk], e[kChunk];
 #pragma unroll
-    for (int i = 0; i < kChunk; ++i) acc[i] = (b0 + i < b1 && b0 + i >= c0) ? Gr[S + b0 + i] : 0.f;
+    for (int i = 0; i < kChunk; ++i) acc[i] = (b0 + i < b1 && b0 + i >= c0) ? Gr[S + b0 + i - gbase] : 0.f;
     for (int q = 0; q < b0; q += 4) {
       float4 eq;
       if constexpr (SMEM) {
@@ -503,6 +510,14 @@ __global__ void sel_proj_prep_kernel(SelState s) {
   }
 }
 
+__global__ void sel_proj_done_kernel(SelState s) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b < s.B) {
+    s.gbase[b] = s.nbasis[b];
+    s.nb_gathered[b] = s.nbasis[b];
+  }
+}
+
 // ------------------------------------------------------------------ outputs
 // keep = picks sorted ascending; pick_order = picks.
 __global__ void sel_finalize_kernel(const int32_t* picks, int K, int32_t* keep, int32_t* order) {
@@ -558,7 +573,7 @@ cudaError_t launch_sel_choose(const SelState& s, cudaStream_t st) {
   if (e != cudaSuccess) return e;
   sel_choose_kernel<<<s.B, 1024, sm, st>>>(s);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  sel_gather_kernel<<<dim3(s.S + s.K, s.B), 128, 0, st>>>(s);
+  sel_gather_kernel<<<dim3(kGatherCtas, s.B), 128, 0, st>>>(s);
   return cudaGetLastError();
 }
 
@@ -595,7 +610,12 @@ cudaError_t launch_sel_proj_prep(const SelState& s, cudaStream_t st) {
 }
 
 cudaError_t launch_sel_gather(const SelState& s, cudaStream_t st) {
-  sel_gather_kernel<<<dim3(s.S + s.K, s.B), 128, 0, st>>>(s);
+  sel_gather_kernel<<<dim3(kGatherCtas, s.B), 128, 0, st>>>(s);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_sel_proj_done(const SelState& s, cudaStream_t st) {
+  sel_proj_done_kernel<<<(s.B + 127) / 128, 128, 0, st>>>(s);
   return cudaGetLastError();
 }
 

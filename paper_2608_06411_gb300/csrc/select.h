@@ -26,6 +26,9 @@ struct SelState {
   int32_t* npicks; int32_t* nbasis; int32_t* nb_gathered; int32_t* done; int32_t* mode;
   int32_t* nlimit;                // [B] Gram block columns (S + nbasis), 0 when done
   int32_t* gb_lo; int32_t* gb_hi;  // [B] basis rows to gather this round
+  int32_t* gbase;                 // [B] first basis vector whose row is in Vg (row S + beta - gbase);
+                                  // after the R0 projection every candidate's coordinates on the
+                                  // R0 basis are cached, so those columns are not recomputed
   uint64_t* theta;                // [B] key of the best candidate outside A (0: none)
   int32_t* aslot;                 // [B, S] active tokens (-1 empty)
   void* Vg;                       // [B, R, D] bf16 gathered rows
@@ -48,5 +51,7 @@ cudaError_t launch_sel_identity(int B, int N, int32_t* keep, int32_t* order, cud
 // Queues the R0 basis rows for gathering into Vg (rows S + beta) ahead of the projection.
 cudaError_t launch_sel_proj_prep(const SelState& s, cudaStream_t st);
 cudaError_t launch_sel_gather(const SelState& s, cudaStream_t st);
+// After the projection: later Gram blocks start at the first basis vector past R0.
+cudaError_t launch_sel_proj_done(const SelState& s, cudaStream_t st);
 
 }  // namespace mapk
