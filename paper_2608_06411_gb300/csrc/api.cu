@@ -420,16 +420,13 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, 
     long long rounds = 0;
     int burst = (K0 + S - 1) / S + 6;   // rounds queued per host check; finished images skip
     if (project) {
-      s.diag_sq = 1;                    // R0 tokens take ||v||^2 from the Gram diagonal
-      for (int r = 0; r < (K0 + S - 1) / S; ++r) {
-        c->counters.launches += 3;
-        CU_TRY(mapk::launch_sel_choose(s, st));
-        MAP_TRY(gemm(c, d, st));
-        CU_TRY(mapk::launch_sel_greedy(s, st));
-        ++rounds;
-        ++c->counters.select_rounds;
-      }
-      s.diag_sq = 0;
+      // R0: gather its rows, G[R0, R0] on the tensor cores, then its Cholesky factor.
+      c->counters.launches += 3;
+      CU_TRY(mapk::launch_sel_choose(s, st));
+      MAP_TRY(gemm(c, d, st));
+      CU_TRY(mapk::launch_sel_chol(s, st));
+      ++rounds;
+      ++c->counters.select_rounds;
       c->counters.launches += 2;
       CU_TRY(mapk::launch_sel_proj_prep(s, st));
       CU_TRY(mapk::launch_sel_gather(s, st));
@@ -450,7 +447,7 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, 
     }
     for (;;) {
       for (int r = 0; r < burst; ++r) {
-        c->counters.launches += 3;
+        c->counters.launches += 4;
         CU_TRY(mapk::launch_sel_choose(s, st));
         MAP_TRY(gemm(c, d, st));
         CU_TRY(mapk::launch_sel_greedy(s, st));

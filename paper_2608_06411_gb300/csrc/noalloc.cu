@@ -164,7 +164,7 @@ extern "C" int map_select_noalloc(map_ctx* ctx, const float* scores, const void*
     int burst = (K0 + S - 1) / S + 6;
     for (;;) {
       for (int r = 0; r < burst; ++r) {
-        *v.launches += 4;
+        *v.launches += 5;
         if ((rc = rc_of(mapk::launch_sel_choose(s, st))) != MAP_OK) return rc;
         cudaError_t e = mapk::launch_gemm(d, v.num_sms, st);
         if (e == cudaErrorInvalidValue) return MAP_EUNSUPPORTED;

@@ -220,7 +220,7 @@ __global__ void __launch_bounds__(1024) sel_choose_kernel(SelState s) {
   if (threadIdx.x == 0) {
     s.mode[b] = mode;
     s.theta[b] = theta;
-    s.nlimit[b] = S + nb - s.gbase[b];
+    s.nlimit[b] = (mode == 1 && nb == s.gbase[b]) ? min(S, s.K0 - np) : S + nb - s.gbase[b];
     s.gb_lo[b] = s.nb_gathered[b];
     s.gb_hi[b] = nb;
     s.nb_gathered[b] = nb;
@@ -252,226 +252,399 @@ __global__ void __launch_bounds__(128) sel_gather_kernel(SelState s) {
   }
 }
 
-// ------------------------------------------------------------------ greedy
-// One CTA of S threads per image; thread = active slot.
-//
-// The coordinates of the active tokens live in E during the round: shared memory laid out
-// [KP][S] when it fits (SMEM = true), else the tokens' global cache rows.
-// Phase 1 brings every active token's coordinates up to the current basis by forward
-// substitution, 32 basis vectors at a time: the 32 rows of L (the basis tokens' own
-// coordinate rows) are staged in shared memory and the 32 results accumulate in registers.
-// Phase 2 makes the picks with one block barrier per pick: the winning slot is carried in
-// the low bits of the key, and every slot's residual is published in shared memory, so
-// all threads derive the basis update from the same values.  Phase 3 writes back.
+// ------------------------------------------------------------------ coordinates
+// Per-slot coordinate rows: [S][P] in shared memory, P = KP rounded up to 8, plus 4, so that
+// eight lanes reading 16 bytes each from eight rows hit disjoint banks.
 constexpr int kChunk = 32;
+constexpr int kRegCoords = 128;
+constexpr int kUpdSlots = 32;
+
+__host__ __device__ inline int coord_pitch(int KP) { return ((KP + 7) / 8) * 8 + 4; }
+
+// ------------------------------------------------------------------ update
+// Brings every active token's coordinates up to the current basis (nb vectors) by forward
+// substitution before the picks:
+//   e_beta[i] = (G[j_beta, i] - sum_{beta' < beta} e_beta'[j_beta] e_beta'[i]) / r_beta,
+// 32 basis vectors at a time.  A CTA serves 32 slots (lane = slot) with kUpdWarps warps: the
+// 32 rows of L (the basis tokens' own coordinate rows) are staged in shared memory, each warp
+// forms the products with the known coordinates for its share of the 32 rows, and warp 0
+// then solves the 32 x 32 triangle.  An image's slots spread over S / 32 CTAs.  Writes Ec,
+// r2 and cstep = nb.
+constexpr int kUpdWarps = 4;
+constexpr int kUpdRows = kChunk / kUpdWarps;
+
+__global__ void __launch_bounds__(kUpdSlots * kUpdWarps, 1) sel_update_kernel(SelState s) {
+  extern __shared__ __align__(16) float shu[];
+  __shared__ float rinv_c[kChunk];
+  __shared__ float accs[kChunk][kUpdSlots];
+  const int b = blockIdx.y;
+  if (s.done[b]) return;
+  const int S = s.S, R = s.R, KP = s.KP, P = coord_pitch(KP);
+  const int nb = s.nbasis[b], gbase = s.gbase[b];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int slot = blockIdx.x * kUpdSlots + lane;
+  const long long base = static_cast<long long>(b) * s.N;
+  const int tok = slot < S ? s.aslot[static_cast<long long>(b) * S + slot] : -1;
+  const int c0 = tok >= 0 ? min(s.cstep[base + tok], nb) : nb;
+  if (!__syncthreads_or(c0 < nb)) return;
+  float* Lc = shu;                                   // [kChunk][KP]
+  float* me = shu + kChunk * KP + lane * P;          // this slot's row
+  if (tok >= 0 && warp == 0) {
+    const float* g = s.Ec + (base + tok) * KP;
+    for (int q = 0; q < c0; q += 4) cp_async16(me + q, g + q);
+  }
+  const int32_t* btok = s.basis_tok + static_cast<long long>(b) * s.K;
+  const float* rnorm = s.rnorm + static_cast<long long>(b) * s.K;
+  const float* Gr = s.G + (static_cast<long long>(b) * S + (tok >= 0 ? slot : 0)) * R;
+  float r2 = tok >= 0 ? s.r2[base + tok] : 0.f;
+  for (int b0 = 0; b0 < nb; b0 += kChunk) {
+    const int b1 = min(nb, b0 + kChunk);
+    if (!__syncthreads_or(tok >= 0 && b1 > c0)) continue;   // uniform; also fences the last chunk
+    {
+      // row i of L: basis token j_{b0+i}'s coordinates 0 .. b0+i-1 (all that is read of it)
+      const int bt = lane < b1 - b0 ? btok[b0 + lane] : 0;
+      for (int i = warp; i < b1 - b0; i += kUpdWarps) {
+        const int ti = __shfl_sync(0xffffffffu, bt, i);
+        const float* src = s.Ec + (base + ti) * KP;
+        for (int q = 4 * lane; q < b0 + i; q += 128) cp_async16(Lc + i * KP + q, src + q);
+      }
+      cp_async_wait_all();
+    }
+    if (threadIdx.x < b1 - b0) rinv_c[threadIdx.x] = 1.0f / rnorm[b0 + threadIdx.x];
+    __syncthreads();
+    const bool work = tok >= 0 && b1 > c0;
+    if (work) {
+      // this warp's rows: G entries minus the products with coordinates 0 .. b0-1
+      const int i0 = warp * kUpdRows;
+      float acc[kUpdRows];
+#pragma unroll
+      for (int r = 0; r < kUpdRows; ++r) {
+        const int beta = b0 + i0 + r;
+        acc[r] = (beta < b1 && beta >= c0) ? Gr[S + beta - gbase] : 0.f;
+      }
+#pragma unroll 2
+      for (int q = 0; q < b0; q += 4) {
+        const float4 eq = *reinterpret_cast<const float4*>(me + q);
+#pragma unroll
+        for (int r = 0; r < kUpdRows; ++r) {
+          const float4 l = *reinterpret_cast<const float4*>(Lc + (i0 + r) * KP + q);
+          acc[r] = fmaf(-l.x, eq.x, acc[r]);
+          acc[r] = fmaf(-l.y, eq.y, acc[r]);
+          acc[r] = fmaf(-l.z, eq.z, acc[r]);
+          acc[r] = fmaf(-l.w, eq.w, acc[r]);
+        }
+      }
+#pragma unroll
+      for (int r = 0; r < kUpdRows; ++r) accs[i0 + r][lane] = acc[r];
+    }
+    __syncthreads();
+    if (work && warp == 0) {
+      float e[kChunk];
+#pragma unroll
+      for (int i = 0; i < kChunk; ++i) {
+        const int beta = b0 + i;
+        if (beta < b1) {
+          if (beta >= c0) {
+            float a = accs[i][lane];
+#pragma unroll
+            for (int q = 0; q < i; ++q) a = fmaf(-Lc[i * KP + b0 + q], e[q], a);
+            e[i] = a * rinv_c[i];
+            me[beta] = e[i];
+            r2 = fmaf(-e[i], e[i], r2);
+          } else {
+            e[i] = me[beta];
+          }
+        }
+      }
+    }
+  }
+  if (warp == 0 && tok >= 0 && c0 < nb) {
+    float* g = s.Ec + (base + tok) * KP;
+    for (int q = c0; q < nb; ++q) g[q] = me[q];
+    s.r2[base + tok] = r2;
+    s.cstep[base + tok] = nb;
+  }
+}
+
+// ------------------------------------------------------------------ R0 basis
+// The K0 forced picks (R0 in p_hat order) need no argmax: their basis is the Cholesky factor
+// of the K0 x K0 Gram matrix G[R0, R0], column by column in pick order (right-looking, in
+// shared memory).  Column t adds basis vector nb unless its residual is degenerate
+// (r^2 <= tau ||v||^2); its entries below the diagonal are the later R0 tokens' coordinates
+// e_nb.  Writes picks, state, basis, Ec rows, cstep and r2 of the R0 tokens.
+constexpr int kCholThreads = kCholMax;
+
+// Left-looking, one thread per R0 position u, G[R0, R0] and the coordinate rows in shared
+// memory; one block barrier per basis vector.
+__global__ void __launch_bounds__(kCholThreads, 1) sel_chol_kernel(SelState s) {
+  extern __shared__ __align__(16) float shc[];
+  __shared__ float r2s[kCholMax], dg[kCholMax], dpick[kCholMax], ps[kCholMax];
+  __shared__ int tk[kCholMax], mine_s[kCholMax], bidx[kCholMax];
+  const int b = blockIdx.x;
+  const int K0 = s.K0, ldg = (K0 + 3) & ~3, PL = coord_pitch(K0);
+  float* Gs = shc;                                   // [K0][ldg]
+  float* Ls = shc + K0 * ldg;                        // [K0][PL] coordinates, zeros past the valid ones
+  const long long base = static_cast<long long>(b) * s.N;
+  const float* Gb = s.G + static_cast<long long>(b) * s.S * s.R;
+  {
+    const int v4 = ldg / 4;                          // G rows are 16-byte aligned (R % 16 == 0)
+    for (int i = threadIdx.x; i < K0 * v4; i += blockDim.x) {
+      const int r = i / v4, c = (i - r * v4) * 4;
+      cp_async16(Gs + r * ldg + c, Gb + static_cast<long long>(r) * s.R + c);
+    }
+  }
+  for (int i = threadIdx.x; i < K0 * PL / 4; i += blockDim.x)
+    reinterpret_cast<float4*>(Ls)[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+  cp_async_wait_all();
+  const int u = threadIdx.x;
+  if (u < K0) {
+    tk[u] = s.r0[static_cast<long long>(b) * s.K + u];
+    ps[u] = s.scores[base + tk[u]];
+  }
+  __syncthreads();
+  float r2 = 0.f;
+  if (u < K0) {
+    r2 = Gs[u * ldg + u];
+    r2s[u] = r2;
+    dg[u] = r2;
+  }
+  __syncthreads();
+  float* me = Ls + u * PL;
+  int nb = 0;
+  for (int t = 0; t < K0; ++t) {
+    const float d = r2s[t], sq = dg[t];
+    const bool ext = d > s.tau * sq && d > 0.f;
+    if (u == t) {                                         // global writes wait for the end
+      mine_s[t] = nb;
+      dpick[t] = d;
+      bidx[t] = ext ? nb : -1;
+    }
+    if (!ext) continue;                                   // uniform
+    if (u > t && u < K0) {
+      const float* lt = Ls + t * PL;
+      float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+#pragma unroll 4
+      for (int q = 0; q < nb; q += 4) {                   // rows are zero past nb
+        const float4 x = *reinterpret_cast<const float4*>(lt + q);
+        const float4 y = *reinterpret_cast<const float4*>(me + q);
+        a0 = fmaf(x.x, y.x, a0);
+        a1 = fmaf(x.y, y.y, a1);
+        a2 = fmaf(x.z, y.z, a2);
+        a3 = fmaf(x.w, y.w, a3);
+      }
+      const float e = (Gs[u * ldg + t] - ((a0 + a1) + (a2 + a3))) * (1.0f / sqrtf(d));
+      me[nb] = e;
+      r2 = fmaf(-e, e, r2);
+      r2s[u] = r2;
+    }
+    __syncthreads();
+    ++nb;
+  }
+  __syncthreads();
+  if (u < K0) {
+    const int tok = tk[u];
+    const float d = dpick[u];
+    s.picks[static_cast<long long>(b) * s.K + u] = tok;
+    s.state[base + tok] = 1;
+    s.cstep[base + tok] = mine_s[u];
+    s.r2[base + tok] = d;
+    s.U[base + tok] = sel_value(ps[u], d, dg[u], s.lambda, s.tau);
+    if (bidx[u] >= 0) {
+      s.basis_tok[static_cast<long long>(b) * s.K + bidx[u]] = tok;
+      s.rnorm[static_cast<long long>(b) * s.K + bidx[u]] = sqrtf(d);
+    }
+  }
+  // coordinate rows of the R0 tokens: e_beta for beta < (basis size at their pick)
+  for (int i = threadIdx.x; i < K0 * PL; i += blockDim.x) {
+    const int r = i / PL, q = i - r * PL;
+    if (q < mine_s[r]) s.Ec[(base + tk[r]) * s.KP + q] = Ls[r * PL + q];
+  }
+  if (threadIdx.x == 0) {
+    s.nbasis[b] = nb;
+    s.npicks[b] = K0;
+  }
+}
+
+// ------------------------------------------------------------------ greedy
+// One CTA of S threads per image; thread = active slot.  Every active token's coordinates
+// are current (sel_update_kernel ran first); they are held in the slot rows ([S][P] shared
+// memory when it fits, else the tokens' global cache rows) and, for the first kRegCoords,
+// in registers.  The picks take one block barrier each: the winning slot is carried in the
+// low bits of the key, and every slot's residual is published in shared memory, so all
+// threads derive the basis update from the same values; the winner's row is read as 16-byte
+// broadcasts and its Gram entry is loaded while the dot product runs.
 
 template <bool SMEM>
 struct Coords {
-  float* Es;            // SMEM: [KP][S]
+  float* Es;            // SMEM: [S][P]
   float* Ec;            // global cache rows
   long long base;
-  int S, KP;
-  __device__ __forceinline__ float* at(int slot, int tok, int q) const {
-    if constexpr (SMEM) return Es + static_cast<long long>(q) * S + slot;
-    else return Ec + (base + tok) * KP + q;
+  int P, KP;
+  __device__ __forceinline__ float* row(int slot, int tok) const {
+    if constexpr (SMEM) return Es + static_cast<long long>(slot) * P;
+    else return Ec + (base + tok) * KP;
   }
 };
 
 // key of a candidate inside the round: (value bits, 0xFFFF - token, slot); the upper 48
 // bits order like make_key (value descending, lower token first).
-__device__ __forceinline__ uint64_t slot_key(float v, int tok, int slot) {
-  const float c = v > 0.f ? v : 0.f;
-  return (static_cast<uint64_t>(__float_as_uint(c)) << 32) | (static_cast<uint64_t>(0xFFFFu - tok) << 16) |
-         static_cast<uint64_t>(slot);
-}
-__device__ __forceinline__ uint64_t theta48(uint64_t theta) {   // make_key -> upper 48 bits of slot_key
+__device__ __forceinline__ uint64_t theta48(uint64_t theta) {   // make_key -> upper 48 bits of the round key
   if (theta == 0) return 0;
   const uint32_t tok = static_cast<uint32_t>(key_index(theta));
   return ((theta >> 32) << 16) | (0xFFFFu - tok);
+}
+
+// Largest (hi, lo) pair over the warp, hi first: two warp reductions on 32-bit words.
+__device__ __forceinline__ uint64_t warp_max_key(uint32_t hi, uint32_t lo) {
+  const uint32_t h = __reduce_max_sync(0xffffffffu, hi);
+  const uint32_t l = __reduce_max_sync(0xffffffffu, hi == h ? lo : 0u);
+  return (static_cast<uint64_t>(h) << 32) | l;
 }
 
 template <bool SMEM>
 __global__ void __launch_bounds__(256, 1) sel_greedy_kernel(SelState s) {
   extern __shared__ __align__(16) float shf[];
   __shared__ uint64_t wkey[2][32];
-  __shared__ float sh_rinv_chunk[kChunk];
   const int b = blockIdx.x;
   if (s.done[b]) return;
   const int S = s.S, R = s.R, KP = s.KP;
-  float* Lc = shf;                                   // [kChunk][KP]
-  float* r2s = shf + kChunk * KP;                    // [S] published residuals
+  float* r2s = shf;                                  // [S] published residuals
   float* sqs = r2s + S;                              // [S]
   int32_t* tks = reinterpret_cast<int32_t*>(sqs + S);   // [S] tokens of the slots
-  Coords<SMEM> E{reinterpret_cast<float*>(tks + S), s.Ec, static_cast<long long>(b) * s.N, S, KP};
+  int32_t* ends = tks + S;                           // [S] valid coordinates of the slots at the end
+  int32_t* pk_tok = ends + S;                        // [KP] this launch's picks
+  float* pk_r2 = reinterpret_cast<float*>(pk_tok + KP);  // [KP] their residuals (-1: no basis vector)
+  const Coords<SMEM> E{pk_r2 + KP, s.Ec, static_cast<long long>(b) * s.N, coord_pitch(KP), KP};
   const long long base = E.base;
   const int slot = threadIdx.x;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
   const int tok = s.aslot[static_cast<long long>(b) * S + slot];
-  const int32_t* btok = s.basis_tok + static_cast<long long>(b) * s.K;
-  const float* rnorm = s.rnorm + static_cast<long long>(b) * s.K;
   const float* Gb = s.G + static_cast<long long>(b) * S * R;
-  const float* Gr = Gb + static_cast<long long>(slot) * R;
   int nb = s.nbasis[b], np = s.npicks[b];
-  const int gbase = s.gbase[b];
   const bool forced = s.mode[b] == 1;
   const uint64_t th48 = theta48(s.theta[b]);
+  float* me = tok >= 0 ? E.row(slot, tok) : nullptr;
 
   float r2 = 0.f, sq = 0.f, p = 0.f, val = 0.f;
-  int c0 = nb, mine = nb;                            // cached coordinates; valid coordinates at the end
+  const int c0 = nb;                                 // coordinates cached at the start (all current)
+  int mine = nb;                                     // valid coordinates at the end
   bool alive = false;
   if (tok >= 0) {
     p = s.scores[base + tok];
     alive = s.state[base + tok] == 0;
-    c0 = min(s.cstep[base + tok], nb);
-    if (s.diag_sq && c0 == 0) {
-      sq = r2 = Gr[slot];                            // <v, v> from the Gram block
-    } else {
-      r2 = s.r2[base + tok];
-      sq = s.sqn[base + tok];
+    if (s.cstep[base + tok] < nb) {                  // sel_update_kernel did not run
+      atomicOr(s.status, ST_INTERNAL);
+      alive = false;
     }
-    if constexpr (SMEM) {
-      const float4* g = reinterpret_cast<const float4*>(s.Ec + (base + tok) * KP);
-      int q = 0;
-      for (; q + 16 <= c0; q += 16) {
-        float4 v[4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) v[u] = g[q / 4 + u];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          *E.at(slot, tok, q + 4 * u) = v[u].x; *E.at(slot, tok, q + 4 * u + 1) = v[u].y;
-          *E.at(slot, tok, q + 4 * u + 2) = v[u].z; *E.at(slot, tok, q + 4 * u + 3) = v[u].w;
-        }
+    r2 = s.r2[base + tok];
+    sq = s.sqn[base + tok];
+  }
+  if constexpr (SMEM) {
+    // the slot's row: cached coordinates, zeros after them
+    float4* row4 = reinterpret_cast<float4*>(E.row(slot, tok));
+    const float4* g = tok >= 0 ? reinterpret_cast<const float4*>(s.Ec + (base + tok) * KP) : nullptr;
+    for (int q = 0; q < E.P; q += 4) {
+      float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (tok >= 0 && q < c0) {
+        v = g[q / 4];
+        if (q + 1 >= c0) v.y = 0.f;
+        if (q + 2 >= c0) v.z = 0.f;
+        if (q + 3 >= c0) v.w = 0.f;
       }
-      for (; q < c0; ++q) *E.at(slot, tok, q) = s.Ec[(base + tok) * KP + q];
+      row4[q / 4] = v;
     }
+    if (slot < 8) reinterpret_cast<float4*>(E.row(S, 0))[slot] = make_float4(0.f, 0.f, 0.f, 0.f);
   }
   tks[slot] = tok;
-
-  // ---- phase 1: forward substitution, chunk by chunk
-  for (int b0 = 0; b0 < nb; b0 += kChunk) {
-    const int b1 = min(nb, b0 + kChunk);
-    __syncthreads();
-    {
-      const int KV = KP / 4, nvec = (b1 - b0) * KV;
-      for (int t0 = threadIdx.x; t0 < nvec; t0 += 4 * blockDim.x) {
-        float4 v[4];
-        int qs[4], is[4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const int t = t0 + u * blockDim.x;
-          is[u] = t / KV;
-          qs[u] = (t - is[u] * KV) * 4;
-          v[u] = t < nvec ? *reinterpret_cast<const float4*>(s.Ec + (base + btok[b0 + is[u]]) * KP + qs[u])
-                          : make_float4(0.f, 0.f, 0.f, 0.f);
-        }
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const int t = t0 + u * blockDim.x;
-          if (t < nvec) {
-            const int lim = b0 + is[u];
-            v[u].x = qs[u] < lim ? v[u].x : 0.f;
-            v[u].y = qs[u] + 1 < lim ? v[u].y : 0.f;
-            v[u].z = qs[u] + 2 < lim ? v[u].z : 0.f;
-            v[u].w = qs[u] + 3 < lim ? v[u].w : 0.f;
-            *reinterpret_cast<float4*>(Lc + is[u] * KP + qs[u]) = v[u];
-          }
-        }
-      }
-    }
-    if (threadIdx.x < b1 - b0) sh_rinv_chunk[threadIdx.x] = 1.0f / rnorm[b0 + threadIdx.x];
-    __syncthreads();
-    if (tok < 0 || b1 <= c0) continue;
-    float acc[kChunk], e[kChunk];
-#pragma unroll
-    for (int i = 0; i < kChunk; ++i) acc[i] = (b0 + i < b1 && b0 + i >= c0) ? Gr[S + b0 + i - gbase] : 0.f;
-    for (int q = 0; q < b0; q += 4) {
-      float4 eq;
-      if constexpr (SMEM) {
-        eq = make_float4(*E.at(slot, tok, q), *E.at(slot, tok, q + 1), *E.at(slot, tok, q + 2), *E.at(slot, tok, q + 3));
-      } else {
-        eq = *reinterpret_cast<const float4*>(E.at(slot, tok, q));
-      }
-#pragma unroll
-      for (int i = 0; i < kChunk; ++i) {
-        const float4 l = *reinterpret_cast<const float4*>(Lc + i * KP + q);
-        acc[i] = fmaf(-l.x, eq.x, acc[i]);
-        acc[i] = fmaf(-l.y, eq.y, acc[i]);
-        acc[i] = fmaf(-l.z, eq.z, acc[i]);
-        acc[i] = fmaf(-l.w, eq.w, acc[i]);
-      }
-    }
-#pragma unroll
-    for (int i = 0; i < kChunk; ++i) {
-      const int beta = b0 + i;
-      if (beta < b1) {
-        if (beta >= c0) {
-          float a = acc[i];
-#pragma unroll
-          for (int q = 0; q < i; ++q) a = fmaf(-Lc[i * KP + b0 + q], e[q], a);
-          e[i] = a * sh_rinv_chunk[i];
-          *E.at(slot, tok, beta) = e[i];
-          r2 = fmaf(-e[i], e[i], r2);
-        } else {
-          e[i] = *E.at(slot, tok, beta);
-        }
-      }
-    }
-  }
   if (tok >= 0) val = sel_value(p, r2, sq, s.lambda, s.tau);
   r2s[slot] = r2;
   sqs[slot] = sq;
+  __syncthreads();
 
-  // ---- phase 2: picks, one block barrier each
-  for (int step = 0, buf = 0; np < s.K; ++step, buf ^= 1) {
-    uint64_t key = alive ? slot_key(val, tok, slot) : 0ull;
+  // the first nreg coordinates of this slot, in registers for the picks
+  float ereg[kRegCoords];
+  const int nreg = min(nb, kRegCoords) & ~3;
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const uint64_t other = __shfl_xor_sync(0xffffffffu, key, o);
-      key = other > key ? other : key;
+  for (int g = 0; g < kRegCoords / 4; ++g) {
+    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (alive && 4 * g < nreg) v = *reinterpret_cast<const float4*>(me + 4 * g);
+    ereg[4 * g] = v.x; ereg[4 * g + 1] = v.y; ereg[4 * g + 2] = v.z; ereg[4 * g + 3] = v.w;
+  }
+
+  for (int step = 0, buf = 0; np < s.K; ++step, buf ^= 1) {
+    {
+      const uint32_t vb = alive ? __float_as_uint(val > 0.f ? val : 0.f) : 0u;
+      const uint32_t lo = alive ? ((0xFFFFu - static_cast<uint32_t>(tok)) << 16) | static_cast<uint32_t>(slot) : 0u;
+      const uint64_t key = warp_max_key(vb, lo);
+      if (lane == 0) wkey[buf][warp] = key;
     }
-    if (lane == 0) wkey[buf][warp] = key;
     __syncthreads();
     int jslot;
     if (forced) {
       jslot = step;
       if (jslot >= S || tks[jslot] < 0) break;
     } else {
-      uint64_t best = lane < nwarps ? wkey[buf][lane] : 0ull;
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        const uint64_t other = __shfl_xor_sync(0xffffffffu, best, o);
-        best = other > best ? other : best;
-      }
+      const uint64_t k = lane < nwarps ? wkey[buf][lane] : 0ull;
+      const uint64_t best = warp_max_key(static_cast<uint32_t>(k >> 32), static_cast<uint32_t>(k));
       if (best == 0 || (best >> 16) <= th48) break;   // uniform
       jslot = static_cast<int>(best & 0xFFFFu);
     }
     const int jt = tks[jslot];
     const float r2j = r2s[jslot], sqj = sqs[jslot];
     const bool ext = (r2j > s.tau * sqj) && (r2j > 0.f);
-    if (slot == jslot) {
+    if (slot == jslot) {                             // global writes wait for the end
       alive = false;
       mine = nb;
-      s.state[base + jt] = 1;
-      s.picks[static_cast<long long>(b) * s.K + np] = jt;
-      if (ext) {
-        s.basis_tok[static_cast<long long>(b) * s.K + nb] = jt;
-        s.rnorm[static_cast<long long>(b) * s.K + nb] = sqrtf(r2j);
-      }
+      pk_tok[step] = jt;
+      pk_r2[step] = ext ? r2j : -1.f;
     }
     if (ext) {
       if (alive) {
+        const float gji = Gb[static_cast<long long>(jslot) * R + slot];   // in flight during the dot product
         const float rinv = 1.0f / sqrtf(r2j);
-        float a0 = Gb[static_cast<long long>(jslot) * R + slot], a1 = 0.f, a2 = 0.f, a3 = 0.f;
-        int q = 0;
-        for (; q + 4 <= nb; q += 4) {
-          a0 = fmaf(-*E.at(jslot, jt, q), *E.at(slot, tok, q), a0);
-          a1 = fmaf(-*E.at(jslot, jt, q + 1), *E.at(slot, tok, q + 1), a1);
-          a2 = fmaf(-*E.at(jslot, jt, q + 2), *E.at(slot, tok, q + 2), a2);
-          a3 = fmaf(-*E.at(jslot, jt, q + 3), *E.at(slot, tok, q + 3), a3);
+        const float* cj = E.row(jslot, jt);
+        float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+        if constexpr (SMEM) {
+          // 32 coordinates per branch, so the loads of a block issue together; shared rows
+          // are zero past their valid coordinates and ereg is zero past nreg
+#pragma unroll
+          for (int blk = 0; blk < kRegCoords / 32; ++blk) {
+            if (32 * blk < nreg) {
+#pragma unroll
+              for (int g = 8 * blk; g < 8 * blk + 8; ++g) {
+                const float4 c = *reinterpret_cast<const float4*>(cj + 4 * g);
+                a0 = fmaf(c.x, ereg[4 * g], a0);
+                a1 = fmaf(c.y, ereg[4 * g + 1], a1);
+                a2 = fmaf(c.z, ereg[4 * g + 2], a2);
+                a3 = fmaf(c.w, ereg[4 * g + 3], a3);
+              }
+            }
+          }
+        } else {
+#pragma unroll
+          for (int g = 0; g < kRegCoords / 4; ++g) {
+            if (4 * g < nreg) {
+              const float4 c = *reinterpret_cast<const float4*>(cj + 4 * g);
+              a0 = fmaf(c.x, ereg[4 * g], a0);
+              a1 = fmaf(c.y, ereg[4 * g + 1], a1);
+              a2 = fmaf(c.z, ereg[4 * g + 2], a2);
+              a3 = fmaf(c.w, ereg[4 * g + 3], a3);
+            }
+          }
         }
-        for (; q < nb; ++q) a0 = fmaf(-*E.at(jslot, jt, q), *E.at(slot, tok, q), a0);
-        const float e = ((a0 + a1) + (a2 + a3)) * rinv;
-        *E.at(slot, tok, nb) = e;
+        int q = nreg;
+#pragma unroll 4
+        for (; q + 4 <= nb; q += 4) {
+          const float4 c = *reinterpret_cast<const float4*>(cj + q);
+          const float4 m = *reinterpret_cast<const float4*>(me + q);
+          a0 = fmaf(c.x, m.x, a0);
+          a1 = fmaf(c.y, m.y, a1);
+          a2 = fmaf(c.z, m.z, a2);
+          a3 = fmaf(c.w, m.w, a3);
+        }
+        for (; q < nb; ++q) a0 = fmaf(cj[q], me[q], a0);
+        const float e = (gji - ((a0 + a1) + (a2 + a3))) * rinv;
+        me[nb] = e;
         r2 = fmaf(-e, e, r2);
         val = sel_value(p, r2, sq, s.lambda, s.tau);
         r2s[slot] = r2;
@@ -480,16 +653,40 @@ __global__ void __launch_bounds__(256, 1) sel_greedy_kernel(SelState s) {
     }
     ++np;
   }
-  // ---- phase 3: write back
+  // write back: this launch's picks, then the active tokens
+  const int np0 = s.npicks[b], nb0 = s.nbasis[b];
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int nbw = nb0;
+    for (int i = 0; i < np - np0; ++i) {
+      if (pk_r2[i] >= 0.f) {
+        s.basis_tok[static_cast<long long>(b) * s.K + nbw] = pk_tok[i];
+        s.rnorm[static_cast<long long>(b) * s.K + nbw] = sqrtf(pk_r2[i]);
+        ++nbw;
+      }
+    }
+  }
+  for (int i = threadIdx.x; i < np - np0; i += blockDim.x) {
+    s.picks[static_cast<long long>(b) * s.K + np0 + i] = pk_tok[i];
+    s.state[base + pk_tok[i]] = 1;
+  }
   if (tok >= 0) {
     if (alive) mine = nb;
-    if constexpr (SMEM) {
-      float* g = s.Ec + (base + tok) * KP;
-      for (int q = c0; q < mine; ++q) g[q] = *E.at(slot, tok, q);
-    }
     s.cstep[base + tok] = mine;
     s.r2[base + tok] = r2;
     s.U[base + tok] = val;
+  }
+  if constexpr (SMEM) {
+    // coordinates [c0, mine) of every slot's row, one warp per row
+    ends[slot] = tok >= 0 ? mine : c0;
+    __syncthreads();
+    for (int r = warp; r < S; r += nwarps) {
+      const int t = tks[r], end = ends[r];
+      if (t < 0) continue;
+      float* g = s.Ec + (base + t) * KP;
+      const float* src = E.row(r, t);
+      for (int q = c0 + lane; q < end; q += 32) g[q] = src[q];
+    }
   }
   if (threadIdx.x == 0) {
     s.nbasis[b] = nb;
@@ -553,10 +750,16 @@ __global__ void sel_identity_kernel(int N, int32_t* keep, int32_t* order) {
 size_t sel_init_smem(int N, int K0) { return (static_cast<size_t>(N) + pow2_at_least(std::max(K0, 1))) * 8; }
 size_t sel_choose_smem(int N) { return static_cast<size_t>(N) * 8; }
 size_t sel_greedy_smem(int KP, int S, bool* smem_coords) {
-  const size_t lc = static_cast<size_t>(kChunk) * KP * 4 + static_cast<size_t>(S) * 12;
-  const size_t es = static_cast<size_t>(KP) * S * 4;
-  *smem_coords = lc + es <= 200 * 1024;
-  return *smem_coords ? lc + es : lc;
+  const size_t small = static_cast<size_t>(S) * 16 + static_cast<size_t>(KP) * 8;
+  const size_t es = (static_cast<size_t>(coord_pitch(KP)) * S + 32) * 4;   // + zeros read past the last row
+  *smem_coords = small + es <= 200 * 1024;
+  return *smem_coords ? small + es : small;
+}
+size_t sel_chol_smem(int K0) {
+  return (static_cast<size_t>(K0) * ((K0 + 3) & ~3) + static_cast<size_t>(K0) * coord_pitch(K0)) * 4;
+}
+size_t sel_update_smem(int KP) {
+  return (static_cast<size_t>(kChunk) * KP + static_cast<size_t>(kUpdSlots) * coord_pitch(KP)) * 4;
 }
 
 cudaError_t launch_sel_init(const SelState& s, cudaStream_t st) {
@@ -578,9 +781,13 @@ cudaError_t launch_sel_choose(const SelState& s, cudaStream_t st) {
 }
 
 cudaError_t launch_sel_greedy(const SelState& s, cudaStream_t st) {
+  const size_t um = sel_update_smem(s.KP);
+  cudaError_t e = cudaFuncSetAttribute(sel_update_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(um));
+  if (e != cudaSuccess) return e;
+  sel_update_kernel<<<dim3((s.S + kUpdSlots - 1) / kUpdSlots, s.B), kUpdSlots * kUpdWarps, um, st>>>(s);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
   bool in_smem = false;
   const size_t sm = sel_greedy_smem(s.KP, s.S, &in_smem);
-  cudaError_t e;
   if (in_smem) {
     e = cudaFuncSetAttribute(sel_greedy_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(sm));
     if (e != cudaSuccess) return e;
@@ -590,6 +797,15 @@ cudaError_t launch_sel_greedy(const SelState& s, cudaStream_t st) {
     if (e != cudaSuccess) return e;
     sel_greedy_kernel<false><<<s.B, s.S, sm, st>>>(s);
   }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_sel_chol(const SelState& s, cudaStream_t st) {
+  if (s.K0 < 1 || s.K0 > kCholMax || s.K0 > s.S) return cudaErrorInvalidValue;
+  const size_t sm = sel_chol_smem(s.K0);
+  cudaError_t e = cudaFuncSetAttribute(sel_chol_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(sm));
+  if (e != cudaSuccess) return e;
+  sel_chol_kernel<<<s.B, kCholThreads, sm, st>>>(s);
   return cudaGetLastError();
 }
 

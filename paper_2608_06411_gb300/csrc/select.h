@@ -6,6 +6,8 @@
 
 namespace mapk {
 
+constexpr int kCholMax = 128;     // largest R0 factored by sel_chol_kernel
+
 struct SelState {
   int B, N, D, K, K0, S;          // S = active-set size (Gram block rows)
   int R;                          // rows per image in Vg = row stride of G (>= S + K, multiple of 16)
@@ -34,8 +36,6 @@ struct SelState {
   void* Vg;                       // [B, R, D] bf16 gathered rows
   float* G;                       // [B, S, R] Gram block
   int32_t* done_count;            // images finished
-  int diag_sq;                    // 1: a token evaluated for the first time takes ||v||^2 from
-                                  // the Gram block's diagonal (before the R0 projection)
   int* status;
 };
 
@@ -44,7 +44,10 @@ size_t sel_choose_smem(int N);
 size_t sel_greedy_smem(int KP, int S, bool* smem_coords);
 cudaError_t launch_sel_init(const SelState& s, cudaStream_t st);
 cudaError_t launch_sel_choose(const SelState& s, cudaStream_t st);
+// sel_update_kernel (coordinates of the active tokens up to the current basis), then the picks.
 cudaError_t launch_sel_greedy(const SelState& s, cudaStream_t st);
+// The K0 forced R0 picks from the Gram block G[R0, R0] of a forced round (K0 <= kCholMax, <= S).
+cudaError_t launch_sel_chol(const SelState& s, cudaStream_t st);
 cudaError_t launch_sel_finalize(const int32_t* picks, int B, int K, int32_t* keep, int32_t* order, cudaStream_t st);
 cudaError_t launch_sel_copy_r0(const int32_t* r0, int B, int K, int32_t* picks, cudaStream_t st);
 cudaError_t launch_sel_identity(int B, int N, int32_t* keep, int32_t* order, cudaStream_t st);
