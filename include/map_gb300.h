@@ -187,9 +187,9 @@ int map_get_counters(map_ctx *ctx, map_counters *out);
 
 /* Kernel ids for timing. */
 #define MAP_K_GEMM_FV1    0   /* f_V layer 1: V [B*N, D] x wV1^T, GELU */
-#define MAP_K_GEMM_FV2    1
-#define MAP_K_GEMM_WK     2
-#define MAP_K_GEMM_TEXT   3   /* the three f_T / W_Q launches together */
+#define MAP_K_GEMM_FV2    1   /* no launches: f_V layer 2 is folded into W_K (W_K wV2) */
+#define MAP_K_GEMM_WK     2   /* folded W_K wV2 projection with RoPE */
+#define MAP_K_GEMM_TEXT   3   /* f_T layer 1 and the folded W_Q wT2 projection together */
 #define MAP_K_SCORES      4   /* softmax statistics + mean */
 #define MAP_K_SELECT      5   /* everything in map_select */
 #define MAP_K_GATHER      6

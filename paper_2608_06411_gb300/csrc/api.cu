@@ -35,8 +35,11 @@ struct map_ctx {
   map_config cfg{};
   int device = 0, num_sms = 148;
   void* w[10] = {};                 // wT1 bT1 wT2 bT2 wQ wV1 bV1 wV2 bV2 wK (device bf16)
+  // W_Q f_T layer 2 and W_K f_V layer 2 folded (no nonlinearity between them): bf16 rows
+  // [hi | hi | lo] of W_Q W_T2 / W_K W_V2 ([dp, 3 Dh]) and fp32 biases W_Q b_T2 / W_K b_V2
+  void* wqt = nullptr; void* wkv = nullptr; float* bqt = nullptr; float* bkv = nullptr;
   DevBuf rope;  int rope_rows = 0;
-  DevBuf h1, h2, kb, th1, th2, qb, stats, qoff, post, sqn, pmean;
+  DevBuf h1, kb, th1, qb, stats, qoff, post, sqn, pmean;
   // selection
   DevBuf sU, sr2, scstep, sstate, sEc, spicks, sr0, sbt, srn, ssmall, stheta, saslot, sVg, sG;
   // map_prune staging
@@ -195,17 +198,16 @@ GemmDesc linear_desc(map_ctx* c, const void* x, long long rows, int K, const voi
   return d;
 }
 
-// Predictor for one modality: x [rows, D] -> RoPE(W f(x)) * scale [rows, dp], stored as
-// three bf16 segments [rows, 3 dp] (split_kind 0: hi|lo|hi, 1: hi|hi|lo) and, if aux is
-// given, as fp32 too.  The hidden activations h1, h2 are kept as bf16 hi/lo pairs
-// [rows, 2 Dh] (about 16 significant bits), and the layers after them run with K = 2 Dh
-// against [W | W].
-int predictor_branch(map_ctx* c, const void* x, long long rows, const void* w1, const void* b1, const void* w2,
-                     const void* b2, const void* wp, DevBuf& h1, DevBuf& h2, void* out3, int split_kind, float scale,
-                     float* aux, const int* pos, int pos_mod, cudaStream_t st, int tid_l1, int tid_l2, int tid_p) {
+// Predictor for one modality (Eq. 3): x [rows, D] -> RoPE(Wp f(x)) * scale [rows, dp] with
+// f = Linear -> GELU -> Linear, stored as three bf16 segments [rows, 3 dp] (split_kind 0:
+// hi|lo|hi, 1: hi|hi|lo) and, if aux is given, as fp32 too.  The hidden activation
+// h1 = GELU(W1 x + b1) is kept as a bf16 hi/lo pair [rows, 2 Dh] (about 16 significant bits);
+// the second layer and the projection are one folded matrix Wf = Wp W2 with bias Wp b2.
+int predictor_branch(map_ctx* c, const void* x, long long rows, const void* w1, const void* b1, const void* wf,
+                     const float* bf, DevBuf& h1, void* out3, int split_kind, float scale, float* aux,
+                     const int* pos, int pos_mod, cudaStream_t st, int tid_l1, int tid_p) {
   const map_config& g = c->cfg;
   MAP_TRY(ensure(h1, static_cast<size_t>(rows) * g.Dh * 4));
-  MAP_TRY(ensure(h2, static_cast<size_t>(rows) * g.Dh * 4));
   {
     Timed t(c, st, tid_l1);
     GemmDesc d = linear_desc(c, x, rows, g.D, w1, g.Dh, b1, h1.p, mapk::EPI_GELU_SPLIT);
@@ -213,14 +215,12 @@ int predictor_branch(map_ctx* c, const void* x, long long rows, const void* w1, 
     MAP_TRY(gemm(c, d, st));
   }
   {
-    Timed t(c, st, tid_l2);
-    GemmDesc d = linear_desc(c, h1.p, rows, 2 * g.Dh, w2, g.Dh, b2, h2.p, mapk::EPI_BIAS_SPLIT);
-    d.ldc = 2LL * g.Dh;
-    MAP_TRY(gemm(c, d, st));
-  }
-  {
+    // K = 3 Dh: A segments [hi | lo | hi] (the K coordinate wraps at 2 Dh) against
+    // [Wf_hi | Wf_hi | Wf_lo]: h_hi Wf_hi + h_lo Wf_hi + h_hi Wf_lo
     Timed t(c, st, tid_p);
-    GemmDesc d = linear_desc(c, h2.p, rows, 2 * g.Dh, wp, g.dp, nullptr, out3, mapk::EPI_ROPE_SPLIT3);
+    GemmDesc d = linear_desc(c, h1.p, rows, 3 * g.Dh, wf, g.dp, nullptr, out3, mapk::EPI_ROPE_SPLIT3);
+    d.a_kwrap = 2 * g.Dh;
+    d.biasf = bf;
     d.ldc = 3LL * g.dp;
     d.rope = static_cast<const float2*>(c->rope.p);
     d.pos = g.rope_on ? pos : nullptr;      // without RoPE every position is 0: cos 1, sin 0
@@ -276,11 +276,11 @@ int score_impl(map_ctx* c, const void* text, const void* vis, const int32_t* len
   const int dp3 = 3 * g.dp;
   MAP_TRY(ensure(c->kb, static_cast<size_t>(vrows) * dp3 * 2));
   MAP_TRY(ensure(c->qb, static_cast<size_t>(total_m) * dp3 * 2));
-  MAP_TRY(predictor_branch(c, vis, vrows, c->w[5], c->w[6], c->w[7], c->w[8], c->w[9], c->h1, c->h2, c->kb.p, 0,
-                           1.0f, k_out, nullptr, N, st, MAP_K_GEMM_FV1, MAP_K_GEMM_FV2, MAP_K_GEMM_WK));
-  MAP_TRY(predictor_branch(c, text, total_m, c->w[0], c->w[1], c->w[2], c->w[3], c->w[4], c->th1, c->th2, c->qb.p, 1,
+  MAP_TRY(predictor_branch(c, vis, vrows, c->w[5], c->w[6], c->wkv, c->bkv, c->h1, c->kb.p, 0, 1.0f, k_out, nullptr,
+                           N, st, MAP_K_GEMM_FV1, MAP_K_GEMM_WK));
+  MAP_TRY(predictor_branch(c, text, total_m, c->w[0], c->w[1], c->wqt, c->bqt, c->th1, c->qb.p, 1,
                            1.0f / std::sqrt(static_cast<float>(g.dp)), q_out, static_cast<const int*>(c->post.p), 1,
-                           st, MAP_K_GEMM_TEXT, MAP_K_GEMM_TEXT, MAP_K_GEMM_TEXT));
+                           st, MAP_K_GEMM_TEXT, MAP_K_GEMM_TEXT));
   // Eq. 3 on the tensor cores: logits tile [visual tokens x question tokens] of one image,
   // pass 1 -> per-slab column (max, sum exp), combine -> (max, 1/sum), pass 2 -> mean.
   const int m_tiles = (N + 127) / 128, nparts = 4 * m_tiles;
@@ -537,21 +537,29 @@ int map_init(const map_config* cfg, const map_weights* w, map_ctx** out) {
   do {
     if (cudaGetDevice(&c->device) != cudaSuccess) { rc = MAP_ECUDA; break; }
     if (cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, c->device) != cudaSuccess) { rc = MAP_ECUDA; break; }
-    // Layers fed by a hi/lo activation pair (f_T, f_V layer 2, W_Q, W_K) are stored as
-    // [W | W] ([out, 2 * in]); the others as given.
     const size_t D = cfg->D, Dh = cfg->Dh, dp = cfg->dp;
     const size_t rows[10] = {Dh, 1, Dh, 1, dp, Dh, 1, Dh, 1, dp};
     const size_t cols[10] = {D, Dh, Dh, Dh, Dh, D, Dh, Dh, Dh, Dh};
-    const bool dup[10] = {false, false, true, false, true, false, false, true, false, true};
     for (int i = 0; i < 10 && rc == MAP_OK; ++i) {
-      const size_t pitch = cols[i] * 2 * (dup[i] ? 2 : 1);
-      if (cudaMalloc(&c->w[i], rows[i] * pitch) != cudaSuccess) { rc = MAP_ENOMEM; break; }
-      for (int h = 0; h < (dup[i] ? 2 : 1) && rc == MAP_OK; ++h)
-        if (cudaMemcpy2D(static_cast<char*>(c->w[i]) + h * cols[i] * 2, pitch, src[i], cols[i] * 2, cols[i] * 2,
-                         rows[i], cudaMemcpyDefault) != cudaSuccess)
-          rc = MAP_ECUDA;
+      if (cudaMalloc(&c->w[i], rows[i] * cols[i] * 2) != cudaSuccess) { rc = MAP_ENOMEM; break; }
+      if (cudaMemcpy(c->w[i], src[i], rows[i] * cols[i] * 2, cudaMemcpyDefault) != cudaSuccess) rc = MAP_ECUDA;
     }
     if (rc != MAP_OK) break;
+    // The projections follow the second MLP layers with nothing in between: fold them.
+    if (cudaMalloc(&c->wqt, dp * 3 * Dh * 2) != cudaSuccess || cudaMalloc(&c->wkv, dp * 3 * Dh * 2) != cudaSuccess ||
+        cudaMalloc(reinterpret_cast<void**>(&c->bqt), dp * 4) != cudaSuccess ||
+        cudaMalloc(reinterpret_cast<void**>(&c->bkv), dp * 4) != cudaSuccess) {
+      rc = MAP_ENOMEM;
+      break;
+    }
+    if (mapk::launch_fold_weights(c->w[4], c->w[2], c->w[3], static_cast<int>(dp), static_cast<int>(Dh), c->wqt,
+                                  c->bqt, nullptr) != cudaSuccess ||
+        mapk::launch_fold_weights(c->w[9], c->w[7], c->w[8], static_cast<int>(dp), static_cast<int>(Dh), c->wkv,
+                                  c->bkv, nullptr) != cudaSuccess ||
+        cudaDeviceSynchronize() != cudaSuccess) {
+      rc = MAP_ECUDA;
+      break;
+    }
     if (cudaMalloc(&c->status, sizeof(int)) != cudaSuccess) { rc = MAP_ENOMEM; break; }
     if (cudaMemset(c->status, 0, sizeof(int)) != cudaSuccess) { rc = MAP_ECUDA; break; }
     if (cudaMallocHost(&c->h_status, sizeof(int)) != cudaSuccess) { rc = MAP_ENOMEM; break; }
@@ -647,7 +655,9 @@ void map_destroy(map_ctx* ctx) {
   cudaDeviceSynchronize();
   for (void*& p : ctx->w)
     if (p) cudaFree(p);
-  DevBuf* bufs[] = {&ctx->rope, &ctx->h1, &ctx->h2, &ctx->kb, &ctx->th1, &ctx->th2, &ctx->qb, &ctx->stats,
+  for (void* p : {ctx->wqt, ctx->wkv, static_cast<void*>(ctx->bqt), static_cast<void*>(ctx->bkv)})
+    if (p) cudaFree(p);
+  DevBuf* bufs[] = {&ctx->rope, &ctx->h1, &ctx->kb, &ctx->th1, &ctx->qb, &ctx->stats,
                     &ctx->qoff, &ctx->post, &ctx->sqn, &ctx->pmean, &ctx->sU, &ctx->sr2, &ctx->scstep, &ctx->sstate,
                     &ctx->sEc, &ctx->spicks, &ctx->sr0, &ctx->sbt, &ctx->srn, &ctx->ssmall, &ctx->stheta,
                     &ctx->saslot, &ctx->sVg, &ctx->sG, &ctx->pvis, &ctx->ptext, &ctx->pout, &ctx->pkeep,

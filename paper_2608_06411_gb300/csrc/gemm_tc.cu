@@ -5,12 +5,15 @@
 // epilogue (section "Cross-Modal Attention Distillation"), and the Gram blocks
 // <v_i, v_j> that the diversity term of Eq. 4 needs.
 //
-// Structure (one CTA per SM, 6 warps; 8 for EPI_PROJECT; the BN = 256 predictor layers run
-// as 2-CTA clusters on vertically adjacent tiles that share one multicast B tile):
+// Structure (one CTA per SM, 6 warps; 8 for EPI_PROJECT):
 //   warp 0      one thread issues TMA loads of 128x64 (A) and BNx64 (B) bf16 tiles, 128-byte
 //               swizzled, into a STAGES-deep shared-memory ring (mbarrier full/empty).
 //   warp 1      allocates TMEM (2 accumulators x BN fp32 columns); one thread issues
 //               tcgen05.mma (M=128, N=BN, K=16) x 4 per stage and commits to mbarriers.
+//   CG2 (the BN = 256 predictor layers): 2-CTA clusters run 2-SM MMAs (cta_group::2,
+//               M = 256): each CTA loads its 128 A rows and half of the B tile, both
+//               complete on the leader's full barrier, the leader's thread issues the MMAs and
+//               its commits release the stage and the accumulator in both CTAs.
 //   warps 2-5   epilogue: tcgen05.ld the accumulator (one TMEM lane = one output row per
 //               thread), apply bias / GELU / RoPE, store (bf16, bf16 hi/lo pair, or fp32);
 //               release the accumulator so the
@@ -45,6 +48,8 @@ struct KArgs {
   const int* col_count;
   int b_base;
   ProjArgs proj;
+  int a_kwrap;
+  const float* biasf;
 };
 
 __device__ __forceinline__ float gelu_erf(float x) {
@@ -58,11 +63,11 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
 
 constexpr int kProjMaxBasis = 128;             // EPI_PROJECT: R0 basis size supported
 
-template <int BN, int STAGES, int EPI>
+template <int BN, int STAGES, int EPI, bool CG2>
 struct Smem {
   static constexpr bool PROJ = EPI == EPI_PROJECT;
   static constexpr uint32_t A_BYTES = kBM * kBK * 2;
-  static constexpr uint32_t B_BYTES = BN * kBK * 2;
+  static constexpr uint32_t B_BYTES = (CG2 ? BN / 2 : BN) * kBK * 2;   // CG2: this CTA's half
   static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr uint32_t TILES = STAGES * STAGE_BYTES;
   static constexpr uint32_t BARS = (2 * STAGES + 5 + (PROJ ? 5 : 0)) * 8;
@@ -74,10 +79,13 @@ struct Smem {
   static constexpr int THREADS = PROJ ? 256 : 192;   // + 2 warps summing ||v||^2 for EPI_PROJECT
 };
 
+// Selection value, squared: p^2 * rho^(2 lambda) orders candidates like p * rho^lambda (both are
+// >= 0) and needs no square root for lambda = 1.  rho^2 = r2 unless r2 <= tau ||v||^2 (then 0).
 __device__ __forceinline__ float proj_value(float p, float r2, float sq, float lam, float tau) {
-  if (lam == 0.f) return p > 0.f ? p : 0.f;
+  if (!(p > 0.f)) return 0.f;
+  if (lam == 0.f) return p * p;
   if (!(r2 > tau * sq) || !(r2 > 0.f)) return 0.f;
-  const float v = lam == 1.f ? p * sqrtf(r2) : p * powf(r2, 0.5f * lam);
+  const float v = lam == 1.f ? (p * p) * r2 : (p * p) * powf(r2, lam);
   return v > 0.f ? v : 0.f;
 }
 
@@ -100,13 +108,12 @@ __device__ __forceinline__ TileCoord tile_coord(const KArgs& a, int t, int m_uni
   return c;
 }
 
-template <int BN, int STAGES, int EPI, bool PAIR>
-__global__ void __launch_bounds__(Smem<BN, STAGES, EPI>::THREADS, 1)
+template <int BN, int STAGES, int EPI, bool CG2>
+__global__ void __launch_bounds__(Smem<BN, STAGES, EPI, CG2>::THREADS, 1)
 gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, KArgs a) {
-  using S = Smem<BN, STAGES, EPI>;
-  constexpr uint32_t IDESC = idesc_bf16(kBM, BN);
-  // PAIR: launched as 2-CTA clusters; each CTA loads half of the shared B tile and multicasts
-  // it to both, and every MMA commit releases the stage in both CTAs.
+  using S = Smem<BN, STAGES, EPI, CG2>;
+  constexpr bool PAIR = CG2;
+  constexpr uint32_t IDESC = idesc_bf16(CG2 ? 2 * kBM : kBM, BN);
   const uint32_t crank = PAIR ? cluster_ctarank() : 0u;
   const int unit0 = PAIR ? static_cast<int>(blockIdx.x >> 1) : static_cast<int>(blockIdx.x);
   const int units_step = PAIR ? static_cast<int>(gridDim.x >> 1) : static_cast<int>(gridDim.x);
@@ -131,8 +138,9 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
-    for (int s = 0; s < STAGES; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], S::PROJ ? 3 : (PAIR ? 2 : 1)); }
-    for (int i = 0; i < 2; ++i) { mbar_init(&tfull[i], 1); mbar_init(&tempty[i], 128); }
+    for (int s = 0; s < STAGES; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], S::PROJ ? 3 : 1); }
+    // tempty: one arrive per epilogue warp (of both CTAs with CG2, on the leader's barrier)
+    for (int i = 0; i < 2; ++i) { mbar_init(&tfull[i], 1); mbar_init(&tempty[i], CG2 ? 8 : 4); }
     mbar_init(drain, 1);
     if constexpr (S::PROJ) {
       for (int i = 0; i < 2; ++i) { mbar_init(&nfull[i], 2); mbar_init(&nempty[i], 128); }
@@ -142,8 +150,11 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     fence_mbar_init();
   }
   if (warp == 0 && lane == 0) { tma_prefetch_desc(&tmA); tma_prefetch_desc(&tmB); }
-  if (warp == 1) { tmem_alloc(tmem_slot, S::TMEM_COLS); tmem_relinquish(); }
-  if constexpr (PAIR) cluster_sync();             // peer barriers initialised before any multicast
+  if (warp == 1) {
+    if constexpr (CG2) { tmem_alloc_cg2(tmem_slot, S::TMEM_COLS); tmem_relinquish_cg2(); }
+    else { tmem_alloc(tmem_slot, S::TMEM_COLS); tmem_relinquish(); }
+  }
+  if constexpr (PAIR) cluster_sync();             // peer barriers initialised before any remote arrive
   else __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
@@ -153,6 +164,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   const int n_tiles = (a.N + BN - 1) / BN;
   const int total = a.batch * m_units * n_tiles;
   const int KB = a.K / kBK;
+  auto a_k = [&](int kb) { return a.a_kwrap > 0 ? (kb * kBK) % a.a_kwrap : kb * kBK; };
 
   if (warp == 0) {
     if (lane == 0) {
@@ -169,27 +181,30 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         const int brow = (a.b_off ? __ldg(a.b_off + c.b) : c.b * a.b_row_stride + a.b_base) + c.n_blk * BN;
         for (int kb = 0; kb < KB; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1, a.status, abort_flag)) { ok = false; break; }
-          mbar_arrive_expect_tx(&full[stage], S::STAGE_BYTES);
-          tma_load_2d(sA + stage * S::A_BYTES, &tmA, &full[stage], kb * kBK, arow);
-          if constexpr (PAIR) {
-            tma_load_2d_mc(sB + stage * S::B_BYTES + crank * (S::B_BYTES / 2), &tmB, &full[stage], kb * kBK,
-                           brow + static_cast<int>(crank) * (BN / 2), static_cast<uint16_t>(3));
+          if constexpr (CG2) {
+            // both CTAs' copies complete on the leader's full barrier, which expects them all
+            if (crank == 0) mbar_arrive_expect_tx(&full[stage], 2 * S::STAGE_BYTES);
+            const uint32_t fb = mapa_u32(&full[stage], 0);
+            tma_load_2d_cg2(sA + stage * S::A_BYTES, &tmA, fb, a_k(kb), arow);
+            tma_load_2d_cg2(sB + stage * S::B_BYTES, &tmB, fb, kb * kBK, brow + static_cast<int>(crank) * (BN / 2));
           } else {
+            mbar_arrive_expect_tx(&full[stage], S::STAGE_BYTES);
+            tma_load_2d(sA + stage * S::A_BYTES, &tmA, &full[stage], a_k(kb), arow);
             tma_load_2d(sB + stage * S::B_BYTES, &tmB, &full[stage], kb * kBK, brow);
           }
           last_par[stage] = static_cast<int>(phase);
           if (++stage == STAGES) { stage = 0; phase ^= 1; }
         }
       }
-      if (!ok) {   // let every copy already in flight land before the CTA exits
+      if (!ok && crank == 0) {   // let every copy already in flight land before the CTA exits
         for (int s = 0; s < STAGES; ++s)
           if (last_par[s] >= 0) mbar_wait(&full[s], static_cast<uint32_t>(last_par[s]), a.status, nullptr);
       }
     }
     __syncwarp();
   } else if (warp == 1) {
-    if (lane == 0) {
-      // ---------------------------------------------------------------- MMA issuer
+    if (lane == 0 && crank == 0) {
+      // ---------------------------------------------------------------- MMA issuer (CG2: leader)
       uint32_t stage = 0, phase = 0, acc = 0, acc_phase = 0;
       bool issued = false, ok = true;
       for (int t = unit0; t < total && ok; t += units_step) {
@@ -203,21 +218,29 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           tc_fence_after();
           const uint32_t a0 = smem_u32(sA + stage * S::A_BYTES);
           const uint32_t b0 = smem_u32(sB + stage * S::B_BYTES);
+          if constexpr (CG2) {
 #pragma unroll
-          for (int k = 0; k < kBK / 16; ++k)
-            umma_bf16(d_tmem, desc_sw128(a0 + k * 32), desc_sw128(b0 + k * 32), IDESC, (kb | k) != 0);
-          if constexpr (PAIR) umma_commit_mc(&empty[stage], static_cast<uint16_t>(3));
-          else umma_commit(&empty[stage]);
+            for (int k = 0; k < kBK / 16; ++k)
+              umma_bf16_cg2(d_tmem, desc_sw128(a0 + k * 32), desc_sw128(b0 + k * 32), IDESC, (kb | k) != 0);
+            umma_commit_cg2_mc(&empty[stage], static_cast<uint16_t>(3));
+          } else {
+#pragma unroll
+            for (int k = 0; k < kBK / 16; ++k)
+              umma_bf16(d_tmem, desc_sw128(a0 + k * 32), desc_sw128(b0 + k * 32), IDESC, (kb | k) != 0);
+            umma_commit(&empty[stage]);
+          }
           issued = true;
           if (++stage == STAGES) { stage = 0; phase ^= 1; }
         }
         if (!ok) break;
-        umma_commit(&tfull[acc]);
+        if constexpr (CG2) umma_commit_cg2_mc(&tfull[acc], static_cast<uint16_t>(3));
+        else umma_commit(&tfull[acc]);
         acc ^= 1;
         if (acc == 0) acc_phase ^= 1;
       }
       if (issued) {   // every MMA of this CTA has completed before TMEM is released
-        umma_commit(drain);
+        if constexpr (CG2) umma_commit_cg2(drain);
+        else umma_commit(drain);
         mbar_wait(drain, 0, a.status, nullptr);
       }
     }
@@ -324,7 +347,11 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
 #pragma unroll
               for (int u = 0; u < 8; ++u) {
                 const float2 cs = __ldg(rt + ch * 32 + j + u);
-                const float x1 = __uint_as_float(r1[j + u]), x2 = __uint_as_float(r2[j + u]);
+                float x1 = __uint_as_float(r1[j + u]), x2 = __uint_as_float(r2[j + u]);
+                if (a.biasf) {
+                  x1 += __ldg(a.biasf + ch * 32 + j + u);
+                  x2 += __ldg(a.biasf + HALF + ch * 32 + j + u);
+                }
                 o1[u] = x1 * cs.x - x2 * cs.y;
                 o2[u] = x2 * cs.x + x1 * cs.y;
               }
@@ -513,7 +540,11 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         }
       }
       tc_fence_before();
-      mbar_arrive(&tempty[acc]);
+      __syncwarp();
+      if (lane == 0) {
+        if constexpr (CG2) mbar_arrive_cluster(mapa_u32(&tempty[acc], 0));
+        else mbar_arrive(&tempty[acc]);
+      }
       acc ^= 1;
       if (acc == 0) acc_phase ^= 1;
     }
@@ -570,11 +601,12 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       }
     }
   }
-  if constexpr (PAIR) cluster_sync();             // no multicast or remote arrive still in flight
+  if constexpr (PAIR) cluster_sync();             // no commit or remote arrive still in flight
   else __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, S::TMEM_COLS);
+    if constexpr (CG2) tmem_dealloc_cg2(tmem_base, S::TMEM_COLS);
+    else tmem_dealloc(tmem_base, S::TMEM_COLS);
   }
 }
 
@@ -607,9 +639,9 @@ bool make_map(CUtensorMap* m, const void* base, long long rows, int K, int box_r
 
 template <int BN, int STAGES, int EPI, bool PAIR = false>
 cudaError_t run(const GemmDesc& d, const KArgs& ka, int num_sms, cudaStream_t st) {
-  using S = Smem<BN, STAGES, EPI>;
+  using S = Smem<BN, STAGES, EPI, PAIR>;
   CUtensorMap ta, tb;
-  if (!make_map(&ta, d.A, d.a_rows_total, d.K, kBM)) return cudaErrorInvalidValue;
+  if (!make_map(&ta, d.A, d.a_rows_total, d.a_kwrap > 0 ? d.a_kwrap : d.K, kBM)) return cudaErrorInvalidValue;
   if (!make_map(&tb, d.B, d.b_rows_total, d.K, PAIR ? BN / 2 : BN)) return cudaErrorInvalidValue;
   auto kern = gemm_tc_kernel<BN, STAGES, EPI, PAIR>;
   static bool attr_set = false;
@@ -648,6 +680,7 @@ cudaError_t run(const GemmDesc& d, const KArgs& ka, int num_sms, cudaStream_t st
 
 cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t st) {
   if (d.K <= 0 || d.K % kBK != 0 || d.M < 0 || d.N <= 0 || d.batch <= 0) return cudaErrorInvalidValue;
+  if (d.a_kwrap < 0 || d.a_kwrap % kBK != 0 || d.a_kwrap > d.K) return cudaErrorInvalidValue;
   if ((reinterpret_cast<uintptr_t>(d.A) | reinterpret_cast<uintptr_t>(d.B)) & 15) return cudaErrorInvalidValue;
   if (d.M == 0) return cudaSuccess;
   // every output row and column block is written with 16-byte vector stores
@@ -673,6 +706,7 @@ cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t st) {
   ka.split_kind = d.split_kind; ka.scale = d.scale; ka.aux = d.aux; ka.b_off = d.b_off;
   ka.stats = d.stats; ka.stat_ld = d.stat_ld; ka.col_count = d.col_count;
   ka.b_base = d.b_base; ka.proj = d.proj;
+  ka.a_kwrap = d.a_kwrap; ka.biasf = d.biasf;
   switch (d.epi) {
     case EPI_GELU_BF16:
       if (d.N % 256 == 0) return run<256, 4, EPI_GELU_BF16>(d, ka, num_sms, st);
@@ -688,11 +722,11 @@ cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t st) {
       if (d.N == 256) return run<256, 4, EPI_ROPE_F32>(d, ka, num_sms, st);
       return cudaErrorInvalidValue;
     case EPI_GELU_SPLIT:
-      if (d.N % 256 == 0) return run<256, 4, EPI_GELU_SPLIT, true>(d, ka, num_sms, st);
+      if (d.N % 256 == 0) return run<256, 6, EPI_GELU_SPLIT, true>(d, ka, num_sms, st);
       if (d.N % 64 == 0) return run<64, 8, EPI_GELU_SPLIT>(d, ka, num_sms, st);
       return cudaErrorInvalidValue;
     case EPI_BIAS_SPLIT:
-      if (d.N % 256 == 0) return run<256, 4, EPI_BIAS_SPLIT, true>(d, ka, num_sms, st);
+      if (d.N % 256 == 0) return run<256, 6, EPI_BIAS_SPLIT, true>(d, ka, num_sms, st);
       if (d.N % 64 == 0) return run<64, 8, EPI_BIAS_SPLIT>(d, ka, num_sms, st);
       return cudaErrorInvalidValue;
     case EPI_ROPE_SPLIT3:

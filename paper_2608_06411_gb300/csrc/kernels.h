@@ -61,10 +61,21 @@ struct GemmDesc {
   // B rows at b * b_row_stride + b_base
   int b_base = 0;
   ProjArgs proj{};
+  // A has a_kwrap columns; its K coordinate wraps (k mod a_kwrap), so a K-segment of A can
+  // be read twice against different B segments (0: A has K columns)
+  int a_kwrap = 0;
+  const float* biasf = nullptr;         // EPI_ROPE_SPLIT3: fp32 bias [N] added before RoPE
 };
 
 // Returns cudaSuccess, or an error for an unsupported shape (cudaErrorInvalidValue).
 cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t st);
+
+// Folds a projection after a linear layer into one matrix: W = Wp W2 ([dp, Dh] = [dp, Dh] x
+// [Dh, Dh]) and bias = Wp b2, accumulated in fp64 from the bf16 inputs.  W is stored as the
+// bf16 rows [hi | hi | lo] ([dp, 3 Dh], hi = bf16(W), lo = bf16(W - hi)) for activations laid
+// out [hi | lo] and read with the K-wrap [hi | lo | hi]; bias in fp32.
+cudaError_t launch_fold_weights(const void* Wp, const void* W2, const void* b2, int dp, int Dh, void* out,
+                                float* bias_out, cudaStream_t st);
 
 // Squared row norms of bf16 rows: out[r] = sum_d x[r, d]^2 (fp32).
 cudaError_t launch_row_sqnorm(const void* x, long long rows, int D, float* out, cudaStream_t st);

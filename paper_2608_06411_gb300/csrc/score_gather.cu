@@ -1,4 +1,4 @@
-// Eq. 3 softmax statistics combine, squared row norms, and the compaction gather.
+// Eq. 3 softmax statistics combine, weight folding, squared row norms, and the compaction gather.
 #include <algorithm>
 
 #include "kernels.h"
@@ -74,7 +74,42 @@ __global__ void sum_tiles_kernel(const float* __restrict__ part, int N, int n_ti
   scores[i] = s;
 }
 
+// out[p, i] (three bf16 segments) = sum_j Wp[p, j] W2[j, i]; thread = (p, i), fp64 sums.
+__global__ void fold_weights_kernel(const __nv_bfloat16* __restrict__ Wp, const __nv_bfloat16* __restrict__ W2,
+                                    const __nv_bfloat16* __restrict__ b2, int dp, int Dh,
+                                    __nv_bfloat16* __restrict__ out, float* __restrict__ bias_out) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x, p = blockIdx.y;
+  if (i < Dh) {
+    double acc = 0.0;
+    for (int j = 0; j < Dh; ++j)
+      acc += static_cast<double>(__bfloat162float(Wp[static_cast<long long>(p) * Dh + j])) *
+             static_cast<double>(__bfloat162float(W2[static_cast<long long>(j) * Dh + i]));
+    const __nv_bfloat16 hi = __float2bfloat16_rn(static_cast<float>(acc));
+    const __nv_bfloat16 lo = __float2bfloat16_rn(static_cast<float>(acc - static_cast<double>(__bfloat162float(hi))));
+    __nv_bfloat16* row = out + static_cast<long long>(p) * 3 * Dh;
+    row[i] = hi;
+    row[Dh + i] = hi;
+    row[2 * Dh + i] = lo;
+  }
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    double acc = 0.0;
+    for (int j = 0; j < Dh; ++j)
+      acc += static_cast<double>(__bfloat162float(Wp[static_cast<long long>(p) * Dh + j])) *
+             static_cast<double>(__bfloat162float(b2[j]));
+    bias_out[p] = static_cast<float>(acc);
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_fold_weights(const void* Wp, const void* W2, const void* b2, int dp, int Dh, void* out,
+                                float* bias_out, cudaStream_t st) {
+  if (dp <= 0 || Dh <= 0) return cudaErrorInvalidValue;
+  fold_weights_kernel<<<dim3((Dh + 127) / 128, dp), 128, 0, st>>>(
+      static_cast<const __nv_bfloat16*>(Wp), static_cast<const __nv_bfloat16*>(W2),
+      static_cast<const __nv_bfloat16*>(b2), dp, Dh, static_cast<__nv_bfloat16*>(out), bias_out);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_stats_combine(const float2* part, int B, int nparts, int ld, const int* lens, float2* fin,
                                  cudaStream_t st) {

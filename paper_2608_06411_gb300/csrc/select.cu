@@ -10,19 +10,25 @@
 // that time (the same quantities Gram-Schmidt would produce, in exact arithmetic).
 //
 // The greedy picks are sequential, but the Gram entries they need are dense products
-// <v_i, v_j>, computed on the tensor cores in blocks.  Selection proceeds in rounds:
+// <v_i, v_j>, computed on the tensor cores in blocks.
+//   R0     : the first K0 picks (top-K0 by p_hat) are forced, in p_hat order; their basis is
+//            the Cholesky factor of G[R0, R0] (sel_chol_kernel).  A tensor-core projection
+//            of every token on that basis (gemm_tc.cu) then gives every candidate its exact
+//            value.
+// Later picks proceed in rounds:
 //   choose : active set A = the s candidates with the largest value bound U (a stale
 //            value, or p_hat * ||v||^lambda for tokens never evaluated; values only shrink
 //            as B grows, so U is always an upper bound); gather their rows and the rows of
 //            new basis tokens into a compact buffer Vg.
-//   gram   : G_blk = Vg[A] Vg[A u basis]^T on tcgen05 (gemm_tc.cu).
-//   greedy : bring each A member's Cholesky coordinates up to date (exact values), then
-//            pick while the best exact value in A beats the largest bound outside A (theta):
+//   gram   : G_blk = Vg[A] Vg[A u new basis]^T on tcgen05 (gemm_tc.cu).
+//   update : bring each A member's coordinates up to date (exact values).
+//   greedy : pick while the best exact value in A beats the largest bound outside A (theta):
 //            such a pick is the exact argmax over all candidates.  Each pick updates the
 //            other A members.  Values are compared as the 64-bit key (value bits, ~index),
-//            i.e. value descending, ties to the lower index.
-// The first K0 picks (R0, top-K0 by p_hat) are forced, in p_hat order.  The result equals
-// the eager fp32 greedy whatever s is; s only changes how much work is batched.
+//            i.e. value descending, ties to the lower index; they are held squared
+//            (p^2 rho^(2 lambda), same order, no square root).
+// The result equals the eager fp32 greedy whatever s is; s only changes how much work is
+// batched.
 #include <algorithm>
 
 #include "ptx.cuh"
@@ -40,10 +46,13 @@ __device__ __forceinline__ int key_index(uint64_t key) {
   return static_cast<int>(0xFFFFFFFFu - static_cast<uint32_t>(key & 0xFFFFFFFFull));
 }
 
+// Selection value, squared: p^2 * rho^(2 lambda) orders candidates like p * rho^lambda (both are
+// >= 0) and needs no square root for lambda = 1.  rho^2 = r2 unless r2 <= tau ||v||^2 (then 0).
 __device__ __forceinline__ float sel_value(float p, float r2, float sq, float lam, float tau) {
-  if (lam == 0.f) return p > 0.f ? p : 0.f;
+  if (!(p > 0.f)) return 0.f;
+  if (lam == 0.f) return p * p;
   if (!(r2 > tau * sq) || !(r2 > 0.f)) return 0.f;
-  const float v = lam == 1.f ? p * sqrtf(r2) : p * powf(r2, 0.5f * lam);
+  const float v = lam == 1.f ? (p * p) * r2 : (p * p) * powf(r2, lam);
   return v > 0.f ? v : 0.f;
 }
 
@@ -139,7 +148,7 @@ __host__ __device__ inline int pow2_at_least(int n) {
 }
 
 // ------------------------------------------------------------------ init
-// U = p_hat * ||v||^lambda, r2 = ||v||^2, nothing cached; R0 = top-K0 by p_hat, in order.
+// U = (p_hat * ||v||^lambda)^2, r2 = ||v||^2, nothing cached; R0 = top-K0 by p_hat, in order.
 __global__ void __launch_bounds__(1024) sel_init_kernel(SelState s) {
   extern __shared__ uint64_t sh64[];
   const int b = blockIdx.x;

@@ -16,7 +16,7 @@ struct SelState {
   const float* scores;            // [B, N] p_hat
   const void* V;                  // [B, N, D] bf16
   const float* sqn;               // [B, N] ||v||^2
-  float* U;                       // [B, N] value bound / exact value
+  float* U;                       // [B, N] squared value bound / exact squared value (sel_value)
   float* r2;                      // [B, N] residual^2 as of cstep
   int32_t* cstep;                 // [B, N] basis coordinates cached
   uint8_t* state;                 // [B, N] 0 candidate, 1 retained
