@@ -155,7 +155,7 @@ int ensure_rope(map_ctx* c, int rows_needed) {
     for (int i = 0; i < half; ++i) {
       const double f = std::pow(static_cast<double>(c->cfg.rope_theta), -2.0 * i / c->cfg.dp);
       const double a = p * f;
-      tab[static_cast<size_t>(p) * half + i] = make_float2(static_cast<float>(std::cos(a)), static_cast<float>(std::sin(a)));
+      tab[static_cast<size_t>(i) * rows + p] = make_float2(static_cast<float>(std::cos(a)), static_cast<float>(std::sin(a)));
     }
   MAP_TRY(ensure(c->rope, tab.size() * sizeof(float2)));
   CU_TRY(cudaMemcpy(c->rope.p, tab.data(), tab.size() * sizeof(float2), cudaMemcpyHostToDevice));
@@ -215,14 +215,16 @@ int predictor_branch(map_ctx* c, const void* x, long long rows, const void* w1, 
     MAP_TRY(gemm(c, d, st));
   }
   {
-    // K = 3 Dh: A segments [hi | lo | hi] (the K coordinate wraps at 2 Dh) against
-    // [Wf_hi | Wf_hi | Wf_lo]: h_hi Wf_hi + h_lo Wf_hi + h_hi Wf_lo
+    // K = 3 Dh: h_hi Wf_hi + h_hi Wf_lo + h_lo Wf_hi, A = [hi | lo] against
+    // [Wf_hi | Wf_hi | Wf_lo], each block of h_hi used twice in a row (split3 K order)
     Timed t(c, st, tid_p);
     GemmDesc d = linear_desc(c, h1.p, rows, 3 * g.Dh, wf, g.dp, nullptr, out3, mapk::EPI_ROPE_SPLIT3);
     d.a_kwrap = 2 * g.Dh;
+    d.split3 = 1;
     d.biasf = bf;
     d.ldc = 3LL * g.dp;
     d.rope = static_cast<const float2*>(c->rope.p);
+    d.rope_ld = c->rope_rows;
     d.pos = g.rope_on ? pos : nullptr;      // without RoPE every position is 0: cos 1, sin 0
     d.pos_mod = g.rope_on ? pos_mod : 1;
     d.split_kind = split_kind;

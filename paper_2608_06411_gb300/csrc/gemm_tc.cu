@@ -39,7 +39,7 @@ struct KArgs {
   const int* n_limit;
   void* C; long long ldc; long long c_batch_stride;
   const __nv_bfloat16* bias;
-  const float2* rope; int rope_half;
+  const float2* rope; int rope_half; int rope_ld;
   const int* pos; int pos_mod;
   int* status;
   int split_kind; float scale; float* aux;
@@ -49,6 +49,7 @@ struct KArgs {
   int b_base;
   ProjArgs proj;
   int a_kwrap;
+  int split3;
   const float* biasf;
 };
 
@@ -164,7 +165,22 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   const int n_tiles = (a.N + BN - 1) / BN;
   const int total = a.batch * m_units * n_tiles;
   const int KB = a.K / kBK;
-  auto a_k = [&](int kb) { return a.a_kwrap > 0 ? (kb * kBK) % a.a_kwrap : kb * kBK; };
+  // K block kb -> (A column, B column)
+  auto kcols = [&](int kb, int& ac, int& bc) {
+    if (a.split3) {
+      const int nbk = KB / 3;
+      if (kb < 2 * nbk) {
+        const int j = kb >> 1;
+        ac = j * kBK;
+        bc = (kb & 1) ? (2 * nbk + j) * kBK : j * kBK;
+      } else {
+        ac = bc = (kb - nbk) * kBK;
+      }
+    } else {
+      ac = a.a_kwrap > 0 ? (kb * kBK) % a.a_kwrap : kb * kBK;
+      bc = kb * kBK;
+    }
+  };
 
   if (warp == 0) {
     if (lane == 0) {
@@ -181,16 +197,18 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         const int brow = (a.b_off ? __ldg(a.b_off + c.b) : c.b * a.b_row_stride + a.b_base) + c.n_blk * BN;
         for (int kb = 0; kb < KB; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1, a.status, abort_flag)) { ok = false; break; }
+          int ac, bc;
+          kcols(kb, ac, bc);
           if constexpr (CG2) {
             // both CTAs' copies complete on the leader's full barrier, which expects them all
             if (crank == 0) mbar_arrive_expect_tx(&full[stage], 2 * S::STAGE_BYTES);
             const uint32_t fb = mapa_u32(&full[stage], 0);
-            tma_load_2d_cg2(sA + stage * S::A_BYTES, &tmA, fb, a_k(kb), arow);
-            tma_load_2d_cg2(sB + stage * S::B_BYTES, &tmB, fb, kb * kBK, brow + static_cast<int>(crank) * (BN / 2));
+            tma_load_2d_cg2(sA + stage * S::A_BYTES, &tmA, fb, ac, arow);
+            tma_load_2d_cg2(sB + stage * S::B_BYTES, &tmB, fb, bc, brow + static_cast<int>(crank) * (BN / 2));
           } else {
             mbar_arrive_expect_tx(&full[stage], S::STAGE_BYTES);
-            tma_load_2d(sA + stage * S::A_BYTES, &tmA, &full[stage], a_k(kb), arow);
-            tma_load_2d(sB + stage * S::B_BYTES, &tmB, &full[stage], kb * kBK, brow);
+            tma_load_2d(sA + stage * S::A_BYTES, &tmA, &full[stage], ac, arow);
+            tma_load_2d(sB + stage * S::B_BYTES, &tmB, &full[stage], bc, brow);
           }
           last_par[stage] = static_cast<int>(phase);
           if (++stage == STAGES) { stage = 0; phase ^= 1; }
@@ -303,7 +321,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         float* out = reinterpret_cast<float*>(a.C) + crow;
         int pos = 0;
         if (row_ok) pos = a.pos ? __ldg(a.pos + row) : row % a.pos_mod;
-        const float2* rt = a.rope + static_cast<long long>(pos) * a.rope_half;
+        const float2* rt = a.rope + pos;
 #pragma unroll 1
         for (int ch = 0; ch < HALF / 32; ++ch) {
           uint32_t r1[32], r2[32];
@@ -315,7 +333,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
               float o1[4], o2[4];
 #pragma unroll
               for (int u = 0; u < 4; ++u) {
-                const float2 cs = __ldg(rt + ch * 32 + j + u);
+                const float2 cs = __ldg(rt + static_cast<long long>(ch * 32 + j + u) * a.rope_ld);
                 const float x1 = __uint_as_float(r1[j + u]), x2 = __uint_as_float(r2[j + u]);
                 o1[u] = x1 * cs.x - x2 * cs.y;
                 o2[u] = x2 * cs.x + x1 * cs.y;
@@ -332,7 +350,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         float* aux = a.aux ? a.aux + static_cast<long long>(row) * BN : nullptr;
         int pos = 0;
         if (row_ok) pos = a.pos ? __ldg(a.pos + row) : row % a.pos_mod;
-        const float2* rt = a.rope + static_cast<long long>(pos) * a.rope_half;
+        const float2* rt = a.rope + pos;
         // segment order: keys [hi, lo, hi], queries [hi, hi, lo]
         const int seg_lo = a.split_kind == 0 ? 1 : 2;
 #pragma unroll 1
@@ -346,7 +364,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
               float o1[8], o2[8];
 #pragma unroll
               for (int u = 0; u < 8; ++u) {
-                const float2 cs = __ldg(rt + ch * 32 + j + u);
+                const float2 cs = __ldg(rt + static_cast<long long>(ch * 32 + j + u) * a.rope_ld);
                 float x1 = __uint_as_float(r1[j + u]), x2 = __uint_as_float(r2[j + u]);
                 if (a.biasf) {
                   x1 += __ldg(a.biasf + ch * 32 + j + u);
@@ -438,6 +456,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       } else if constexpr (EPI == EPI_PROJECT) {
         // Cholesky coordinates of token `row` on the R0 basis by forward substitution,
         // 32 basis vectors at a time: e_beta = (g_beta - sum_{q<beta} L[beta][q] e_q) / r_beta.
+        // Each finished chunk of e replaces its g columns in TMEM, where later chunks read it.
         const ProjArgs& pj = a.proj;
         const int nb0 = min(kProjMaxBasis, __ldg(pj.nbasis + c.b));
         const long long tok = static_cast<long long>(c.b) * a.M + row;
@@ -447,34 +466,58 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         float r2 = sq;
 #pragma unroll 1
         for (int b0 = 0; b0 < nb0; b0 += 32) {
-          uint32_t g[32];
-          tmem_ld32(tbase + b0, g);
-          if (!alive) continue;
+          float accv[32];
+          {
+            uint32_t g[32];
+            tmem_ld32(tbase + b0, g);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) accv[i] = __uint_as_float(g[i]);
+          }
           const int b1 = min(nb0, b0 + 32);
-          float accv[32], e[32];
+#pragma unroll 1
+          for (int qc = 0; qc < b0; qc += 8) {
+            uint32_t ep[8];
+            tmem_ld8(tbase + qc, ep);
+            if (alive) {
 #pragma unroll
-          for (int i = 0; i < 32; ++i) accv[i] = __uint_as_float(g[i]);
-          for (int q = 0; q < b0; q += 4) {
-            const float4 eq = *reinterpret_cast<const float4*>(erow + q);
+              for (int qq = 0; qq < 8; qq += 4) {
 #pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              const float4 l = *reinterpret_cast<const float4*>(Lsm + (b0 + i) * kProjMaxBasis + q);
-              accv[i] = fmaf(-l.x, eq.x, accv[i]);
-              accv[i] = fmaf(-l.y, eq.y, accv[i]);
-              accv[i] = fmaf(-l.z, eq.z, accv[i]);
-              accv[i] = fmaf(-l.w, eq.w, accv[i]);
+                for (int i = 0; i < 32; ++i) {
+                  const float4 l = *reinterpret_cast<const float4*>(Lsm + (b0 + i) * kProjMaxBasis + qc + qq);
+                  accv[i] = fmaf(-l.x, __uint_as_float(ep[qq]), accv[i]);
+                  accv[i] = fmaf(-l.y, __uint_as_float(ep[qq + 1]), accv[i]);
+                  accv[i] = fmaf(-l.z, __uint_as_float(ep[qq + 2]), accv[i]);
+                  accv[i] = fmaf(-l.w, __uint_as_float(ep[qq + 3]), accv[i]);
+                }
+              }
             }
           }
+          // the triangle, in place: accv[i] becomes e_{b0+i}
 #pragma unroll
           for (int i = 0; i < 32; ++i) {
-            if (b0 + i < b1) {
-              float v = accv[i];
+            float v = 0.f;
+            if (alive && b0 + i < b1) {
+              v = accv[i];
 #pragma unroll
-              for (int q = 0; q < i; ++q) v = fmaf(-Lsm[(b0 + i) * kProjMaxBasis + b0 + q], e[q], v);
-              e[i] = v * rinv_sm[b0 + i];
-              erow[b0 + i] = e[i];
-              r2 = fmaf(-e[i], e[i], r2);
+              for (int q = 0; q < i; ++q) v = fmaf(-Lsm[(b0 + i) * kProjMaxBasis + b0 + q], accv[q], v);
+              v *= rinv_sm[b0 + i];
+              r2 = fmaf(-v, v, r2);
             }
+            accv[i] = v;
+          }
+          if (alive) {
+#pragma unroll
+            for (int i = 0; i < 32; i += 4)
+              if (b0 + i + 4 <= b1)
+                *reinterpret_cast<float4*>(erow + b0 + i) = make_float4(accv[i], accv[i + 1], accv[i + 2], accv[i + 3]);
+              else
+                for (int u = i; u < b1 - b0 && u < i + 4; ++u) erow[b0 + u] = accv[u];
+          }
+          if (b0 + 32 < nb0) {
+            uint32_t eb[32];
+#pragma unroll
+            for (int i = 0; i < 32; ++i) eb[i] = __float_as_uint(accv[i]);
+            tmem_st32(tbase + b0, eb);
           }
         }
         if (alive) {
@@ -681,6 +724,7 @@ cudaError_t run(const GemmDesc& d, const KArgs& ka, int num_sms, cudaStream_t st
 cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t st) {
   if (d.K <= 0 || d.K % kBK != 0 || d.M < 0 || d.N <= 0 || d.batch <= 0) return cudaErrorInvalidValue;
   if (d.a_kwrap < 0 || d.a_kwrap % kBK != 0 || d.a_kwrap > d.K) return cudaErrorInvalidValue;
+  if (d.split3 && (d.K % (3 * kBK) != 0 || d.a_kwrap != 2 * (d.K / 3))) return cudaErrorInvalidValue;
   if ((reinterpret_cast<uintptr_t>(d.A) | reinterpret_cast<uintptr_t>(d.B)) & 15) return cudaErrorInvalidValue;
   if (d.M == 0) return cudaSuccess;
   // every output row and column block is written with 16-byte vector stores
@@ -701,12 +745,12 @@ cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t st) {
   ka.a_row_stride = d.a_row_stride; ka.b_row_stride = d.b_row_stride;
   ka.n_limit = d.n_limit; ka.C = d.C; ka.ldc = d.ldc; ka.c_batch_stride = d.c_batch_stride;
   ka.bias = static_cast<const __nv_bfloat16*>(d.bias);
-  ka.rope = d.rope; ka.rope_half = d.rope_half; ka.pos = d.pos; ka.pos_mod = d.pos_mod > 0 ? d.pos_mod : 1;
+  ka.rope = d.rope; ka.rope_half = d.rope_half; ka.rope_ld = d.rope_ld; ka.pos = d.pos; ka.pos_mod = d.pos_mod > 0 ? d.pos_mod : 1;
   ka.status = d.status;
   ka.split_kind = d.split_kind; ka.scale = d.scale; ka.aux = d.aux; ka.b_off = d.b_off;
   ka.stats = d.stats; ka.stat_ld = d.stat_ld; ka.col_count = d.col_count;
   ka.b_base = d.b_base; ka.proj = d.proj;
-  ka.a_kwrap = d.a_kwrap; ka.biasf = d.biasf;
+  ka.a_kwrap = d.a_kwrap; ka.biasf = d.biasf; ka.split3 = d.split3;
   switch (d.epi) {
     case EPI_GELU_BF16:
       if (d.N % 256 == 0) return run<256, 4, EPI_GELU_BF16>(d, ka, num_sms, st);
@@ -729,9 +773,9 @@ cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t st) {
       if (d.N % 256 == 0) return run<256, 6, EPI_BIAS_SPLIT, true>(d, ka, num_sms, st);
       if (d.N % 64 == 0) return run<64, 8, EPI_BIAS_SPLIT>(d, ka, num_sms, st);
       return cudaErrorInvalidValue;
-    case EPI_ROPE_SPLIT3:
+    case EPI_ROPE_SPLIT3:   // dp = 128: 2-SM pairs share the B tile (each CTA loads 64 of its rows)
       if (d.N == 64) return run<64, 8, EPI_ROPE_SPLIT3>(d, ka, num_sms, st);
-      if (d.N == 128) return run<128, 6, EPI_ROPE_SPLIT3>(d, ka, num_sms, st);
+      if (d.N == 128) return run<128, 9, EPI_ROPE_SPLIT3, true>(d, ka, num_sms, st);
       return cudaErrorInvalidValue;
     case EPI_SM_STATS:
       return run<256, 4, EPI_SM_STATS>(d, ka, num_sms, st);
@@ -740,8 +784,8 @@ cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t st) {
     case EPI_PROJECT:
       if (d.N > kProjMaxBasis || d.batch < 1) return cudaErrorInvalidValue;
       return run<128, 4, EPI_PROJECT>(d, ka, num_sms, st);
-    case EPI_F32:
-      return run<128, 6, EPI_F32>(d, ka, num_sms, st);
+    case EPI_F32:   // Gram blocks: one 256 x 256 pair tile per image and 256 columns
+      return run<256, 6, EPI_F32, true>(d, ka, num_sms, st);
     default:
       return cudaErrorInvalidValue;
   }

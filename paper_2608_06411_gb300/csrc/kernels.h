@@ -45,7 +45,8 @@ struct GemmDesc {
   const int* n_limit;                   // per-batch output-column limit (device) or nullptr
   void* C; long long ldc; long long c_batch_stride;   // elements
   const void* bias;                     // bf16 [N] or nullptr
-  const float2* rope; int rope_half;    // (cos, sin) table [pos][rope_half]
+  const float2* rope; int rope_half;    // (cos, sin) table [rope_half][rope_ld]: position-minor, so
+  int rope_ld = 0;                      // lanes (consecutive rows) read consecutive entries
   const int* pos; int pos_mod;          // per-row positions (device) or row % pos_mod
   int epi;
   int* status;
@@ -64,6 +65,10 @@ struct GemmDesc {
   // A has a_kwrap columns; its K coordinate wraps (k mod a_kwrap), so a K-segment of A can
   // be read twice against different B segments (0: A has K columns)
   int a_kwrap = 0;
+  // split3 = 1 (with K = 3 Dh, A = [hi | lo] and B = [W_hi | W_hi | W_lo]): K blocks are taken
+  // as (hi_j, W_hi_j), (hi_j, W_lo_j) for every j, then (lo_j, W_hi_j), so each block of A_hi
+  // is read twice back to back (the second time from L2)
+  int split3 = 0;
   const float* biasf = nullptr;         // EPI_ROPE_SPLIT3: fp32 bias [N] added before RoPE
 };
 
