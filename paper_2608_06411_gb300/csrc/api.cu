@@ -364,6 +364,7 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, 
   MAP_TRY(ensure(c->sbt, static_cast<size_t>(B) * K * 4));
   MAP_TRY(ensure(c->srn, static_cast<size_t>(B) * K * 4));
   MAP_TRY(ensure(c->ssmall, static_cast<size_t>(B) * 4 * 16 + 20 * 256));
+  static_assert(mapk::kReprojMax <= kProjMaxBasis, "re-projection basis limit");
   MAP_TRY(ensure(c->stheta, static_cast<size_t>(B) * 8));
   MAP_TRY(ensure(c->saslot, static_cast<size_t>(B) * S * 4));
   s.sqn = static_cast<float*>(c->sqn.p);
@@ -385,6 +386,9 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, 
   s.gb_lo = carve<int32_t>(sm, B);
   s.gb_hi = carve<int32_t>(sm, B);
   s.gbase = carve<int32_t>(sm, B);
+  s.proj_lim = carve<int32_t>(sm, B);
+  s.blist = carve<int32_t>(sm, B);
+  s.bcount = carve<int32_t>(sm, 1);
   s.done_count = carve<int32_t>(sm, 1);
   s.theta = static_cast<uint64_t*>(c->stheta.p);
   s.aslot = static_cast<int32_t*>(c->saslot.p);
@@ -418,6 +422,7 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, 
     d.M = S; d.N = R; d.K = g.D; d.batch = B; d.n_limit = s.nlimit;
     d.C = s.G; d.ldc = R; d.c_batch_stride = static_cast<long long>(S) * R;
     d.epi = mapk::EPI_F32; d.status = c->status;
+    d.blist = s.blist; d.bcount = s.bcount;     // images still selecting (built by choose)
     const long long cap = 8LL * (K + N / S) + 64;
     long long rounds = 0;
     int burst = (K0 + S - 1) / S + 6;   // rounds queued per host check; finished images skip
@@ -429,23 +434,40 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, 
       CU_TRY(mapk::launch_sel_chol(s, st));
       ++rounds;
       ++c->counters.select_rounds;
-      c->counters.launches += 2;
-      CU_TRY(mapk::launch_sel_proj_prep(s, st));
-      CU_TRY(mapk::launch_sel_gather(s, st));
+      // every candidate's exact value: one tensor-core pass over V against the R0 basis
       GemmDesc pd{};
       pd.A = vis; pd.a_rows_total = BN; pd.a_row_stride = N;
       pd.B = s.Vg; pd.b_rows_total = static_cast<long long>(B) * R; pd.b_row_stride = R; pd.b_base = S;
-      pd.M = N; pd.N = kProjMaxBasis; pd.K = g.D; pd.batch = B; pd.n_limit = nullptr;
+      pd.M = N; pd.N = kProjMaxBasis; pd.K = g.D; pd.batch = B; pd.n_limit = s.proj_lim;
+      pd.blist = s.blist; pd.bcount = s.bcount;   // images to project (built by proj_prep)
       pd.C = nullptr; pd.ldc = 0; pd.c_batch_stride = 0;
       pd.epi = mapk::EPI_PROJECT; pd.status = c->status;
       pd.proj.state = s.state; pd.proj.scores = scores; pd.proj.Ec = s.Ec; pd.proj.KP = KP;
       pd.proj.basis_tok = s.basis_tok; pd.proj.rnorm = s.rnorm; pd.proj.nbasis = s.nbasis; pd.proj.Kcap = K;
       pd.proj.lambda = g.lambda; pd.proj.tau = g.tau;
       pd.proj.r2 = s.r2; pd.proj.U = s.U; pd.proj.sqn = static_cast<float*>(c->sqn.p); pd.proj.cstep = s.cstep;
-      MAP_TRY(gemm(c, pd, st));
-      ++c->counters.launches;
-      CU_TRY(mapk::launch_sel_proj_done(s, st));
-      burst = 6;
+      auto project_all = [&](bool first) -> int {
+        c->counters.launches += 3;
+        CU_TRY(mapk::launch_sel_proj_prep(s, first, st));
+        CU_TRY(mapk::launch_sel_gather(s, st));
+        MAP_TRY(gemm(c, pd, st));
+        CU_TRY(mapk::launch_sel_proj_done(s, st));
+        return MAP_OK;
+      };
+      pd.N = K0 <= 96 ? 96 : kProjMaxBasis;   // basis columns the R0 projection needs
+      MAP_TRY(project_all(true));
+      pd.N = kProjMaxBasis;
+      // one greedy round, then the images still selecting are projected again on their whole
+      // basis (when it has at most kReprojMax vectors): exact values for every candidate make
+      // the next active set the true top S
+      c->counters.launches += 4;
+      CU_TRY(mapk::launch_sel_choose(s, st));
+      MAP_TRY(gemm(c, d, st));
+      CU_TRY(mapk::launch_sel_greedy(s, st));
+      ++rounds;
+      ++c->counters.select_rounds;
+      MAP_TRY(project_all(false));
+      burst = 3;
     }
     for (;;) {
       for (int r = 0; r < burst; ++r) {

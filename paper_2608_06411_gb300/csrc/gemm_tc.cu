@@ -5,7 +5,7 @@
 // epilogue (section "Cross-Modal Attention Distillation"), and the Gram blocks
 // <v_i, v_j> that the diversity term of Eq. 4 needs.
 //
-// Structure (one CTA per SM, 6 warps; 8 for EPI_PROJECT):
+// Structure (one CTA per SM, 6 warps):
 //   warp 0      one thread issues TMA loads of 128x64 (A) and BNx64 (B) bf16 tiles, 128-byte
 //               swizzled, into a STAGES-deep shared-memory ring (mbarrier full/empty).
 //   warp 1      allocates TMEM (2 accumulators x BN fp32 columns); one thread issues
@@ -18,7 +18,8 @@
 //               thread), apply bias / GELU / RoPE, store (bf16, bf16 hi/lo pair, or fp32);
 //               release the accumulator so the
 //               MMA warp can start the tile after next while this one drains.
-//   warps 6-7   (EPI_PROJECT only) sum ||row||^2 of every A tile from shared memory.
+//   EPI_PROJECT: the MMA thread also accumulates A A^T (N = 128) of every stage into a second
+//               TMEM accumulator, whose diagonal is ||row||^2.
 // All waits are bounded (ptx.cuh); a timeout sets ST_TIMEOUT and every role drains and exits.
 #include <algorithm>
 #include <cstdio>
@@ -51,6 +52,7 @@ struct KArgs {
   int a_kwrap;
   int split3;
   const float* biasf;
+  const int* blist; const int* bcount;
 };
 
 __device__ __forceinline__ float gelu_erf(float x) {
@@ -71,13 +73,13 @@ struct Smem {
   static constexpr uint32_t B_BYTES = (CG2 ? BN / 2 : BN) * kBK * 2;   // CG2: this CTA's half
   static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr uint32_t TILES = STAGES * STAGE_BYTES;
-  static constexpr uint32_t BARS = (2 * STAGES + 5 + (PROJ ? 5 : 0)) * 8;
+  static constexpr uint32_t BARS = (2 * STAGES + 5 + (PROJ ? 1 : 0)) * 8;
   static constexpr uint32_t XPOSE = EPI == EPI_SM_STATS ? 4 * 32 * 33 * 4 : 0;   // per-warp 32x32 transposes
-  static constexpr uint32_t LSM = PROJ ? kProjMaxBasis * kProjMaxBasis * 4 : 0;  // L rows of the R0 basis
-  static constexpr uint32_t PEXTRA = PROJ ? (kProjMaxBasis + 2 * kBM) * 4 : 0;   // 1/r, ||v||^2 x 2 buffers
+  static constexpr uint32_t LSM = PROJ ? BN * BN * 4 : 0;       // L rows of the basis (pitch BN)
+  static constexpr uint32_t PEXTRA = PROJ ? BN * 4 : 0;          // 1/r of the basis
   static constexpr uint32_t TOTAL = 1024 + TILES + BARS + 16 + XPOSE + LSM + PEXTRA;
-  static constexpr uint32_t TMEM_COLS = 2 * BN;
-  static constexpr int THREADS = PROJ ? 256 : 192;   // + 2 warps summing ||v||^2 for EPI_PROJECT
+  static constexpr uint32_t TMEM_COLS = PROJ ? (2 * BN + 2 * kBM <= 256 ? 256u : 512u) : 2 * BN;   // + A A^T
+  static constexpr int THREADS = 192;
 };
 
 // Selection value, squared: p^2 * rho^(2 lambda) orders candidates like p * rho^lambda (both are
@@ -101,6 +103,7 @@ __device__ __forceinline__ TileCoord tile_coord(const KArgs& a, int t, int m_uni
   int per = m_units * n_tiles;
   c.b = t / per;
   int rem = t - c.b * per;
+  if (a.blist) c.b = __ldg(a.blist + c.b);
   const int mu = rem / n_tiles;
   c.n_blk = rem - mu * n_tiles;
   c.m_blk = PAIR ? 2 * mu + static_cast<int>(crank) : mu;
@@ -127,24 +130,20 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   uint64_t* tfull = empty + STAGES;
   uint64_t* tempty = tfull + 2;
   uint64_t* drain = tempty + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1 + (S::PROJ ? 5 : 0));
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1 + (S::PROJ ? 1 : 0));
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  uint64_t* nfull = drain + 1;                   // EPI_PROJECT: ||v||^2 of a tile ready / consumed
-  uint64_t* nempty = nfull + 2;
-  uint64_t* egsync = nempty + 2;                 // EPI_PROJECT: epilogue warps' group barrier
+  uint64_t* egsync = drain + 1;                  // EPI_PROJECT: epilogue warps' group barrier
   float* xpose = reinterpret_cast<float*>(smem + S::TILES + S::BARS + 16);
   float* Lsm = xpose + S::XPOSE / 4;
   float* rinv_sm = Lsm + S::LSM / 4;
-  float* sqbuf = rinv_sm + (S::PROJ ? kProjMaxBasis : 0);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
-    for (int s = 0; s < STAGES; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], S::PROJ ? 3 : 1); }
+    for (int s = 0; s < STAGES; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
     // tempty: one arrive per epilogue warp (of both CTAs with CG2, on the leader's barrier)
     for (int i = 0; i < 2; ++i) { mbar_init(&tfull[i], 1); mbar_init(&tempty[i], CG2 ? 8 : 4); }
     mbar_init(drain, 1);
     if constexpr (S::PROJ) {
-      for (int i = 0; i < 2; ++i) { mbar_init(&nfull[i], 2); mbar_init(&nempty[i], 128); }
       mbar_init(egsync, 128);
     }
     *abort_flag = 0;
@@ -163,7 +162,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   const int m_tiles = (a.M + kBM - 1) / kBM;
   const int m_units = PAIR ? (m_tiles + 1) / 2 : m_tiles;
   const int n_tiles = (a.N + BN - 1) / BN;
-  const int total = a.batch * m_units * n_tiles;
+  const int total = (a.blist ? min(a.batch, *a.bcount) : a.batch) * m_units * n_tiles;
   const int KB = a.K / kBK;
   // K block kb -> (A column, B column)
   auto kcols = [&](int kb, int& ac, int& bc) {
@@ -245,6 +244,13 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
 #pragma unroll
             for (int k = 0; k < kBK / 16; ++k)
               umma_bf16(d_tmem, desc_sw128(a0 + k * 32), desc_sw128(b0 + k * 32), IDESC, (kb | k) != 0);
+            if constexpr (S::PROJ) {   // A A^T: its diagonal is ||row||^2
+              const uint32_t n_tmem = tmem_base + 2 * BN + acc * kBM;
+#pragma unroll
+              for (int k = 0; k < kBK / 16; ++k)
+                umma_bf16(n_tmem, desc_sw128(a0 + k * 32), desc_sw128(a0 + k * 32), idesc_bf16(kBM, kBM),
+                          (kb | k) != 0);
+            }
             umma_commit(&empty[stage]);
           }
           issued = true;
@@ -281,9 +287,9 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           if (!mbar_wait(egsync, eg_phase, a.status, abort_flag)) { eg_ok = false; break; }
           eg_phase ^= 1;
           const ProjArgs& pj = a.proj;
-          const int nb0 = min(kProjMaxBasis, __ldg(pj.nbasis + c.b));
+          const int nb0 = min(BN, __ldg(pj.nbasis + c.b));
           const long long ibase = static_cast<long long>(c.b) * a.M;
-          const int KV = kProjMaxBasis / 4;
+          const int KV = BN / 4;
           for (int t4 = threadIdx.x - 64; t4 < nb0 * KV; t4 += 128) {
             const int i = t4 / KV, q = (t4 - i * KV) * 4;
             float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -295,7 +301,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
               v.z = q + 2 < i ? row[2] : 0.f;
               v.w = q + 3 < i ? row[3] : 0.f;
             }
-            *reinterpret_cast<float4*>(Lsm + i * kProjMaxBasis + q) = v;
+            *reinterpret_cast<float4*>(Lsm + i * BN + q) = v;
           }
           for (int i = threadIdx.x - 64; i < nb0; i += 128)
             rinv_sm[i] = 1.0f / __ldg(pj.rnorm + static_cast<long long>(c.b) * pj.Kcap + i);
@@ -304,7 +310,6 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           eg_phase ^= 1;
           staged_b = c.b;
         }
-        if (!mbar_wait(&nfull[acc], acc_phase, a.status, abort_flag)) break;
       }
       if (!mbar_wait(&tfull[acc], acc_phase, a.status, abort_flag)) break;
       tc_fence_after();
@@ -458,11 +463,17 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         // 32 basis vectors at a time: e_beta = (g_beta - sum_{q<beta} L[beta][q] e_q) / r_beta.
         // Each finished chunk of e replaces its g columns in TMEM, where later chunks read it.
         const ProjArgs& pj = a.proj;
-        const int nb0 = min(kProjMaxBasis, __ldg(pj.nbasis + c.b));
+        const int nb0 = min(BN, __ldg(pj.nbasis + c.b));
         const long long tok = static_cast<long long>(c.b) * a.M + row;
         const bool alive = row_ok && __ldg(pj.state + tok) == 0;
         float* erow = pj.Ec + tok * pj.KP;
-        const float sq = sqbuf[acc * kBM + r_in_tile];
+        float sq = 0.f;
+        {
+          uint32_t dg[32];
+          tmem_ld32(tmem_base + (static_cast<uint32_t>(lane_grp * 32) << 16) + 2 * BN + acc * kBM + lane_grp * 32, dg);
+#pragma unroll
+          for (int j = 0; j < 32; ++j) sq = j == lane ? __uint_as_float(dg[j]) : sq;
+        }
         float r2 = sq;
 #pragma unroll 1
         for (int b0 = 0; b0 < nb0; b0 += 32) {
@@ -483,7 +494,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
               for (int qq = 0; qq < 8; qq += 4) {
 #pragma unroll
                 for (int i = 0; i < 32; ++i) {
-                  const float4 l = *reinterpret_cast<const float4*>(Lsm + (b0 + i) * kProjMaxBasis + qc + qq);
+                  const float4 l = *reinterpret_cast<const float4*>(Lsm + (b0 + i) * BN + qc + qq);
                   accv[i] = fmaf(-l.x, __uint_as_float(ep[qq]), accv[i]);
                   accv[i] = fmaf(-l.y, __uint_as_float(ep[qq + 1]), accv[i]);
                   accv[i] = fmaf(-l.z, __uint_as_float(ep[qq + 2]), accv[i]);
@@ -499,7 +510,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             if (alive && b0 + i < b1) {
               v = accv[i];
 #pragma unroll
-              for (int q = 0; q < i; ++q) v = fmaf(-Lsm[(b0 + i) * kProjMaxBasis + b0 + q], accv[q], v);
+              for (int q = 0; q < i; ++q) v = fmaf(-Lsm[(b0 + i) * BN + b0 + q], accv[q], v);
               v *= rinv_sm[b0 + i];
               r2 = fmaf(-v, v, r2);
             }
@@ -526,7 +537,6 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           pj.U[tok] = proj_value(__ldg(pj.scores + tok), r2, sq, pj.lambda, pj.tau);
           pj.cstep[tok] = nb0;
         }
-        mbar_arrive(&nempty[acc]);
       } else if constexpr (EPI == EPI_F32) {
         float* out = reinterpret_cast<float*>(a.C) + crow + col0;
 #pragma unroll 1
@@ -590,58 +600,6 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       }
       acc ^= 1;
       if (acc == 0) acc_phase ^= 1;
-    }
-  }
-  if constexpr (S::PROJ) {
-    if (warp >= 6) {
-      // ---------------------------------------------------------------- ||v||^2 warps
-      // Warp 6 sums rows 0..63 of each A tile, warp 7 rows 64..127: 8 lanes per row, one
-      // 16-byte chunk each (the 128-byte swizzle only permutes chunks within a row).
-      const int rbase = (warp - 6) * 64;
-      uint32_t stage = 0, phase = 0, nb = 0, nb_phase = 0;
-      bool ok = true;
-      for (int t = unit0; t < total && ok; t += units_step) {
-        TileCoord c = tile_coord<PAIR>(a, t, m_units, n_tiles, BN, crank);
-        if (c.skip) continue;
-        float sacc[16];
-#pragma unroll
-        for (int i = 0; i < 16; ++i) sacc[i] = 0.f;
-        for (int kb = 0; kb < KB; ++kb) {
-          if (!mbar_wait(&full[stage], phase, a.status, abort_flag)) { ok = false; break; }
-          const uint8_t* tileA = sA + stage * S::A_BYTES;
-#pragma unroll
-          for (int i = 0; i < 16; ++i) {
-            const int r = rbase + 4 * i + (lane >> 3);
-            const uint4 u = *reinterpret_cast<const uint4*>(tileA + r * 128 + (lane & 7) * 16);
-            const uint32_t w[4] = {u.x, u.y, u.z, u.w};
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-              const float lo = __uint_as_float(w[j] << 16), hi = __uint_as_float(w[j] & 0xFFFF0000u);
-              sacc[i] = fmaf(lo, lo, sacc[i]);
-              sacc[i] = fmaf(hi, hi, sacc[i]);
-            }
-          }
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&empty[stage]);
-          if (++stage == STAGES) { stage = 0; phase ^= 1; }
-        }
-        if (!ok) break;
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          sacc[i] += __shfl_xor_sync(0xffffffffu, sacc[i], 1);
-          sacc[i] += __shfl_xor_sync(0xffffffffu, sacc[i], 2);
-          sacc[i] += __shfl_xor_sync(0xffffffffu, sacc[i], 4);
-        }
-        if (!mbar_wait(&nempty[nb], nb_phase ^ 1, a.status, abort_flag)) break;
-        if ((lane & 7) == 0) {
-#pragma unroll
-          for (int i = 0; i < 16; ++i) sqbuf[nb * kBM + rbase + 4 * i + (lane >> 3)] = sacc[i];
-        }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&nfull[nb]);
-        nb ^= 1;
-        if (nb == 0) nb_phase ^= 1;
-      }
     }
   }
   if constexpr (PAIR) cluster_sync();             // no commit or remote arrive still in flight
@@ -751,6 +709,8 @@ cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t st) {
   ka.stats = d.stats; ka.stat_ld = d.stat_ld; ka.col_count = d.col_count;
   ka.b_base = d.b_base; ka.proj = d.proj;
   ka.a_kwrap = d.a_kwrap; ka.biasf = d.biasf; ka.split3 = d.split3;
+  ka.blist = d.blist; ka.bcount = d.blist ? d.bcount : nullptr;
+  if (d.blist && !d.bcount) return cudaErrorInvalidValue;
   switch (d.epi) {
     case EPI_GELU_BF16:
       if (d.N % 256 == 0) return run<256, 4, EPI_GELU_BF16>(d, ka, num_sms, st);
@@ -783,7 +743,8 @@ cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t st) {
       return run<256, 4, EPI_SM_MEAN>(d, ka, num_sms, st);
     case EPI_PROJECT:
       if (d.N > kProjMaxBasis || d.batch < 1) return cudaErrorInvalidValue;
-      return run<128, 4, EPI_PROJECT>(d, ka, num_sms, st);
+      if (d.N <= 96) return run<96, 6, EPI_PROJECT>(d, ka, num_sms, st);
+      return run<128, 5, EPI_PROJECT>(d, ka, num_sms, st);
     case EPI_F32:   // Gram blocks: one 256 x 256 pair tile per image and 256 columns
       return run<256, 6, EPI_F32, true>(d, ka, num_sms, st);
     default:

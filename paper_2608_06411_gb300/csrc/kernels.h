@@ -70,6 +70,9 @@ struct GemmDesc {
   // is read twice back to back (the second time from L2)
   int split3 = 0;
   const float* biasf = nullptr;         // EPI_ROPE_SPLIT3: fp32 bias [N] added before RoPE
+  // Batch entries to process (device): blist[0 .. *bcount) instead of 0 .. batch-1, so that a
+  // launch over a few active images spreads their tiles over all SMs (grid sized for batch)
+  const int* blist = nullptr; const int* bcount = nullptr;
 };
 
 // Returns cudaSuccess, or an error for an unsupported shape (cudaErrorInvalidValue).

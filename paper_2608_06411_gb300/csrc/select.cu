@@ -195,6 +195,7 @@ __global__ void __launch_bounds__(1024) sel_choose_kernel(SelState s) {
     if (threadIdx.x == 0) s.nlimit[b] = 0;
     return;
   }
+  if (s.blist && threadIdx.x == 0) s.blist[atomicAdd(s.bcount, 1)] = b;
   const int np = s.npicks[b], nb = s.nbasis[b];
   uint64_t theta = 0;
   int mode;
@@ -705,20 +706,29 @@ __global__ void __launch_bounds__(256, 1) sel_greedy_kernel(SelState s) {
 }
 
 // ------------------------------------------------------------------ projection set-up
-// After the R0 rounds: gather every R0 basis row (no active tokens) for the projection.
-__global__ void sel_proj_prep_kernel(SelState s) {
+// Gathers every basis row of the images to project (no active tokens) for the projection.
+__global__ void sel_proj_prep_kernel(SelState s, int first) {
   const int b = blockIdx.x;
+  const int nb = s.nbasis[b];
+  const bool go = first || (!s.done[b] && nb > s.gbase[b] && nb <= kReprojMax);
+  if (!go) {
+    if (threadIdx.x == 0) s.proj_lim[b] = 0;
+    return;
+  }
   for (int i = threadIdx.x; i < s.S; i += blockDim.x) s.aslot[static_cast<long long>(b) * s.S + i] = -1;
   if (threadIdx.x == 0) {
-    s.gb_lo[b] = s.nb_gathered[b];
-    s.gb_hi[b] = s.nbasis[b];
-    s.nb_gathered[b] = s.nbasis[b];
+    if (s.blist) s.blist[atomicAdd(s.bcount, 1)] = b;
+    s.proj_lim[b] = kReprojMax;
+    s.gbase[b] = 0;                                  // rows S + beta for the whole basis
+    s.gb_lo[b] = 0;
+    s.gb_hi[b] = nb;
+    s.nb_gathered[b] = nb;
   }
 }
 
 __global__ void sel_proj_done_kernel(SelState s) {
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
-  if (b < s.B) {
+  if (b < s.B && s.proj_lim[b] > 0) {
     s.gbase[b] = s.nbasis[b];
     s.nb_gathered[b] = s.nbasis[b];
   }
@@ -780,6 +790,10 @@ cudaError_t launch_sel_init(const SelState& s, cudaStream_t st) {
 }
 
 cudaError_t launch_sel_choose(const SelState& s, cudaStream_t st) {
+  if (s.bcount) {
+    const cudaError_t z = cudaMemsetAsync(s.bcount, 0, sizeof(int32_t), st);
+    if (z != cudaSuccess) return z;
+  }
   const size_t sm = sel_choose_smem(s.N);
   cudaError_t e = cudaFuncSetAttribute(sel_choose_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(sm));
   if (e != cudaSuccess) return e;
@@ -829,8 +843,12 @@ cudaError_t launch_sel_copy_r0(const int32_t* r0, int B, int K, int32_t* picks, 
   return cudaGetLastError();
 }
 
-cudaError_t launch_sel_proj_prep(const SelState& s, cudaStream_t st) {
-  sel_proj_prep_kernel<<<s.B, 256, 0, st>>>(s);
+cudaError_t launch_sel_proj_prep(const SelState& s, bool first, cudaStream_t st) {
+  if (s.bcount) {
+    const cudaError_t z = cudaMemsetAsync(s.bcount, 0, sizeof(int32_t), st);
+    if (z != cudaSuccess) return z;
+  }
+  sel_proj_prep_kernel<<<s.B, 256, 0, st>>>(s, first ? 1 : 0);
   return cudaGetLastError();
 }
 

@@ -36,6 +36,8 @@ struct SelState {
   void* Vg;                       // [B, R, D] bf16 gathered rows
   float* G;                       // [B, S, R] Gram block
   int32_t* done_count;            // images finished
+  int32_t* proj_lim;              // [B] basis columns the projection GEMM computes (0: image skipped)
+  int32_t* blist; int32_t* bcount;  // images the next Gram / projection GEMM processes (optional)
   int* status;
 };
 
@@ -51,10 +53,14 @@ cudaError_t launch_sel_chol(const SelState& s, cudaStream_t st);
 cudaError_t launch_sel_finalize(const int32_t* picks, int B, int K, int32_t* keep, int32_t* order, cudaStream_t st);
 cudaError_t launch_sel_copy_r0(const int32_t* r0, int B, int K, int32_t* picks, cudaStream_t st);
 cudaError_t launch_sel_identity(int B, int N, int32_t* keep, int32_t* order, cudaStream_t st);
-// Queues the R0 basis rows for gathering into Vg (rows S + beta) ahead of the projection.
-cudaError_t launch_sel_proj_prep(const SelState& s, cudaStream_t st);
+// Queues basis rows for gathering into Vg (rows S + beta) ahead of a projection of every
+// candidate on the whole basis: first = the R0 basis of every image; otherwise (after a
+// greedy round) the basis of each image still selecting whose basis has grown and has at
+// most kReprojMax vectors, other images are skipped (proj_lim 0).
+constexpr int kReprojMax = 128;
+cudaError_t launch_sel_proj_prep(const SelState& s, bool first, cudaStream_t st);
 cudaError_t launch_sel_gather(const SelState& s, cudaStream_t st);
-// After the projection: later Gram blocks start at the first basis vector past R0.
+// After a projection: the projected images' later Gram blocks start past their basis.
 cudaError_t launch_sel_proj_done(const SelState& s, cudaStream_t st);
 
 }  // namespace mapk
