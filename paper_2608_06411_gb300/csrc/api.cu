@@ -430,7 +430,11 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, 
       // R0: gather its rows, G[R0, R0] on the tensor cores, then its Cholesky factor.
       c->counters.launches += 3;
       CU_TRY(mapk::launch_sel_choose(s, st));
-      MAP_TRY(gemm(c, d, st));
+      {
+        GemmDesc d0 = d;              // only the K0 x K0 corner of the block
+        d0.M = K0; d0.N = K0;
+        MAP_TRY(gemm(c, d0, st));
+      }
       CU_TRY(mapk::launch_sel_chol(s, st));
       ++rounds;
       ++c->counters.select_rounds;

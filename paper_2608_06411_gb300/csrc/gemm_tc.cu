@@ -746,6 +746,7 @@ cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t st) {
       if (d.N <= 96) return run<96, 6, EPI_PROJECT>(d, ka, num_sms, st);
       return run<128, 5, EPI_PROJECT>(d, ka, num_sms, st);
     case EPI_F32:   // Gram blocks: one 256 x 256 pair tile per image and 256 columns
+      if (d.M <= kBM && d.N <= 128) return run<128, 6, EPI_F32>(d, ka, num_sms, st);   // G[R0, R0]
       return run<256, 6, EPI_F32, true>(d, ka, num_sms, st);
     default:
       return cudaErrorInvalidValue;
