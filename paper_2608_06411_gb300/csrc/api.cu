@@ -45,10 +45,10 @@ struct map_ctx {
   // map_prune staging
   DevBuf pvis, ptext, pout, pkeep, pscores;
   int* status = nullptr;            // device status word
-  int* h_status = nullptr;          // pinned
-  int32_t* h_done = nullptr;        // pinned
-  void* h_stage = nullptr; size_t h_stage_cap = 0;   // pinned host staging (offsets, positions)
-  cudaEvent_t stage_ev = nullptr; bool stage_pending = false;
+  int* h_status = nullptr;          // pinned, mapped
+  int32_t* h_done = nullptr;        // pinned, mapped
+  int* h_status_dev = nullptr; int32_t* h_done_dev = nullptr;   // their device aliases
+  cudaStream_t s_in = nullptr, s_out = nullptr;   // map_prune copy streams (host buffers)
   bool timing = false;
   std::vector<TimedPair> pairs;
   std::vector<cudaEvent_t> free_events;
@@ -163,21 +163,6 @@ int ensure_rope(map_ctx* c, int rows_needed) {
   return MAP_OK;
 }
 
-int stage_host(map_ctx* c, size_t bytes, void** out) {
-  if (c->stage_pending) {
-    cudaEventSynchronize(c->stage_ev);
-    c->stage_pending = false;
-  }
-  if (bytes > c->h_stage_cap) {
-    if (c->h_stage) cudaFreeHost(c->h_stage);
-    c->h_stage = nullptr;
-    c->h_stage_cap = 0;
-    if (cudaMallocHost(&c->h_stage, bytes + 4096) != cudaSuccess) { cudaGetLastError(); return MAP_ENOMEM; }
-    c->h_stage_cap = bytes + 4096;
-  }
-  *out = c->h_stage;
-  return MAP_OK;
-}
 
 int gemm(map_ctx* c, const GemmDesc& d, cudaStream_t st) {
   ++c->counters.launches;
@@ -251,26 +236,19 @@ int score_impl(map_ctx* c, const void* text, const void* vis, const int32_t* len
   const map_config& g = c->cfg;
   CU_TRY(cudaSetDevice(c->device));
   MAP_TRY(ensure_rope(c, g.rope_on ? N + max_m + 1 : 1));
-  // per-image query offsets, lengths and question-token positions N + m
+  // per-image query offsets, lengths and question-token positions N + m, written on the device
   const size_t off_bytes = static_cast<size_t>(B + 1) * 4, len_bytes = static_cast<size_t>(B) * 4;
   const size_t pos_bytes = static_cast<size_t>(total_m) * 4;
-  void* hs = nullptr;
-  MAP_TRY(stage_host(c, off_bytes + len_bytes + pos_bytes, &hs));
-  int32_t* hoff = static_cast<int32_t*>(hs);
-  int32_t* hlen = hoff + (B + 1);
-  int32_t* hpos = hlen + B;
-  hoff[0] = 0;
-  for (int b = 0; b < B; ++b) {
-    hoff[b + 1] = hoff[b] + lens[b];
-    hlen[b] = lens[b];
-    for (int m = 0; m < lens[b]; ++m) hpos[hoff[b] + m] = N + m;
-  }
   MAP_TRY(ensure(c->qoff, off_bytes + len_bytes));
   MAP_TRY(ensure(c->post, pos_bytes));
-  CU_TRY(cudaMemcpyAsync(c->qoff.p, hoff, off_bytes + len_bytes, cudaMemcpyHostToDevice, st));
-  CU_TRY(cudaMemcpyAsync(c->post.p, hpos, pos_bytes, cudaMemcpyHostToDevice, st));
-  CU_TRY(cudaEventRecord(c->stage_ev, st));
-  c->stage_pending = true;
+  {
+    std::vector<long long> offs(B);
+    long long acc = 0;
+    for (int b = 0; b < B; ++b) { offs[b] = acc; acc += lens[b]; }
+    int32_t* qo = static_cast<int32_t*>(c->qoff.p);
+    CU_TRY(mapk::launch_query_meta(lens, offs.data(), B, N, qo, qo + (B + 1), static_cast<int32_t*>(c->post.p), st));
+    c->counters.launches += (B + 1023) / 1024;
+  }
   const int* d_off = static_cast<const int*>(c->qoff.p);
   const int* d_len = d_off + (B + 1);
 
@@ -482,9 +460,15 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, 
       }
       rounds += burst;
       c->counters.select_rounds += burst;
-      CU_TRY(cudaMemcpyAsync(c->h_done, s.done_count, 4, cudaMemcpyDeviceToHost, st));
+      // through host-mapped words (no copy engine: bulk copies on other streams do not delay it)
+      CU_TRY(mapk::launch_flags_to_host(s.done_count, c->status, c->h_done_dev, c->h_status_dev, st));
+      ++c->counters.launches;
       CU_TRY(cudaStreamSynchronize(st));
       if (*c->h_done >= B) break;
+      if (*c->h_status) {               // a kernel gave up (bounded wait) or saw a bad index: stop here
+        c->deferred = dev_status_error(*c->h_status);
+        return c->deferred;
+      }
       if (rounds > cap) {
         c->deferred = MAP_EINTERNAL;
         return MAP_EINTERNAL;
@@ -590,9 +574,13 @@ int map_init(const map_config* cfg, const map_weights* w, map_ctx** out) {
     }
     if (cudaMalloc(&c->status, sizeof(int)) != cudaSuccess) { rc = MAP_ENOMEM; break; }
     if (cudaMemset(c->status, 0, sizeof(int)) != cudaSuccess) { rc = MAP_ECUDA; break; }
-    if (cudaMallocHost(&c->h_status, sizeof(int)) != cudaSuccess) { rc = MAP_ENOMEM; break; }
-    if (cudaMallocHost(&c->h_done, sizeof(int32_t)) != cudaSuccess) { rc = MAP_ENOMEM; break; }
-    if (cudaEventCreateWithFlags(&c->stage_ev, cudaEventDisableTiming) != cudaSuccess) { rc = MAP_ECUDA; break; }
+    if (cudaHostAlloc(&c->h_status, sizeof(int), cudaHostAllocMapped) != cudaSuccess) { rc = MAP_ENOMEM; break; }
+    if (cudaHostAlloc(&c->h_done, sizeof(int32_t), cudaHostAllocMapped) != cudaSuccess) { rc = MAP_ENOMEM; break; }
+    if (cudaHostGetDevicePointer(reinterpret_cast<void**>(&c->h_status_dev), c->h_status, 0) != cudaSuccess ||
+        cudaHostGetDevicePointer(reinterpret_cast<void**>(&c->h_done_dev), c->h_done, 0) != cudaSuccess) {
+      rc = MAP_ECUDA;
+      break;
+    }
   } while (false);
   if (rc != MAP_OK) {
     cudaGetLastError();
@@ -643,23 +631,95 @@ int map_prune(map_ctx* ctx, const void* text_feats, const void* vis_feats, const
   const bool dkeep = is_device_ptr(keep_idx), dsc = scores ? is_device_ptr(scores) : true;
   const void* v = vis_feats;
   const void* t = text_feats;
-  if (!dv) { MAP_TRY(ensure(c->pvis, vis_bytes)); CU_TRY(cudaMemcpyAsync(c->pvis.p, vis_feats, vis_bytes, cudaMemcpyHostToDevice, st)); v = c->pvis.p; }
-  if (!dt) { MAP_TRY(ensure(c->ptext, text_bytes)); CU_TRY(cudaMemcpyAsync(c->ptext.p, text_feats, text_bytes, cudaMemcpyHostToDevice, st)); t = c->ptext.p; }
+  if (!dv) { MAP_TRY(ensure(c->pvis, vis_bytes)); v = c->pvis.p; }
+  if (!dt) { MAP_TRY(ensure(c->ptext, text_bytes)); t = c->ptext.p; }
   void* o = out;
   int32_t* kp = keep_idx;
   float* sp = scores;
   if (!dout) { MAP_TRY(ensure(c->pout, out_bytes)); o = c->pout.p; }
   if (!dkeep) { MAP_TRY(ensure(c->pkeep, keep_bytes)); kp = static_cast<int32_t*>(c->pkeep.p); }
   if (!dsc || !scores) { MAP_TRY(ensure(c->pscores, sc_bytes)); sp = static_cast<float*>(c->pscores.p); }
-  MAP_TRY(score_impl(c, t, v, lens, B, N, sp, nullptr, nullptr, st));
-  MAP_TRY(select_impl(c, sp, v, B, N, k, kp, nullptr, st));
-  MAP_TRY(gather_impl(c, v, kp, B, N, k, o, st));
-  bool sync = !dv || !dt;
-  if (!dout) { CU_TRY(cudaMemcpyAsync(out, o, out_bytes, cudaMemcpyDeviceToHost, st)); sync = true; }
-  if (!dkeep) { CU_TRY(cudaMemcpyAsync(keep_idx, kp, keep_bytes, cudaMemcpyDeviceToHost, st)); sync = true; }
-  if (scores && !dsc) { CU_TRY(cudaMemcpyAsync(scores, sp, sc_bytes, cudaMemcpyDeviceToHost, st)); sync = true; }
-  if (sync) CU_TRY(cudaStreamSynchronize(st));
-  return MAP_OK;
+  const bool host_io = !dv || !dt || !dout || !dkeep || (scores && !dsc);
+
+  // With host buffers the batch runs as a pipeline of image chunks: chunk i+1 is copied in
+  // (stream s_in) while chunk i is scored, selected and gathered (the caller's stream) and
+  // chunk i-1 is copied out (stream s_out).  Results equal the one-shot path.
+  const int nchunk = host_io ? std::min(B, 4) : 1;
+  if (nchunk > 1) {
+    if (!c->s_in) CU_TRY(cudaStreamCreateWithFlags(&c->s_in, cudaStreamNonBlocking));
+    if (!c->s_out) CU_TRY(cudaStreamCreateWithFlags(&c->s_out, cudaStreamNonBlocking));
+  }
+  std::vector<long long> toff(B + 1, 0);
+  for (int b = 0; b < B; ++b) toff[b + 1] = toff[b] + lens[b];
+  cudaStream_t si = nchunk > 1 ? c->s_in : st, so = nchunk > 1 ? c->s_out : st;
+  std::vector<cudaEvent_t> evs;
+  auto ev = [&]() { cudaEvent_t e = take_event(c); evs.push_back(e); return e; };
+  auto finish = [&](int rc) {
+    for (cudaEvent_t e : evs) c->free_events.push_back(e);
+    return rc;
+  };
+  if (nchunk > 1) {                         // buffers reused from earlier work on the caller's stream
+    cudaEvent_t e0 = ev();
+    if (cudaEventRecord(e0, st) != cudaSuccess || cudaStreamWaitEvent(si, e0, 0) != cudaSuccess ||
+        cudaStreamWaitEvent(so, e0, 0) != cudaSuccess)
+      return finish(MAP_ECUDA);
+  }
+  std::vector<cudaEvent_t> ev_in(nchunk);
+  auto chunk = [&](int i, int& b0, int& b1) { b0 = static_cast<int>(static_cast<long long>(B) * i / nchunk);
+                                               b1 = static_cast<int>(static_cast<long long>(B) * (i + 1) / nchunk); };
+  for (int i = 0; i < nchunk; ++i) {
+    int b0, b1;
+    chunk(i, b0, b1);
+    const size_t vo = static_cast<size_t>(b0) * N * D * 2, vn = static_cast<size_t>(b1 - b0) * N * D * 2;
+    const size_t to = static_cast<size_t>(toff[b0]) * D * 2, tn = static_cast<size_t>(toff[b1] - toff[b0]) * D * 2;
+    if (!dv && cudaMemcpyAsync(static_cast<char*>(c->pvis.p) + vo, static_cast<const char*>(vis_feats) + vo, vn,
+                               cudaMemcpyHostToDevice, si) != cudaSuccess)
+      return finish(MAP_ECUDA);
+    if (!dt && cudaMemcpyAsync(static_cast<char*>(c->ptext.p) + to, static_cast<const char*>(text_feats) + to, tn,
+                               cudaMemcpyHostToDevice, si) != cudaSuccess)
+      return finish(MAP_ECUDA);
+    ev_in[i] = ev();
+    if (cudaEventRecord(ev_in[i], si) != cudaSuccess) return finish(MAP_ECUDA);
+  }
+  for (int i = 0; i < nchunk; ++i) {
+    int b0, b1;
+    chunk(i, b0, b1);
+    const int Bc = b1 - b0;
+    if (cudaStreamWaitEvent(st, ev_in[i], 0) != cudaSuccess) return finish(MAP_ECUDA);
+    const void* vc = static_cast<const char*>(v) + static_cast<size_t>(b0) * N * D * 2;
+    const void* tc = static_cast<const char*>(t) + static_cast<size_t>(toff[b0]) * D * 2;
+    float* spc = sp + static_cast<size_t>(b0) * N;
+    int32_t* kpc = kp + static_cast<size_t>(b0) * k;
+    void* oc = static_cast<char*>(o) + static_cast<size_t>(b0) * k * D * 2;
+    int rc = score_impl(c, tc, vc, lens + b0, Bc, N, spc, nullptr, nullptr, st);
+    if (rc == MAP_OK) rc = select_impl(c, spc, vc, Bc, N, k, kpc, nullptr, st);
+    if (rc == MAP_OK) rc = gather_impl(c, vc, kpc, Bc, N, k, oc, st);
+    if (rc != MAP_OK) return finish(rc);
+    if (host_io) {
+      cudaEvent_t ed = ev();
+      if (cudaEventRecord(ed, st) != cudaSuccess || cudaStreamWaitEvent(so, ed, 0) != cudaSuccess) return finish(MAP_ECUDA);
+      const size_t oo = static_cast<size_t>(b0) * k * D * 2, on = static_cast<size_t>(Bc) * k * D * 2;
+      const size_t ko = static_cast<size_t>(b0) * k * 4, kn = static_cast<size_t>(Bc) * k * 4;
+      const size_t so_ = static_cast<size_t>(b0) * N * 4, sn = static_cast<size_t>(Bc) * N * 4;
+      if (!dout && on && cudaMemcpyAsync(static_cast<char*>(out) + oo, static_cast<char*>(o) + oo, on,
+                                         cudaMemcpyDeviceToHost, so) != cudaSuccess)
+        return finish(MAP_ECUDA);
+      if (!dkeep && kn && cudaMemcpyAsync(reinterpret_cast<char*>(keep_idx) + ko, reinterpret_cast<char*>(kp) + ko, kn,
+                                          cudaMemcpyDeviceToHost, so) != cudaSuccess)
+        return finish(MAP_ECUDA);
+      if (scores && !dsc && cudaMemcpyAsync(reinterpret_cast<char*>(scores) + so_, reinterpret_cast<char*>(sp) + so_,
+                                            sn, cudaMemcpyDeviceToHost, so) != cudaSuccess)
+        return finish(MAP_ECUDA);
+    }
+  }
+  if (host_io) {
+    if (nchunk > 1) {
+      cudaEvent_t ee = ev();
+      if (cudaEventRecord(ee, so) != cudaSuccess || cudaStreamWaitEvent(st, ee, 0) != cudaSuccess) return finish(MAP_ECUDA);
+    }
+    if (cudaStreamSynchronize(st) != cudaSuccess) return finish(MAP_ECUDA);
+  }
+  return finish(MAP_OK);
 }
 
 int map_status(map_ctx* ctx, void* stream) {
@@ -694,8 +754,8 @@ void map_destroy(map_ctx* ctx) {
   if (ctx->status) cudaFree(ctx->status);
   if (ctx->h_status) cudaFreeHost(ctx->h_status);
   if (ctx->h_done) cudaFreeHost(ctx->h_done);
-  if (ctx->h_stage) cudaFreeHost(ctx->h_stage);
-  if (ctx->stage_ev) cudaEventDestroy(ctx->stage_ev);
+  if (ctx->s_in) cudaStreamDestroy(ctx->s_in);
+  if (ctx->s_out) cudaStreamDestroy(ctx->s_out);
   for (auto& pr : ctx->pairs) { cudaEventDestroy(pr.a); cudaEventDestroy(pr.b); }
   for (auto e : ctx->free_events) cudaEventDestroy(e);
   delete ctx;

@@ -85,6 +85,15 @@ cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t st);
 cudaError_t launch_fold_weights(const void* Wp, const void* W2, const void* b2, int dp, int Dh, void* out,
                                 float* bias_out, cudaStream_t st);
 
+// Per-image question metadata written on the device from values passed as kernel parameters
+// (no host-to-device copy, so nothing queues behind bulk input copies on the copy engines):
+// off[b] = first query row of image b (off[B] = total), len[b], pos[row] = N + m for the
+// m-th question token of its image.  lens has B entries; offs are their exclusive prefix sums.
+cudaError_t launch_query_meta(const int32_t* lens, const long long* offs, int B, int N, int32_t* off, int32_t* len,
+                              int32_t* pos, cudaStream_t st);
+// Copies two device ints into host-mapped memory (device aliases of pinned host words).
+cudaError_t launch_flags_to_host(const int32_t* a, const int* b, int32_t* a_host_dev, int* b_host_dev, cudaStream_t st);
+
 // Squared row norms of bf16 rows: out[r] = sum_d x[r, d]^2 (fp32).
 cudaError_t launch_row_sqnorm(const void* x, long long rows, int D, float* out, cudaStream_t st);
 

@@ -19,6 +19,7 @@
 
 #include "../../include/map_gb300.h"
 #include "kernels.h"
+#include "ptx.cuh"
 #include "select.h"
 
 namespace mapk {
@@ -176,6 +177,9 @@ extern "C" int map_select_noalloc(map_ctx* ctx, const float* scores, const void*
       if ((rc = rc_of(cudaMemcpyAsync(v.h_done, s.done_count, 4, cudaMemcpyDeviceToHost, st))) != MAP_OK) return rc;
       if ((rc = rc_of(cudaStreamSynchronize(st))) != MAP_OK) return rc;
       if (*v.h_done >= B) break;
+      int dev_status = 0;             // a kernel that gave up stops the loop at once
+      if ((rc = rc_of(cudaMemcpy(&dev_status, v.status, sizeof(int), cudaMemcpyDeviceToHost))) != MAP_OK) return rc;
+      if (dev_status) return (dev_status & mapk::ST_TIMEOUT) ? MAP_ETIMEOUT : MAP_EINTERNAL;
       if (rounds > cap) return MAP_EINTERNAL;
       burst = 2;
     }

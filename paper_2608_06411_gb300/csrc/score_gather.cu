@@ -100,7 +100,56 @@ __global__ void fold_weights_kernel(const __nv_bfloat16* __restrict__ Wp, const 
   }
 }
 
+constexpr int kMetaImages = 1024;
+struct MetaChunk {
+  int b0, count, N, last;
+  int32_t lens[kMetaImages];
+  int32_t offs[kMetaImages];
+};
+
+// One CTA per image of the chunk.
+__global__ void query_meta_kernel(const __grid_constant__ MetaChunk m, int32_t* __restrict__ off,
+                                  int32_t* __restrict__ len, int32_t* __restrict__ pos) {
+  const int i = blockIdx.x, b = m.b0 + i;
+  const int o = m.offs[i], l = m.lens[i];
+  if (threadIdx.x == 0) {
+    off[b] = o;
+    len[b] = l;
+    if (m.last && i == m.count - 1) off[b + 1] = o + l;
+  }
+  for (int t = threadIdx.x; t < l; t += blockDim.x) pos[o + t] = m.N + t;
+}
+
+__global__ void flags_to_host_kernel(const int32_t* a, const int* b, volatile int32_t* ah, volatile int* bh) {
+  *ah = *a;
+  *bh = *b;
+}
+
 }  // namespace
+
+cudaError_t launch_query_meta(const int32_t* lens, const long long* offs, int B, int N, int32_t* off, int32_t* len,
+                              int32_t* pos, cudaStream_t st) {
+  for (int b0 = 0; b0 < B; b0 += kMetaImages) {
+    MetaChunk m;
+    m.b0 = b0;
+    m.count = B - b0 < kMetaImages ? B - b0 : kMetaImages;
+    m.N = N;
+    m.last = b0 + m.count == B;
+    for (int i = 0; i < m.count; ++i) {
+      m.lens[i] = lens[b0 + i];
+      m.offs[i] = static_cast<int32_t>(offs[b0 + i]);
+    }
+    query_meta_kernel<<<m.count, 128, 0, st>>>(m, off, len, pos);
+    const cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+cudaError_t launch_flags_to_host(const int32_t* a, const int* b, int32_t* a_host_dev, int* b_host_dev, cudaStream_t st) {
+  flags_to_host_kernel<<<1, 1, 0, st>>>(a, b, a_host_dev, b_host_dev);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_fold_weights(const void* Wp, const void* W2, const void* b2, int dp, int Dh, void* out,
                                 float* bias_out, cudaStream_t st) {

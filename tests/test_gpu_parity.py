@@ -227,8 +227,8 @@ def test_prune_host_buffers_equal_device_path():
     dims = W.PredictorDims(D=512, Dh=256, dp=64)
     ctx, w = make_ctx(dims)
     wl = W.WORKLOADS["c1"]
-    B, N, K = 2, 400, 30
-    lens = np.array([12, 40], np.int32)
+    B, N, K = 5, 400, 30            # host buffers run as a pipeline of 4 image chunks (1, 1, 1, 2)
+    lens = np.array([12, 40, 7, 33, 20], np.int32)
     vis = np.stack([W.make_image(wl, b, N=N, D=dims.D) for b in range(B)])
     text = np.concatenate([W.make_text(wl, b, int(lens[b]), D=dims.D) for b in range(B)])
     out_h = np.zeros((B, K, dims.D), np.uint16)
