@@ -449,7 +449,7 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, 
       ++rounds;
       ++c->counters.select_rounds;
       MAP_TRY(project_all(false));
-      burst = 3;
+      burst = 2;
     }
     for (;;) {
       for (int r = 0; r < burst; ++r) {

@@ -59,7 +59,9 @@ __device__ __forceinline__ float sel_value(float p, float r2, float sq, float la
 // k-th largest of n distinct 64-bit keys in shared memory (1 <= k <= n): MSB-first radix
 // select, 8 bits per pass.  Lanes of a warp that hit the same bin add their count once
 // (__match_any_sync), so bins shared by most keys (a common exponent) are not a
-// serialisation point; one warp finds the bin with a shuffle scan.
+// serialisation point; one warp finds the bin with a shuffle scan.  As soon as the bin that
+// holds the k-th key holds no other key, that key is the answer (usually after 2-3 passes).
+// hist needs 256 entries, bc 4.
 __device__ uint64_t block_kth_largest(const uint64_t* keys, int n, int k, uint32_t* hist, uint32_t* bc) {
   uint64_t prefix = 0, mask = 0;
   int want = k;
@@ -95,6 +97,7 @@ __device__ uint64_t block_kth_largest(const uint64_t* keys, int n, int k, uint32
           if (cum + c[j] >= static_cast<uint32_t>(want)) {
             bc[0] = 255 - 8 * lane - j;
             bc[1] = want - cum;
+            bc[2] = c[j];                           // keys in that bin
             break;
           }
           cum += c[j];
@@ -105,6 +108,15 @@ __device__ uint64_t block_kth_largest(const uint64_t* keys, int n, int k, uint32
     prefix |= static_cast<uint64_t>(bc[0]) << shift;
     mask |= 255ull << shift;
     want = static_cast<int>(bc[1]);
+    if (bc[2] == 1u && shift > 0) {                 // uniform: the k-th key is the bin's only key
+      __shared__ uint64_t found;
+      for (int i = threadIdx.x; i < n; i += blockDim.x)
+        if ((keys[i] & mask) == prefix) found = keys[i];
+      __syncthreads();
+      const uint64_t r = found;
+      __syncthreads();
+      return r;
+    }
     __syncthreads();
   }
   return prefix;
@@ -153,7 +165,7 @@ __global__ void __launch_bounds__(1024) sel_init_kernel(SelState s) {
   extern __shared__ uint64_t sh64[];
   const int b = blockIdx.x;
   const long long base = static_cast<long long>(b) * s.N;
-  __shared__ uint32_t hist[256], bc[2];
+  __shared__ uint32_t hist[256], bc[4];
   __shared__ int cnt;
   for (int i = threadIdx.x; i < s.N; i += blockDim.x) {
     const float p = s.scores[base + i], sq = s.sqn ? s.sqn[base + i] : 0.f;
@@ -205,7 +217,7 @@ __global__ void __launch_bounds__(1024) sel_choose_kernel(SelState s) {
       aslot[i] = i < na ? s.r0[static_cast<long long>(b) * s.K + np + i] : -1;
     mode = 1;
   } else {
-    __shared__ uint32_t hist[256], bc[2];
+    __shared__ uint32_t hist[256], bc[4];
     __shared__ int cnt, n_alive;
     if (threadIdx.x == 0) { cnt = 0; n_alive = 0; }
     __syncthreads();
@@ -432,6 +444,7 @@ __global__ void __launch_bounds__(kCholThreads, 1) sel_chol_kernel(SelState s) {
     if (!ext) continue;                                   // uniform
     if (u > t && u < K0) {
       const float* lt = Ls + t * PL;
+      const float rinv = 1.0f / sqrtf(d), gut = Gs[u * ldg + t];   // independent of the dot product
       float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
 #pragma unroll 4
       for (int q = 0; q < nb; q += 4) {                   // rows are zero past nb
@@ -442,7 +455,7 @@ __global__ void __launch_bounds__(kCholThreads, 1) sel_chol_kernel(SelState s) {
         a2 = fmaf(x.z, y.z, a2);
         a3 = fmaf(x.w, y.w, a3);
       }
-      const float e = (Gs[u * ldg + t] - ((a0 + a1) + (a2 + a3))) * (1.0f / sqrtf(d));
+      const float e = (gut - ((a0 + a1) + (a2 + a3))) * rinv;
       me[nb] = e;
       r2 = fmaf(-e, e, r2);
       r2s[u] = r2;
