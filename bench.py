@@ -90,54 +90,104 @@ def profile_traffic(kernel_file: str):
 
 
 class ClockSampler:
+    """SM clock and clock-event reasons while the timed region runs.  NVML through ctypes,
+    polled every 5 ms (reading only), when libnvidia-ml loads; else nvidia-smi -lms 50.
+    mark()/stop() bracket the timed region; only samples taken inside it are reported."""
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    REASON_BITS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown", 0x40: "hw_thermal_slowdown"}
 
     def __init__(self, gpu_index: int):
         self.gpu = gpu_index
         self.proc = None
-        self.lines = []
+        self.nvml = None
+        self.samples = []          # (time, sm_mhz, sm_max_mhz, reasons)
+        self.t0 = None
+        self.stop_flag = False
+
+    def _nvml_handle(self):
+        import ctypes
+        lib = ctypes.CDLL("libnvidia-ml.so.1")
+        if lib.nvmlInit_v2() != 0:
+            return None
+        h = ctypes.c_void_p()
+        vis = os.environ.get("CUDA_VISIBLE_DEVICES", "").split(",")
+        entry = vis[self.gpu].strip() if vis and vis[0] != "" and self.gpu < len(vis) else str(self.gpu)
+        if entry.isdigit():
+            rc = lib.nvmlDeviceGetHandleByIndex_v2(ctypes.c_uint(int(entry)), ctypes.byref(h))
+        else:
+            rc = lib.nvmlDeviceGetHandleByUUID(entry.encode(), ctypes.byref(h))
+        return (lib, h) if rc == 0 else None
 
     def start(self):
+        try:
+            self.nvml = self._nvml_handle()
+        except OSError:
+            self.nvml = None
+        if self.nvml:
+            self.t = threading.Thread(target=self._poll_nvml, daemon=True)
+            self.t.start()
+            return
         try:
             self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
                                           "--format=csv,noheader,nounits", "-lms", "50"],
                                          stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
-            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t = threading.Thread(target=self._read_smi, daemon=True)
             self.t.start()
         except (OSError, FileNotFoundError):
             self.proc = None
 
-    def _read(self):
-        for line in self.proc.stdout:
-            self.lines.append(line.strip())
+    def _poll_nvml(self):
+        import ctypes
+        lib, h = self.nvml
+        clk, cmax, rs = ctypes.c_uint(), ctypes.c_uint(), ctypes.c_ulonglong()
+        get_reasons = getattr(lib, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+            lib.nvmlDeviceGetCurrentClocksThrottleReasons
+        while not self.stop_flag:
+            ok = lib.nvmlDeviceGetClockInfo(h, 1, ctypes.byref(clk)) == 0      # NVML_CLOCK_SM
+            lib.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(cmax))
+            get_reasons(h, ctypes.byref(rs))
+            if ok:
+                names = [n for bit, n in self.REASON_BITS.items() if rs.value & bit]
+                self.samples.append((time.perf_counter(), float(clk.value), float(cmax.value), names))
+            time.sleep(0.005)
 
-    def stop(self):
-        if not self.proc:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
-        self.proc.terminate()
-        try:
-            self.proc.wait(timeout=5)
-        except subprocess.TimeoutExpired:
-            self.proc.kill()
-        self.t.join(timeout=5)
-        sm, smax, reasons = [], None, set()
+    def _read_smi(self):
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for ln in self.lines:
-            parts = [x.strip() for x in ln.split(",")]
+        for line in self.proc.stdout:
+            parts = [x.strip() for x in line.strip().split(",")]
             if len(parts) < 9:
                 continue
             try:
-                sm.append(float(parts[1]))
-                smax = float(parts[2])
+                sm, smax = float(parts[1]), float(parts[2])
             except ValueError:
                 continue
-            for nm, v in zip(names, parts[5:9]):
-                if v.lower().startswith("active"):
-                    reasons.add(nm)
-        return {"sm_mhz": float(np.median(sm)) if sm else None, "sm_max_mhz": smax, "reasons": sorted(reasons),
-                "samples": len(sm)}
+            rs = [nm for nm, v in zip(names, parts[5:9]) if v.lower().startswith("active")]
+            self.samples.append((time.perf_counter(), sm, smax, rs))
+
+    def mark(self):
+        self.t0 = time.perf_counter()
+
+    def stop(self):
+        t1 = time.perf_counter()
+        if not self.nvml and not self.proc:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["clock sampling unavailable"], "samples": 0}
+        self.stop_flag = True
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+        self.t.join(timeout=5)
+        inside = [x for x in self.samples if self.t0 is None or self.t0 <= x[0] <= t1]
+        if not inside and self.samples:           # region shorter than one sample period
+            inside = [min(self.samples, key=lambda x: abs(x[0] - t1))]
+        sm = [x[1] for x in inside]
+        reasons = sorted({r for x in inside for r in x[3]})
+        return {"sm_mhz": float(np.median(sm)) if sm else None, "sm_max_mhz": inside[-1][2] if inside else None,
+                "reasons": reasons, "samples": len(sm), "source": "nvml" if self.nvml else "nvidia-smi"}
 
 
 def time_oracle(n_images: int, first_image: int = 0) -> float:
@@ -196,7 +246,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--cpu-images", type=int, default=1, help="oracle images timed for cpu_baseline")
-    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--batch", type=int, default=WORKLOAD.B, help="images per GPU (profiling on a smaller case)")
     ap.add_argument("--minimal", action="store_true",
@@ -246,7 +296,6 @@ def main():
         for _ in range(2):
             step()
         torch.cuda.synchronize()
-        sampler.lines.clear()
 
     # ---------------------------------------------------------------- timed region
     ctx.set_timing(True)
@@ -257,6 +306,7 @@ def main():
         pg.barrier()
     torch.cuda.synchronize()
     evs = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+    sampler.mark()
     evs[0].record(stream)
     for i in range(args.steps):
         step()
@@ -324,7 +374,8 @@ def main():
     text_h = torch.from_numpy(text_np.view(np.int16)).pin_memory()
     out_h = torch.empty((B, K, D), dtype=torch.int16).pin_memory()
     keep_h = torch.empty((B, K), dtype=torch.int32).pin_memory()
-    ctx.prune(text_h, vis_h, lens, K, out_h, keep_h)       # warm
+    for _ in range(3):                                    # warm (first pinned-buffer uses)
+        ctx.prune(text_h, vis_h, lens, K, out_h, keep_h)
     if pg:
         pg.barrier()
     t0 = time.perf_counter()
