@@ -75,9 +75,12 @@ struct Smem {
   static constexpr uint32_t TILES = STAGES * STAGE_BYTES;
   static constexpr uint32_t BARS = (2 * STAGES + 5 + (PROJ ? 1 : 0)) * 8;
   static constexpr uint32_t XPOSE = EPI == EPI_SM_STATS ? 4 * 32 * 33 * 4 : 0;   // per-warp 32x32 transposes
+  // hi/lo split epilogues: per epilogue warp two buffers of (hi, lo) 32x32 bf16 boxes for TMA stores
+  static constexpr bool TSTORE = EPI == EPI_GELU_SPLIT || EPI == EPI_BIAS_SPLIT;
+  static constexpr uint32_t STG = TSTORE ? 4 * 2 * 2 * 32 * 32 * 2 : 0;
   static constexpr uint32_t LSM = PROJ ? BN * BN * 4 : 0;       // L rows of the basis (pitch BN)
   static constexpr uint32_t PEXTRA = PROJ ? BN * 4 : 0;          // 1/r of the basis
-  static constexpr uint32_t TOTAL = 1024 + TILES + BARS + 16 + XPOSE + LSM + PEXTRA;
+  static constexpr uint32_t TOTAL = 1024 + TILES + STG + BARS + 16 + XPOSE + LSM + PEXTRA;
   static constexpr uint32_t TMEM_COLS = PROJ ? (2 * BN + 2 * kBM <= 256 ? 256u : 512u) : 2 * BN;   // + A A^T
   static constexpr int THREADS = 192;
 };
@@ -114,7 +117,8 @@ __device__ __forceinline__ TileCoord tile_coord(const KArgs& a, int t, int m_uni
 
 template <int BN, int STAGES, int EPI, bool CG2>
 __global__ void __launch_bounds__(Smem<BN, STAGES, EPI, CG2>::THREADS, 1)
-gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, KArgs a) {
+gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+               const __grid_constant__ CUtensorMap tmC, KArgs a) {
   using S = Smem<BN, STAGES, EPI, CG2>;
   constexpr bool PAIR = CG2;
   constexpr uint32_t IDESC = idesc_bf16(CG2 ? 2 * kBM : kBM, BN);
@@ -125,7 +129,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
   uint8_t* sB = smem + STAGES * S::A_BYTES;
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S::TILES);
+  uint8_t* stg = smem + S::TILES;                // TSTORE staging boxes (1024-aligned)
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S::TILES + S::STG);
   uint64_t* empty = full + STAGES;
   uint64_t* tfull = empty + STAGES;
   uint64_t* tempty = tfull + 2;
@@ -133,7 +138,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1 + (S::PROJ ? 1 : 0));
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   uint64_t* egsync = drain + 1;                  // EPI_PROJECT: epilogue warps' group barrier
-  float* xpose = reinterpret_cast<float*>(smem + S::TILES + S::BARS + 16);
+  float* xpose = reinterpret_cast<float*>(smem + S::TILES + S::STG + S::BARS + 16);
   float* Lsm = xpose + S::XPOSE / 4;
   float* rinv_sm = Lsm + S::LSM / 4;
 
@@ -558,6 +563,48 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             }
           }
         }
+      } else if constexpr (S::TSTORE) {
+        // (hi, lo) of each 32x32 chunk go through shared memory to two TMA box stores
+        // (coalesced, asynchronous); buffers alternate, reused once their store has read them
+        const int ew = warp - 2;
+        const int y = c.b * a.a_row_stride + c.m_blk * kBM + lane_grp * 32;   // first row of this warp
+#pragma unroll 1
+        for (int ch = 0; ch < BN / 32; ++ch) {
+          uint32_t r[32];
+          tmem_ld32(tbase + ch * 32, r);
+          const int cbase = col0 + ch * 32;
+          uint8_t* hb = stg + (ew * 2 + (ch & 1)) * 4096;     // [hi 32x32 | lo 32x32] bf16
+          if (lane == 0) bulk_wait_group_read<1>();      // this buffer's previous store has read it
+          __syncwarp();
+          uint32_t pk[16], pl[16];
+#pragma unroll
+          for (int j = 0; j < 32; j += 2) {
+            float x0 = __uint_as_float(r[j]), x1 = __uint_as_float(r[j + 1]);
+            if (a.bias) {
+              const __nv_bfloat162 bb = __ldg(reinterpret_cast<const __nv_bfloat162*>(a.bias + cbase + j));
+              x0 += __bfloat162float(bb.x);
+              x1 += __bfloat162float(bb.y);
+            }
+            if constexpr (EPI == EPI_GELU_SPLIT) { x0 = gelu_erf(x0); x1 = gelu_erf(x1); }
+            const __nv_bfloat162 hi = __floats2bfloat162_rn(x0, x1);
+            pk[j / 2] = *reinterpret_cast<const uint32_t*>(&hi);
+            pl[j / 2] = pack_bf16(x0 - __bfloat162float(hi.x), x1 - __bfloat162float(hi.y));
+          }
+          uint4* oh = reinterpret_cast<uint4*>(hb + lane * 64);
+          uint4* ol = reinterpret_cast<uint4*>(hb + 2048 + lane * 64);
+#pragma unroll
+          for (int v = 0; v < 4; ++v) {
+            oh[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+            ol[v] = make_uint4(pl[4 * v], pl[4 * v + 1], pl[4 * v + 2], pl[4 * v + 3]);
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0 && cbase < lim) {                  // rows past M are clipped by the store
+            tma_store_2d(&tmC, hb, cbase, y);
+            tma_store_2d(&tmC, hb + 2048, a.N + cbase, y);
+            bulk_commit_group();
+          }
+        }
       } else {
         __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(a.C) + crow + col0;
 #pragma unroll 1
@@ -600,6 +647,10 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       }
       acc ^= 1;
       if (acc == 0) acc_phase ^= 1;
+    }
+    if constexpr (S::TSTORE) {
+      if (lane == 0) bulk_wait_group_all();              // every box store has completed
+      __syncwarp();
     }
   }
   if constexpr (PAIR) cluster_sync();             // no commit or remote arrive still in flight
@@ -644,6 +695,19 @@ cudaError_t run(const GemmDesc& d, const KArgs& ka, int num_sms, cudaStream_t st
   CUtensorMap ta, tb;
   if (!make_map(&ta, d.A, d.a_rows_total, d.a_kwrap > 0 ? d.a_kwrap : d.K, kBM)) return cudaErrorInvalidValue;
   if (!make_map(&tb, d.B, d.b_rows_total, d.K, PAIR ? BN / 2 : BN)) return cudaErrorInvalidValue;
+  CUtensorMap tc = ta;
+  if constexpr (S::TSTORE) {       // output [rows, ldc] bf16, 32x32 boxes, no swizzle
+    auto fn = encode_fn();
+    if (!fn) return cudaErrorInvalidValue;
+    cuuint64_t dims[2] = {static_cast<cuuint64_t>(d.ldc), static_cast<cuuint64_t>(d.a_rows_total)};
+    cuuint64_t strides[1] = {static_cast<cuuint64_t>(d.ldc) * 2};
+    cuuint32_t box[2] = {32, 32};
+    cuuint32_t estr[2] = {1, 1};
+    if (fn(&tc, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, d.C, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+           CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) !=
+        CUDA_SUCCESS)
+      return cudaErrorInvalidValue;
+  }
   auto kern = gemm_tc_kernel<BN, STAGES, EPI, PAIR>;
   static bool attr_set = false;
   if (!attr_set) {
@@ -668,12 +732,12 @@ cudaError_t run(const GemmDesc& d, const KArgs& ka, int num_sms, cudaStream_t st
     attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, kern, ta, tb, ka);
+    return cudaLaunchKernelEx(&cfg, kern, ta, tb, tc, ka);
   }
   const int tiles = d.batch * m_tiles * n_tiles;
   if (tiles == 0) return cudaSuccess;
   const int grid = std::max(1, std::min(tiles, num_sms));
-  kern<<<grid, S::THREADS, S::TOTAL, st>>>(ta, tb, ka);
+  kern<<<grid, S::THREADS, S::TOTAL, st>>>(ta, tb, tc, ka);
   return cudaGetLastError();
 }
 
