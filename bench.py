@@ -385,6 +385,15 @@ def main():
     e2e_s = max_over_ranks(e2e_s, dev)
     e2e_value = B * args.e2e_steps * ws / e2e_s
     ctx.check()
+    # context for the end-to-end figure: this box's plain pinned host -> device copy rate
+    vis_tmp = torch.empty_like(vis)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(3):
+        vis_tmp.copy_(vis_h, non_blocking=True)
+    torch.cuda.synchronize()
+    h2d_gbs = 3 * vis_np.nbytes / (time.perf_counter() - t0) / 1e9
+    del vis_tmp
 
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu:
@@ -419,7 +428,8 @@ def main():
             "clocks": clocks,
             "e2e": {"value": e2e_value, "unit": "images/s",
                     "h2d_bytes_per_step": int(vis_np.nbytes + text_np.nbytes),
-                    "d2h_bytes_per_step": int(B * K * D * 2 + B * K * 4)},
+                    "d2h_bytes_per_step": int(B * K * D * 2 + B * K * 4),
+                    "host_to_device_gbs": round(h2d_gbs, 1)},
             "gpu_launches": int(launches),
             "cpu_baseline": cpu,
         }
