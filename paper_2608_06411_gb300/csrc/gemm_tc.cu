@@ -75,9 +75,11 @@ struct Smem {
   static constexpr uint32_t TILES = STAGES * STAGE_BYTES;
   static constexpr uint32_t BARS = (2 * STAGES + 5 + (PROJ ? 1 : 0)) * 8;
   static constexpr uint32_t XPOSE = EPI == EPI_SM_STATS ? 4 * 32 * 33 * 4 : 0;   // per-warp 32x32 transposes
-  // hi/lo split epilogues: per epilogue warp two buffers of (hi, lo) 32x32 bf16 boxes for TMA stores
-  static constexpr bool TSTORE = EPI == EPI_GELU_SPLIT || EPI == EPI_BIAS_SPLIT;
-  static constexpr uint32_t STG = TSTORE ? 4 * 2 * 2 * 32 * 32 * 2 : 0;
+  // bf16 outputs written by TMA box stores from per-warp staging: hi/lo split epilogues use two
+  // buffers of (hi, lo) 32x32 boxes, EPI_ROPE_SPLIT3 (BN = 128) one buffer of (hi, lo) x 2 halves
+  static constexpr bool TSTORE_ROPE = EPI == EPI_ROPE_SPLIT3 && BN == 128;
+  static constexpr bool TSTORE = EPI == EPI_GELU_SPLIT || EPI == EPI_BIAS_SPLIT || TSTORE_ROPE;
+  static constexpr uint32_t STG = TSTORE ? 4 * 4 * 32 * 32 * 2 : 0;
   static constexpr uint32_t LSM = PROJ ? BN * BN * 4 : 0;       // L rows of the basis (pitch BN)
   static constexpr uint32_t PEXTRA = PROJ ? BN * 4 : 0;          // 1/r of the basis
   static constexpr uint32_t TOTAL = 1024 + TILES + STG + BARS + 16 + XPOSE + LSM + PEXTRA;
@@ -351,6 +353,77 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
               *reinterpret_cast<float4*>(out + ch * 32 + j) = make_float4(o1[0], o1[1], o1[2], o1[3]);
               *reinterpret_cast<float4*>(out + HALF + ch * 32 + j) = make_float4(o2[0], o2[1], o2[2], o2[3]);
             }
+          }
+        }
+      } else if constexpr (S::TSTORE_ROPE) {
+        // BN == dp = 128; x = RoPE(acc + bias) * scale as bf16 (hi, lo) segments, staged per warp
+        // in shared memory and written by TMA box stores (rows past M are clipped)
+        constexpr int HALF = BN / 2;
+        float* aux = (a.aux && row_ok) ? a.aux + static_cast<long long>(row) * BN : nullptr;
+        int pos = 0;
+        if (row_ok) pos = a.pos ? __ldg(a.pos + row) : row % a.pos_mod;
+        const float2* rt = a.rope + pos;
+        const int seg_lo = a.split_kind == 0 ? 1 : 2;   // keys [hi, lo, hi], queries [hi, hi, lo]
+        const int ew = warp - 2;
+        const int y = c.b * a.a_row_stride + c.m_blk * kBM + lane_grp * 32;
+        uint8_t* sb = stg + ew * 8192;                 // [hi1 | lo1 | hi2 | lo2], 32 rows x 64 B each
+#pragma unroll 1
+        for (int ch = 0; ch < HALF / 32; ++ch) {
+          uint32_t r1[32], r2[32];
+          tmem_ld32(tbase + ch * 32, r1);
+          tmem_ld32(tbase + HALF + ch * 32, r2);
+          if (lane == 0) bulk_wait_group_read<0>();    // the previous chunk's stores have read sb
+          __syncwarp();
+#pragma unroll
+          for (int j = 0; j < 32; j += 8) {
+            float o1[8], o2[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+              const float2 cs = __ldg(rt + static_cast<long long>(ch * 32 + j + u) * a.rope_ld);
+              float x1 = __uint_as_float(r1[j + u]), x2 = __uint_as_float(r2[j + u]);
+              if (a.biasf) {
+                x1 += __ldg(a.biasf + ch * 32 + j + u);
+                x2 += __ldg(a.biasf + HALF + ch * 32 + j + u);
+              }
+              o1[u] = x1 * cs.x - x2 * cs.y;
+              o2[u] = x2 * cs.x + x1 * cs.y;
+            }
+            if (aux) {
+#pragma unroll
+              for (int u = 0; u < 8; u += 4) {
+                *reinterpret_cast<float4*>(aux + ch * 32 + j + u) = make_float4(o1[u], o1[u + 1], o1[u + 2], o1[u + 3]);
+                *reinterpret_cast<float4*>(aux + HALF + ch * 32 + j + u) =
+                    make_float4(o2[u], o2[u + 1], o2[u + 2], o2[u + 3]);
+              }
+            }
+#pragma unroll
+            for (int u = 0; u < 8; ++u) { o1[u] *= a.scale; o2[u] *= a.scale; }
+            uint32_t h1[4], l1[4], h2[4], l2[4];
+#pragma unroll
+            for (int u = 0; u < 8; u += 2) {
+              const __nv_bfloat162 a1 = __floats2bfloat162_rn(o1[u], o1[u + 1]);
+              const __nv_bfloat162 a2 = __floats2bfloat162_rn(o2[u], o2[u + 1]);
+              h1[u / 2] = *reinterpret_cast<const uint32_t*>(&a1);
+              h2[u / 2] = *reinterpret_cast<const uint32_t*>(&a2);
+              l1[u / 2] = pack_bf16(o1[u] - __bfloat162float(a1.x), o1[u + 1] - __bfloat162float(a1.y));
+              l2[u / 2] = pack_bf16(o2[u] - __bfloat162float(a2.x), o2[u + 1] - __bfloat162float(a2.y));
+            }
+            uint8_t* rowp = sb + lane * 64 + (j / 8) * 16;
+            *reinterpret_cast<uint4*>(rowp) = make_uint4(h1[0], h1[1], h1[2], h1[3]);
+            *reinterpret_cast<uint4*>(rowp + 2048) = make_uint4(l1[0], l1[1], l1[2], l1[3]);
+            *reinterpret_cast<uint4*>(rowp + 4096) = make_uint4(h2[0], h2[1], h2[2], h2[3]);
+            *reinterpret_cast<uint4*>(rowp + 6144) = make_uint4(l2[0], l2[1], l2[2], l2[3]);
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+#pragma unroll
+            for (int sg = 0; sg < 3; ++sg) {
+              const int x = sg * BN + ch * 32;
+              tma_store_2d(&tmC, sb + (sg == seg_lo ? 2048 : 0), x, y);
+              tma_store_2d(&tmC, sb + (sg == seg_lo ? 6144 : 4096), x + HALF, y);
+            }
+            bulk_commit_group();
           }
         }
       } else if constexpr (EPI == EPI_ROPE_SPLIT3) {
@@ -697,6 +770,8 @@ cudaError_t run(const GemmDesc& d, const KArgs& ka, int num_sms, cudaStream_t st
   if (!make_map(&tb, d.B, d.b_rows_total, d.K, PAIR ? BN / 2 : BN)) return cudaErrorInvalidValue;
   CUtensorMap tc = ta;
   if constexpr (S::TSTORE) {       // output [rows, ldc] bf16, 32x32 boxes, no swizzle
+    // box stores clip at a_rows_total, which is the row bound M only for one flat batch
+    if (d.batch != 1 || d.a_rows_total != d.M) return cudaErrorInvalidValue;
     auto fn = encode_fn();
     if (!fn) return cudaErrorInvalidValue;
     cuuint64_t dims[2] = {static_cast<cuuint64_t>(d.ldc), static_cast<cuuint64_t>(d.a_rows_total)};
@@ -799,7 +874,7 @@ cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t st) {
       return cudaErrorInvalidValue;
     case EPI_ROPE_SPLIT3:   // dp = 128: 2-SM pairs share the B tile (each CTA loads 64 of its rows)
       if (d.N == 64) return run<64, 8, EPI_ROPE_SPLIT3>(d, ka, num_sms, st);
-      if (d.N == 128) return run<128, 9, EPI_ROPE_SPLIT3, true>(d, ka, num_sms, st);
+      if (d.N == 128) return run<128, 8, EPI_ROPE_SPLIT3, true>(d, ka, num_sms, st);
       return cudaErrorInvalidValue;
     case EPI_SM_STATS:
       return run<256, 4, EPI_SM_STATS>(d, ka, num_sms, st);
