@@ -408,7 +408,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
               l1[u / 2] = pack_bf16(o1[u] - __bfloat162float(a1.x), o1[u + 1] - __bfloat162float(a1.y));
               l2[u / 2] = pack_bf16(o2[u] - __bfloat162float(a2.x), o2[u + 1] - __bfloat162float(a2.y));
             }
-            uint8_t* rowp = sb + lane * 64 + (j / 8) * 16;
+            uint8_t* rowp = sb + lane * 64 + ((j / 8) ^ ((lane >> 1) & 3)) * 16;   // 64-byte swizzle
             *reinterpret_cast<uint4*>(rowp) = make_uint4(h1[0], h1[1], h1[2], h1[3]);
             *reinterpret_cast<uint4*>(rowp + 2048) = make_uint4(l1[0], l1[1], l1[2], l1[3]);
             *reinterpret_cast<uint4*>(rowp + 4096) = make_uint4(h2[0], h2[1], h2[2], h2[3]);
@@ -663,12 +663,15 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             pk[j / 2] = *reinterpret_cast<const uint32_t*>(&hi);
             pl[j / 2] = pack_bf16(x0 - __bfloat162float(hi.x), x1 - __bfloat162float(hi.y));
           }
+          // 64-byte swizzle: 16-byte unit v of row r sits at unit v ^ ((r >> 1) & 3), so the
+          // eight rows of a quarter warp hit distinct banks
           uint4* oh = reinterpret_cast<uint4*>(hb + lane * 64);
           uint4* ol = reinterpret_cast<uint4*>(hb + 2048 + lane * 64);
+          const int sw = (lane >> 1) & 3;
 #pragma unroll
           for (int v = 0; v < 4; ++v) {
-            oh[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
-            ol[v] = make_uint4(pl[4 * v], pl[4 * v + 1], pl[4 * v + 2], pl[4 * v + 3]);
+            oh[v ^ sw] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+            ol[v ^ sw] = make_uint4(pl[4 * v], pl[4 * v + 1], pl[4 * v + 2], pl[4 * v + 3]);
           }
           fence_proxy_async_smem();
           __syncwarp();
@@ -769,7 +772,7 @@ cudaError_t run(const GemmDesc& d, const KArgs& ka, int num_sms, cudaStream_t st
   if (!make_map(&ta, d.A, d.a_rows_total, d.a_kwrap > 0 ? d.a_kwrap : d.K, kBM)) return cudaErrorInvalidValue;
   if (!make_map(&tb, d.B, d.b_rows_total, d.K, PAIR ? BN / 2 : BN)) return cudaErrorInvalidValue;
   CUtensorMap tc = ta;
-  if constexpr (S::TSTORE) {       // output [rows, ldc] bf16, 32x32 boxes, no swizzle
+  if constexpr (S::TSTORE) {       // output [rows, ldc] bf16, 32x32 boxes, 64-byte swizzle
     // box stores clip at a_rows_total, which is the row bound M only for one flat batch
     if (d.batch != 1 || d.a_rows_total != d.M) return cudaErrorInvalidValue;
     auto fn = encode_fn();
@@ -779,7 +782,7 @@ cudaError_t run(const GemmDesc& d, const KArgs& ka, int num_sms, cudaStream_t st
     cuuint32_t box[2] = {32, 32};
     cuuint32_t estr[2] = {1, 1};
     if (fn(&tc, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, d.C, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-           CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) !=
+           CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) !=
         CUDA_SUCCESS)
       return cudaErrorInvalidValue;
   }
