@@ -366,7 +366,7 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, 
   s.gbase = carve<int32_t>(sm, B);
   s.proj_lim = carve<int32_t>(sm, B);
   s.blist = carve<int32_t>(sm, B);
-  s.bcount = carve<int32_t>(sm, 1);
+  s.bcount = carve<int32_t>(sm, 2);
   s.done_count = carve<int32_t>(sm, 1);
   s.theta = static_cast<uint64_t*>(c->stheta.p);
   s.aslot = static_cast<int32_t*>(c->saslot.p);
@@ -393,14 +393,15 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, 
     s.Ec = static_cast<float*>(c->sEc.p);
     s.Vg = c->sVg.p;
     s.G = static_cast<float*>(c->sG.p);
-    CU_TRY(cudaMemsetAsync(s.done_count, 0, 4, st));
     GemmDesc d{};
     d.A = s.Vg; d.a_rows_total = static_cast<long long>(B) * R; d.a_row_stride = R;
     d.B = s.Vg; d.b_rows_total = static_cast<long long>(B) * R; d.b_row_stride = R;
     d.M = S; d.N = R; d.K = g.D; d.batch = B; d.n_limit = s.nlimit;
     d.C = s.G; d.ldc = R; d.c_batch_stride = static_cast<long long>(S) * R;
     d.epi = mapk::EPI_F32; d.status = c->status;
-    d.blist = s.blist; d.bcount = s.bcount;     // images still selecting (built by choose)
+    d.blist = s.blist;                           // images still selecting (built by choose)
+    // the GEMM after a list producer reads the count that producer appended through
+    auto take_list = [&](GemmDesc& g) { g.bcount = s.bcount + s.bc_par; s.bc_par ^= 1; };
     const long long cap = 8LL * (K + N / S) + 64;
     long long rounds = 0;
     int burst = (K0 + S - 1) / S + 6;   // rounds queued per host check; finished images skip
@@ -411,6 +412,7 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, 
       {
         GemmDesc d0 = d;              // only the K0 x K0 corner of the block
         d0.M = K0; d0.N = K0;
+        take_list(d0);
         MAP_TRY(gemm(c, d0, st));
       }
       CU_TRY(mapk::launch_sel_chol(s, st));
@@ -421,7 +423,7 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, 
       pd.A = vis; pd.a_rows_total = BN; pd.a_row_stride = N;
       pd.B = s.Vg; pd.b_rows_total = static_cast<long long>(B) * R; pd.b_row_stride = R; pd.b_base = S;
       pd.M = N; pd.N = kProjMaxBasis; pd.K = g.D; pd.batch = B; pd.n_limit = s.proj_lim;
-      pd.blist = s.blist; pd.bcount = s.bcount;   // images to project (built by proj_prep)
+      pd.blist = s.blist;                         // images to project (built by proj_prep)
       pd.C = nullptr; pd.ldc = 0; pd.c_batch_stride = 0;
       pd.epi = mapk::EPI_PROJECT; pd.status = c->status;
       pd.proj.state = s.state; pd.proj.scores = scores; pd.proj.Ec = s.Ec; pd.proj.KP = KP;
@@ -432,6 +434,7 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, 
         c->counters.launches += 3;
         CU_TRY(mapk::launch_sel_proj_prep(s, first, st));
         CU_TRY(mapk::launch_sel_gather(s, st));
+        take_list(pd);
         MAP_TRY(gemm(c, pd, st));
         CU_TRY(mapk::launch_sel_proj_done(s, st));
         return MAP_OK;
@@ -444,6 +447,7 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, 
       // the next active set the true top S
       c->counters.launches += 4;
       CU_TRY(mapk::launch_sel_choose(s, st));
+      take_list(d);
       MAP_TRY(gemm(c, d, st));
       CU_TRY(mapk::launch_sel_greedy(s, st));
       ++rounds;
@@ -455,6 +459,7 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, 
       for (int r = 0; r < burst; ++r) {
         c->counters.launches += 4;
         CU_TRY(mapk::launch_sel_choose(s, st));
+        take_list(d);
         MAP_TRY(gemm(c, d, st));
         CU_TRY(mapk::launch_sel_greedy(s, st));
       }

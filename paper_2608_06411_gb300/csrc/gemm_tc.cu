@@ -157,6 +157,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     fence_mbar_init();
   }
   if (warp == 0 && lane == 0) { tma_prefetch_desc(&tmA); tma_prefetch_desc(&tmB); }
+  pdl_enter();                                    // inputs below come from the previous kernel
   if (warp == 1) {
     if constexpr (CG2) { tmem_alloc_cg2(tmem_slot, S::TMEM_COLS); tmem_relinquish_cg2(); }
     else { tmem_alloc(tmem_slot, S::TMEM_COLS); tmem_relinquish(); }
@@ -803,20 +804,21 @@ cudaError_t run(const GemmDesc& d, const KArgs& ka, int num_sms, cudaStream_t st
     cfg.blockDim = dim3(S::THREADS);
     cfg.dynamicSmemBytes = S::TOTAL;
     cfg.stream = st;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = 2;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 2;
     return cudaLaunchKernelEx(&cfg, kern, ta, tb, tc, ka);
   }
   const int tiles = d.batch * m_tiles * n_tiles;
   if (tiles == 0) return cudaSuccess;
   const int grid = std::max(1, std::min(tiles, num_sms));
-  kern<<<grid, S::THREADS, S::TOTAL, st>>>(ta, tb, tc, ka);
-  return cudaGetLastError();
+  return launch_k(kern, dim3(grid), dim3(S::THREADS), S::TOTAL, st, ta, tb, tc, ka);
 }
 
 }  // namespace

@@ -152,8 +152,7 @@ extern "C" int map_select_noalloc(map_ctx* ctx, const float* scores, const void*
   if (rc != MAP_OK) return rc;
   ++*v.launches;
   if ((rc = rc_of(mapk::launch_sel_init(s, st))) != MAP_OK) return rc;
-  if (K0 < K) {
-    if ((rc = rc_of(cudaMemsetAsync(s.done_count, 0, 4, st))) != MAP_OK) return rc;
+  if (K0 < K) {                   // sel_init has zeroed done_count
     mapk::GemmDesc d{};
     d.A = s.Vg; d.a_rows_total = static_cast<long long>(B) * R; d.a_row_stride = R;
     d.B = s.Vg; d.b_rows_total = static_cast<long long>(B) * R; d.b_row_stride = R;

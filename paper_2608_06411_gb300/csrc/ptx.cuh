@@ -5,6 +5,8 @@
 #include <cstdint>
 #include <cuda.h>
 #include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <utility>
 
 namespace mapk {
 
@@ -302,6 +304,35 @@ __device__ __forceinline__ uint64_t desc_sw128(uint32_t saddr) {
 __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
   return (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(N >> 3) << 17) |
          (static_cast<uint32_t>(M >> 4) << 24);
+}
+
+// Programmatic dependent launch.  Every kernel of the library starts with pdl_enter(): it
+// waits until the grid launched before it on the stream has completed and its writes are
+// visible (a no-op when there is none), then lets the next grid be scheduled, so that grid's
+// blocks become resident and reach their own wait while this one runs instead of being
+// launched after it ends.  Blocks of the next grid occupy only what this grid leaves free:
+// it is scheduled once every block of this grid has started.
+__device__ __forceinline__ void pdl_enter() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// Launch with the programmatic-serialisation attribute (the next kernel may be scheduled
+// early; its pdl_enter() orders it after this one); extra attributes are appended.
+template <typename... KParams, typename... Args>
+cudaError_t launch_k(void (*kern)(KParams...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                     Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
 }
 
 }  // namespace mapk

@@ -12,6 +12,7 @@ namespace {
 // One warp per row; 16-byte loads; fp32 accumulation in a fixed order.
 __global__ void row_sqnorm_kernel(const uint4* __restrict__ x, long long rows, int vec_per_row,
                                   float* __restrict__ out) {
+  pdl_enter();
   const long long row = static_cast<long long>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (row >= rows) return;
@@ -36,6 +37,7 @@ __global__ void row_sqnorm_kernel(const uint4* __restrict__ x, long long rows, i
 // out[b, j, :] = V[b, idx[b, j], :]; one CTA per output row, uint4 copies.
 __global__ void gather_rows_kernel(const uint4* __restrict__ V, const int32_t* __restrict__ idx, int N, int k,
                                    int vec_per_row, uint4* __restrict__ out, int* status) {
+  pdl_enter();
   const long long r = blockIdx.x;           // b * k + j
   const long long b = r / k;
   const int src = __ldg(idx + r);
@@ -51,6 +53,7 @@ __global__ void gather_rows_kernel(const uint4* __restrict__ V, const int32_t* _
 // (max, sum) partials of one column over all slabs -> (max, 1/sum); thread = column.
 __global__ void stats_combine_kernel(const float2* __restrict__ part, int nparts, int ld, const int* __restrict__ lens,
                                      float2* __restrict__ fin) {
+  pdl_enter();
   const int b = blockIdx.y, col = blockIdx.x * blockDim.x + threadIdx.x;
   if (col >= lens[b]) return;
   const float2* p = part + static_cast<long long>(b) * nparts * ld + col;
@@ -66,6 +69,7 @@ __global__ void stats_combine_kernel(const float2* __restrict__ part, int nparts
 
 __global__ void sum_tiles_kernel(const float* __restrict__ part, int N, int n_tiles, long long total,
                                  float* __restrict__ scores) {
+  pdl_enter();
   const long long i = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
   if (i >= total) return;
   const long long b = i / N, n = i - b * N;
@@ -78,6 +82,7 @@ __global__ void sum_tiles_kernel(const float* __restrict__ part, int N, int n_ti
 __global__ void fold_weights_kernel(const __nv_bfloat16* __restrict__ Wp, const __nv_bfloat16* __restrict__ W2,
                                     const __nv_bfloat16* __restrict__ b2, int dp, int Dh,
                                     __nv_bfloat16* __restrict__ out, float* __restrict__ bias_out) {
+  pdl_enter();
   const int i = blockIdx.x * blockDim.x + threadIdx.x, p = blockIdx.y;
   if (i < Dh) {
     double acc = 0.0;
@@ -110,6 +115,7 @@ struct MetaChunk {
 // One CTA per image of the chunk.
 __global__ void query_meta_kernel(const __grid_constant__ MetaChunk m, int32_t* __restrict__ off,
                                   int32_t* __restrict__ len, int32_t* __restrict__ pos) {
+  pdl_enter();
   const int i = blockIdx.x, b = m.b0 + i;
   const int o = m.offs[i], l = m.lens[i];
   if (threadIdx.x == 0) {
@@ -121,6 +127,7 @@ __global__ void query_meta_kernel(const __grid_constant__ MetaChunk m, int32_t* 
 }
 
 __global__ void flags_to_host_kernel(const int32_t* a, const int* b, volatile int32_t* ah, volatile int* bh) {
+  pdl_enter();
   *ah = *a;
   *bh = *b;
 }
@@ -139,32 +146,29 @@ cudaError_t launch_query_meta(const int32_t* lens, const long long* offs, int B,
       m.lens[i] = lens[b0 + i];
       m.offs[i] = static_cast<int32_t>(offs[b0 + i]);
     }
-    query_meta_kernel<<<m.count, 128, 0, st>>>(m, off, len, pos);
-    const cudaError_t e = cudaGetLastError();
+    const cudaError_t e = launch_k(query_meta_kernel, dim3(m.count), dim3(128), 0, st, m, off, len, pos);
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;
 }
 
 cudaError_t launch_flags_to_host(const int32_t* a, const int* b, int32_t* a_host_dev, int* b_host_dev, cudaStream_t st) {
-  flags_to_host_kernel<<<1, 1, 0, st>>>(a, b, a_host_dev, b_host_dev);
-  return cudaGetLastError();
+  return launch_k(flags_to_host_kernel, dim3(1), dim3(1), 0, st, a, b, static_cast<volatile int32_t*>(a_host_dev),
+                  static_cast<volatile int*>(b_host_dev));
 }
 
 cudaError_t launch_fold_weights(const void* Wp, const void* W2, const void* b2, int dp, int Dh, void* out,
                                 float* bias_out, cudaStream_t st) {
   if (dp <= 0 || Dh <= 0) return cudaErrorInvalidValue;
-  fold_weights_kernel<<<dim3((Dh + 127) / 128, dp), 128, 0, st>>>(
-      static_cast<const __nv_bfloat16*>(Wp), static_cast<const __nv_bfloat16*>(W2),
-      static_cast<const __nv_bfloat16*>(b2), dp, Dh, static_cast<__nv_bfloat16*>(out), bias_out);
-  return cudaGetLastError();
+  return launch_k(fold_weights_kernel, dim3((Dh + 127) / 128, dp), dim3(128), 0, st,
+                  static_cast<const __nv_bfloat16*>(Wp), static_cast<const __nv_bfloat16*>(W2),
+                  static_cast<const __nv_bfloat16*>(b2), dp, Dh, static_cast<__nv_bfloat16*>(out), bias_out);
 }
 
 cudaError_t launch_stats_combine(const float2* part, int B, int nparts, int ld, const int* lens, float2* fin,
                                  cudaStream_t st) {
   dim3 g((ld + 127) / 128, B);
-  stats_combine_kernel<<<g, 128, 0, st>>>(part, nparts, ld, lens, fin);
-  return cudaGetLastError();
+  return launch_k(stats_combine_kernel, g, dim3(128), 0, st, part, nparts, ld, lens, fin);
 }
 
 cudaError_t launch_row_sqnorm(const void* x, long long rows, int D, float* out, cudaStream_t st) {
@@ -172,9 +176,8 @@ cudaError_t launch_row_sqnorm(const void* x, long long rows, int D, float* out, 
   if (D % 8 != 0) return cudaErrorInvalidValue;
   const int warps = 8;
   const long long blocks = (rows + warps - 1) / warps;
-  row_sqnorm_kernel<<<static_cast<unsigned>(blocks), warps * 32, 0, st>>>(static_cast<const uint4*>(x), rows, D / 8,
-                                                                          out);
-  return cudaGetLastError();
+  return launch_k(row_sqnorm_kernel, dim3(static_cast<unsigned>(blocks)), dim3(warps * 32), 0, st,
+                  static_cast<const uint4*>(x), rows, D / 8, out);
 }
 
 cudaError_t launch_gather(const void* V, const int32_t* idx, int B, int N, int k, int D, void* out, int* status,
@@ -182,15 +185,14 @@ cudaError_t launch_gather(const void* V, const int32_t* idx, int B, int N, int k
   if (B <= 0 || k <= 0) return cudaSuccess;
   if (D % 8 != 0) return cudaErrorInvalidValue;
   const long long rows = static_cast<long long>(B) * k;
-  gather_rows_kernel<<<static_cast<unsigned>(rows), 128, 0, st>>>(static_cast<const uint4*>(V), idx, N, k, D / 8,
-                                                                   static_cast<uint4*>(out), status);
-  return cudaGetLastError();
+  return launch_k(gather_rows_kernel, dim3(static_cast<unsigned>(rows)), dim3(128), 0, st,
+                  static_cast<const uint4*>(V), idx, N, k, D / 8, static_cast<uint4*>(out), status);
 }
 
 cudaError_t launch_sum_tiles(const float* part, int B, int N, int n_tiles, float* scores, cudaStream_t st) {
   const long long total = static_cast<long long>(B) * N;
-  sum_tiles_kernel<<<static_cast<unsigned>((total + 255) / 256), 256, 0, st>>>(part, N, n_tiles, total, scores);
-  return cudaGetLastError();
+  return launch_k(sum_tiles_kernel, dim3(static_cast<unsigned>((total + 255) / 256)), dim3(256), 0, st, part, N,
+                  n_tiles, total, scores);
 }
 
 }  // namespace mapk

@@ -162,6 +162,7 @@ __host__ __device__ inline int pow2_at_least(int n) {
 // ------------------------------------------------------------------ init
 // U = (p_hat * ||v||^lambda)^2, r2 = ||v||^2, nothing cached; R0 = top-K0 by p_hat, in order.
 __global__ void __launch_bounds__(1024) sel_init_kernel(SelState s) {
+  pdl_enter();
   extern __shared__ uint64_t sh64[];
   const int b = blockIdx.x;
   const long long base = static_cast<long long>(b) * s.N;
@@ -174,6 +175,10 @@ __global__ void __launch_bounds__(1024) sel_init_kernel(SelState s) {
     s.cstep[base + i] = 0;
     s.state[base + i] = 0;
     sh64[i] = make_key(p, i);
+  }
+  if (b == 0 && threadIdx.x == 0) {   // counters of this selection (earlier readers have completed)
+    if (s.bcount) { s.bcount[0] = 0; s.bcount[1] = 0; }
+    if (s.done_count) *s.done_count = 0;
   }
   if (threadIdx.x == 0) {
     s.npicks[b] = 0; s.nbasis[b] = 0; s.nb_gathered[b] = 0; s.done[b] = 0; s.nlimit[b] = 0;
@@ -198,16 +203,18 @@ __global__ void __launch_bounds__(1024) sel_init_kernel(SelState s) {
 // Active set of the next round: the next R0 chunk (forced), else the S candidates with the
 // largest bound U (value descending, ties to the lower index) and theta = the next key.
 __global__ void __launch_bounds__(1024) sel_choose_kernel(SelState s) {
+  pdl_enter();
   extern __shared__ uint64_t sh64[];
   const int b = blockIdx.x;
   const long long base = static_cast<long long>(b) * s.N;
   const int S = s.S;
   int32_t* aslot = s.aslot + static_cast<long long>(b) * S;
+  if (s.blist && b == 0 && threadIdx.x == 0) s.bcount[s.bc_par ^ 1] = 0;
   if (s.done[b]) {
     if (threadIdx.x == 0) s.nlimit[b] = 0;
     return;
   }
-  if (s.blist && threadIdx.x == 0) s.blist[atomicAdd(s.bcount, 1)] = b;
+  if (s.blist && threadIdx.x == 0) s.blist[atomicAdd(s.bcount + s.bc_par, 1)] = b;
   const int np = s.npicks[b], nb = s.nbasis[b];
   uint64_t theta = 0;
   int mode;
@@ -255,6 +262,7 @@ __global__ void __launch_bounds__(1024) sel_choose_kernel(SelState s) {
 constexpr int kGatherCtas = 64;
 
 __global__ void __launch_bounds__(128) sel_gather_kernel(SelState s) {
+  pdl_enter();
   const int b = blockIdx.y;
   if (s.done[b]) return;
   const int gb = s.gbase[b], lo = s.gb_lo[b], hi = s.gb_hi[b];
@@ -296,6 +304,7 @@ constexpr int kUpdWarps = 4;
 constexpr int kUpdRows = kChunk / kUpdWarps;
 
 __global__ void __launch_bounds__(kUpdSlots * kUpdWarps, 1) sel_update_kernel(SelState s) {
+  pdl_enter();
   extern __shared__ __align__(16) float shu[];
   __shared__ float rinv_c[kChunk];
   __shared__ float accs[kChunk][kUpdSlots];
@@ -399,6 +408,7 @@ constexpr int kCholThreads = kCholMax;
 // Left-looking, one thread per R0 position u, G[R0, R0] and the coordinate rows in shared
 // memory; one block barrier per basis vector.
 __global__ void __launch_bounds__(kCholThreads, 1) sel_chol_kernel(SelState s) {
+  pdl_enter();
   extern __shared__ __align__(16) float shc[];
   __shared__ float r2s[kCholMax], dg[kCholMax], dpick[kCholMax], ps[kCholMax];
   __shared__ int tk[kCholMax], mine_s[kCholMax], bidx[kCholMax];
@@ -526,6 +536,7 @@ __device__ __forceinline__ uint64_t warp_max_key(uint32_t hi, uint32_t lo) {
 
 template <bool SMEM>
 __global__ void __launch_bounds__(256, 1) sel_greedy_kernel(SelState s) {
+  pdl_enter();
   extern __shared__ __align__(16) float shf[];
   __shared__ uint64_t wkey[2][32];
   const int b = blockIdx.x;
@@ -721,16 +732,18 @@ __global__ void __launch_bounds__(256, 1) sel_greedy_kernel(SelState s) {
 // ------------------------------------------------------------------ projection set-up
 // Gathers every basis row of the images to project (no active tokens) for the projection.
 __global__ void sel_proj_prep_kernel(SelState s, int first) {
+  pdl_enter();
   const int b = blockIdx.x;
   const int nb = s.nbasis[b];
   const bool go = first || (!s.done[b] && nb > s.gbase[b] && nb <= kReprojMax);
+  if (s.blist && b == 0 && threadIdx.x == 0) s.bcount[s.bc_par ^ 1] = 0;
   if (!go) {
     if (threadIdx.x == 0) s.proj_lim[b] = 0;
     return;
   }
   for (int i = threadIdx.x; i < s.S; i += blockDim.x) s.aslot[static_cast<long long>(b) * s.S + i] = -1;
   if (threadIdx.x == 0) {
-    if (s.blist) s.blist[atomicAdd(s.bcount, 1)] = b;
+    if (s.blist) s.blist[atomicAdd(s.bcount + s.bc_par, 1)] = b;
     s.proj_lim[b] = kReprojMax;
     s.gbase[b] = 0;                                  // rows S + beta for the whole basis
     s.gb_lo[b] = 0;
@@ -740,6 +753,7 @@ __global__ void sel_proj_prep_kernel(SelState s, int first) {
 }
 
 __global__ void sel_proj_done_kernel(SelState s) {
+  pdl_enter();
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b < s.B && s.proj_lim[b] > 0) {
     s.gbase[b] = s.nbasis[b];
@@ -750,6 +764,7 @@ __global__ void sel_proj_done_kernel(SelState s) {
 // ------------------------------------------------------------------ outputs
 // keep = picks sorted ascending; pick_order = picks.
 __global__ void sel_finalize_kernel(const int32_t* picks, int K, int32_t* keep, int32_t* order) {
+  pdl_enter();
   extern __shared__ int32_t sh32[];
   const int b = blockIdx.x;
   const int32_t* p = picks + static_cast<long long>(b) * K;
@@ -764,12 +779,14 @@ __global__ void sel_finalize_kernel(const int32_t* picks, int K, int32_t* keep, 
 
 // top-K by p_hat (lambda = 0 or K0 = K): R0 computed by sel_init is the whole answer.
 __global__ void sel_copy_r0_kernel(const int32_t* r0, int K, int32_t* picks) {
+  pdl_enter();
   const int b = blockIdx.x;
   for (int i = threadIdx.x; i < K; i += blockDim.x)
     picks[static_cast<long long>(b) * K + i] = r0[static_cast<long long>(b) * K + i];
 }
 
 __global__ void sel_identity_kernel(int N, int32_t* keep, int32_t* order) {
+  pdl_enter();
   const int b = blockIdx.x;
   for (int i = threadIdx.x; i < N; i += blockDim.x) {
     keep[static_cast<long long>(b) * N + i] = i;
@@ -798,42 +815,34 @@ cudaError_t launch_sel_init(const SelState& s, cudaStream_t st) {
   const size_t sm = sel_init_smem(s.N, s.K0);
   cudaError_t e = cudaFuncSetAttribute(sel_init_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(sm));
   if (e != cudaSuccess) return e;
-  sel_init_kernel<<<s.B, 1024, sm, st>>>(s);
-  return cudaGetLastError();
+  return launch_k(sel_init_kernel, dim3(s.B), dim3(1024), sm, st, s);
 }
 
 cudaError_t launch_sel_choose(const SelState& s, cudaStream_t st) {
-  if (s.bcount) {
-    const cudaError_t z = cudaMemsetAsync(s.bcount, 0, sizeof(int32_t), st);
-    if (z != cudaSuccess) return z;
-  }
   const size_t sm = sel_choose_smem(s.N);
   cudaError_t e = cudaFuncSetAttribute(sel_choose_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(sm));
   if (e != cudaSuccess) return e;
-  sel_choose_kernel<<<s.B, 1024, sm, st>>>(s);
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  sel_gather_kernel<<<dim3(kGatherCtas, s.B), 128, 0, st>>>(s);
-  return cudaGetLastError();
+  if ((e = launch_k(sel_choose_kernel, dim3(s.B), dim3(1024), sm, st, s)) != cudaSuccess) return e;
+  return launch_k(sel_gather_kernel, dim3(kGatherCtas, s.B), dim3(128), 0, st, s);
 }
 
 cudaError_t launch_sel_greedy(const SelState& s, cudaStream_t st) {
   const size_t um = sel_update_smem(s.KP);
   cudaError_t e = cudaFuncSetAttribute(sel_update_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(um));
   if (e != cudaSuccess) return e;
-  sel_update_kernel<<<dim3((s.S + kUpdSlots - 1) / kUpdSlots, s.B), kUpdSlots * kUpdWarps, um, st>>>(s);
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  e = launch_k(sel_update_kernel, dim3((s.S + kUpdSlots - 1) / kUpdSlots, s.B), dim3(kUpdSlots * kUpdWarps), um, st, s);
+  if (e != cudaSuccess) return e;
   bool in_smem = false;
   const size_t sm = sel_greedy_smem(s.KP, s.S, &in_smem);
   if (in_smem) {
     e = cudaFuncSetAttribute(sel_greedy_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(sm));
     if (e != cudaSuccess) return e;
-    sel_greedy_kernel<true><<<s.B, s.S, sm, st>>>(s);
+    return launch_k(sel_greedy_kernel<true>, dim3(s.B), dim3(s.S), sm, st, s);
   } else {
     e = cudaFuncSetAttribute(sel_greedy_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(sm));
     if (e != cudaSuccess) return e;
-    sel_greedy_kernel<false><<<s.B, s.S, sm, st>>>(s);
+    return launch_k(sel_greedy_kernel<false>, dim3(s.B), dim3(s.S), sm, st, s);
   }
-  return cudaGetLastError();
 }
 
 cudaError_t launch_sel_chol(const SelState& s, cudaStream_t st) {
@@ -841,43 +850,32 @@ cudaError_t launch_sel_chol(const SelState& s, cudaStream_t st) {
   const size_t sm = sel_chol_smem(s.K0);
   cudaError_t e = cudaFuncSetAttribute(sel_chol_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(sm));
   if (e != cudaSuccess) return e;
-  sel_chol_kernel<<<s.B, kCholThreads, sm, st>>>(s);
-  return cudaGetLastError();
+  return launch_k(sel_chol_kernel, dim3(s.B), dim3(kCholThreads), sm, st, s);
 }
 
 cudaError_t launch_sel_finalize(const int32_t* picks, int B, int K, int32_t* keep, int32_t* order, cudaStream_t st) {
   const size_t sm = static_cast<size_t>(pow2_at_least(K)) * 4;
-  sel_finalize_kernel<<<B, 1024, sm, st>>>(picks, K, keep, order);
-  return cudaGetLastError();
+  return launch_k(sel_finalize_kernel, dim3(B), dim3(1024), sm, st, picks, K, keep, order);
 }
 
 cudaError_t launch_sel_copy_r0(const int32_t* r0, int B, int K, int32_t* picks, cudaStream_t st) {
-  sel_copy_r0_kernel<<<B, 256, 0, st>>>(r0, K, picks);
-  return cudaGetLastError();
+  return launch_k(sel_copy_r0_kernel, dim3(B), dim3(256), 0, st, r0, K, picks);
 }
 
 cudaError_t launch_sel_proj_prep(const SelState& s, bool first, cudaStream_t st) {
-  if (s.bcount) {
-    const cudaError_t z = cudaMemsetAsync(s.bcount, 0, sizeof(int32_t), st);
-    if (z != cudaSuccess) return z;
-  }
-  sel_proj_prep_kernel<<<s.B, 256, 0, st>>>(s, first ? 1 : 0);
-  return cudaGetLastError();
+  return launch_k(sel_proj_prep_kernel, dim3(s.B), dim3(256), 0, st, s, first ? 1 : 0);
 }
 
 cudaError_t launch_sel_gather(const SelState& s, cudaStream_t st) {
-  sel_gather_kernel<<<dim3(kGatherCtas, s.B), 128, 0, st>>>(s);
-  return cudaGetLastError();
+  return launch_k(sel_gather_kernel, dim3(kGatherCtas, s.B), dim3(128), 0, st, s);
 }
 
 cudaError_t launch_sel_proj_done(const SelState& s, cudaStream_t st) {
-  sel_proj_done_kernel<<<(s.B + 127) / 128, 128, 0, st>>>(s);
-  return cudaGetLastError();
+  return launch_k(sel_proj_done_kernel, dim3((s.B + 127) / 128), dim3(128), 0, st, s);
 }
 
 cudaError_t launch_sel_identity(int B, int N, int32_t* keep, int32_t* order, cudaStream_t st) {
-  sel_identity_kernel<<<B, 256, 0, st>>>(N, keep, order);
-  return cudaGetLastError();
+  return launch_k(sel_identity_kernel, dim3(B), dim3(256), 0, st, N, keep, order);
 }
 
 }  // namespace mapk

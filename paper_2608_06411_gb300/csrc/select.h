@@ -37,7 +37,11 @@ struct SelState {
   float* G;                       // [B, S, R] Gram block
   int32_t* done_count;            // images finished
   int32_t* proj_lim;              // [B] basis columns the projection GEMM computes (0: image skipped)
-  int32_t* blist; int32_t* bcount;  // images the next Gram / projection GEMM processes (optional)
+  // Images the next Gram / projection GEMM processes (optional): blist[0 .. bcount[bc_par]).
+  // A list producer (choose, projection prep) appends through bcount[bc_par] and zeroes
+  // bcount[bc_par ^ 1] for the next producer, so no separate reset precedes it; the host
+  // flips bc_par after each producer's consumer.
+  int32_t* blist; int32_t* bcount; int bc_par;
   int* status;
 };
 
