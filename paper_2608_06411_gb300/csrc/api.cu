@@ -670,8 +670,19 @@ int map_prune(map_ctx* ctx, const void* text_feats, const void* vis_feats, const
       return finish(MAP_ECUDA);
   }
   std::vector<cudaEvent_t> ev_in(nchunk);
-  auto chunk = [&](int i, int& b0, int& b1) { b0 = static_cast<int>(static_cast<long long>(B) * i / nchunk);
-                                               b1 = static_cast<int>(static_cast<long long>(B) * (i + 1) / nchunk); };
+  // Chunk boundaries, weights 3 : 3 : ... : 1.  The copy engine idles from the end of the last
+  // copy-in until the call returns, i.e. while the last chunk is scored, selected, gathered and
+  // copied out, so the last chunk is the small one; the others stay copy-bound.
+  std::vector<int> cb(nchunk + 1, 0);
+  {
+    const int wsum = 3 * (nchunk - 1) + 1;
+    for (int i = 1; i < nchunk; ++i) {
+      const int v = static_cast<int>(static_cast<long long>(B) * 3 * i / wsum);
+      cb[i] = std::min(std::max(v, cb[i - 1] + 1), B - (nchunk - i));
+    }
+    cb[nchunk] = B;
+  }
+  auto chunk = [&](int i, int& b0, int& b1) { b0 = cb[i]; b1 = cb[i + 1]; };
   for (int i = 0; i < nchunk; ++i) {
     int b0, b1;
     chunk(i, b0, b1);

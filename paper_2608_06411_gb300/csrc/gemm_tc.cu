@@ -564,6 +564,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             for (int i = 0; i < 32; ++i) accv[i] = __uint_as_float(g[i]);
           }
           const int b1 = min(nb0, b0 + 32);
+          const bool full32 = b1 - b0 > 16;             // uniform: rows 16..31 of this chunk exist
 #pragma unroll 1
           for (int qc = 0; qc < b0; qc += 8) {
             uint32_t ep[8];
@@ -572,12 +573,22 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
 #pragma unroll
               for (int qq = 0; qq < 8; qq += 4) {
 #pragma unroll
-                for (int i = 0; i < 32; ++i) {
+                for (int i = 0; i < 16; ++i) {
                   const float4 l = *reinterpret_cast<const float4*>(Lsm + (b0 + i) * BN + qc + qq);
                   accv[i] = fmaf(-l.x, __uint_as_float(ep[qq]), accv[i]);
                   accv[i] = fmaf(-l.y, __uint_as_float(ep[qq + 1]), accv[i]);
                   accv[i] = fmaf(-l.z, __uint_as_float(ep[qq + 2]), accv[i]);
                   accv[i] = fmaf(-l.w, __uint_as_float(ep[qq + 3]), accv[i]);
+                }
+                if (full32) {
+#pragma unroll
+                  for (int i = 16; i < 32; ++i) {
+                    const float4 l = *reinterpret_cast<const float4*>(Lsm + (b0 + i) * BN + qc + qq);
+                    accv[i] = fmaf(-l.x, __uint_as_float(ep[qq]), accv[i]);
+                    accv[i] = fmaf(-l.y, __uint_as_float(ep[qq + 1]), accv[i]);
+                    accv[i] = fmaf(-l.z, __uint_as_float(ep[qq + 2]), accv[i]);
+                    accv[i] = fmaf(-l.w, __uint_as_float(ep[qq + 3]), accv[i]);
+                  }
                 }
               }
             }
