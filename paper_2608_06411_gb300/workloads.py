@@ -189,3 +189,105 @@ def k0_for(K: int, k0_frac: float = 0.5, k0_abs: int = -1) -> int:
     clamped to [0, K].  The paper does not state K0; K/2 is the default reading."""
     k0 = k0_abs if k0_abs >= 0 else int(np.floor(k0_frac * K))
     return max(0, min(K, k0))
+
+
+# ----------------------------------------------------------------------------- QCTS inputs
+
+@dataclasses.dataclass(frozen=True)
+class AttentionWorkload:
+    """Text-to-vision attention maps of a host MLLM, the input of Question Contrastive
+    Teacher Selection (section "Question Contrastive Teacher Selection", Eq. 1-2).
+
+    For each image/question pair: the attention A[l, h, m, n] of question token m to visual
+    token n at head h of layer l, for the sample's own question (M_b tokens, ragged) and for
+    the fixed reference question (m_ref tokens).  The real maps come from a forward pass of
+    the MLLM on the paper's training data, which is not available; these are drawn with the
+    LLaVA shapes (L = 32 layers, H = 32 heads for the 7B backbones)."""
+    name: str
+    config_id: int
+    B: int          # image/question pairs
+    L: int          # language-model layers
+    H: int          # attention heads per layer
+    crops: int
+    grid: int
+    m_lo: int       # question length range (inclusive)
+    m_hi: int
+    m_ref: int      # tokens of the reference question ("What is shown in this image?")
+
+    @property
+    def N(self) -> int:
+        return self.crops * self.grid * self.grid
+
+
+ATTENTION_WORKLOADS = {
+    # LLaVA-1.5-7B: one 24x24 grid
+    "q0": AttentionWorkload("q0_llava15_n576", 10, 4, 32, 32, 1, 24, 8, 64, 7),
+    # LLaVA-NeXT-7B: 5 AnyRes crops of 24x24
+    "q1": AttentionWorkload("q1_llava_next_n2880", 11, 2, 32, 32, 5, 24, 16, 128, 7),
+}
+
+
+def attention_lens(w: AttentionWorkload, B: int | None = None) -> np.ndarray:
+    """Question lengths M_b, uniform in [m_lo, m_hi]."""
+    B = B or w.B
+    rng = np.random.Generator(np.random.PCG64(1000 * w.config_id + 999_999))
+    return rng.integers(w.m_lo, w.m_hi + 1, size=B).astype(np.int32)
+
+
+def make_attention(w: AttentionWorkload, sample: int, M: int, ref: bool = False, L: int | None = None,
+                   H: int | None = None, N: int | None = None, threads: int = 8) -> np.ndarray:
+    """Attention of one sample as bf16 bits [L, H, M, N].
+
+    Structure shared by both questions of a sample: a log-normal visual saliency per token
+    (the generic attention an image draws) and one rectangular region of interest in one
+    crop.  The sample's own question additionally pulls attention onto that region in the
+    middle layers: the pull has a Gaussian profile over layers, peaked at a random layer in
+    the middle half, scaled per head.  Every row gets log-normal noise and a random share in
+    [0.05, 0.5] of the query's attention mass (the rest goes to non-visual keys), so rows do
+    not sum to one.
+    """
+    L = L or w.L
+    H = H or w.H
+    N = N or w.N
+    base = np.random.Generator(np.random.PCG64(1000 * w.config_id + sample))
+    sal = base.standard_normal(N, dtype=np.float32) * np.float32(0.5)
+    roi = np.zeros(N, dtype=np.float32)
+    g = w.grid
+    crop = int(base.integers(w.crops))
+    rh, rw = (int(x) for x in base.integers(4, min(g, 10) + 1, size=2))
+    r0, c0 = int(base.integers(0, g - rh + 1)), int(base.integers(0, g - rw + 1))
+    rr, cc = np.meshgrid(np.arange(r0, r0 + rh), np.arange(c0, c0 + rw), indexing="ij")
+    idx = crop * g * g + rr.reshape(-1) * g + cc.reshape(-1)
+    roi[idx[idx < N]] = 1.0
+    l_peak = int(base.integers(L // 4, 3 * L // 4 + 1))
+    layer_gain = 3.0 * np.exp(-0.5 * ((np.arange(L) - l_peak) / max(L / 8.0, 1.0)) ** 2)
+    head_gain = base.uniform(0.3, 1.2, H)
+    out = np.empty((L, H, M, N), dtype=np.uint16)
+
+    def layer(l):
+        rng = np.random.Generator(np.random.PCG64([1000 * w.config_id + sample, int(ref), l]))
+        z = rng.standard_normal((H, M, N), dtype=np.float32) * np.float32(0.7)
+        z += sal
+        if not ref:
+            z += (layer_gain[l] * head_gain).astype(np.float32)[:, None, None] * roi
+        np.exp(z, out=z)
+        share = rng.uniform(0.05, 0.5, (H, M, 1)).astype(np.float32)
+        z *= share / z.sum(axis=-1, keepdims=True)
+        out[l] = f32_to_bf16_bits(z)
+
+    if M > 0:
+        with ThreadPoolExecutor(max_workers=max(1, threads)) as ex:
+            list(ex.map(layer, range(L)))
+    return out
+
+
+def make_attention_batch(w: AttentionWorkload, B: int | None = None, lens=None, threads: int = 8, L=None, H=None,
+                         N=None):
+    """(attn, lens, attn_ref): attn = the samples' [L, H, M_b, N] blocks flattened and packed
+    in sample order (uint16, 1-D), lens [B] int32, attn_ref [B, L, H, m_ref, N] uint16."""
+    B = B or w.B
+    lens = attention_lens(w, B) if lens is None else np.asarray(lens, dtype=np.int32)
+    blocks = [make_attention(w, b, int(lens[b]), False, L, H, N, threads).reshape(-1) for b in range(B)]
+    attn = np.concatenate(blocks) if blocks else np.zeros(0, np.uint16)
+    ref = np.stack([make_attention(w, b, w.m_ref, True, L, H, N, threads) for b in range(B)])
+    return attn, lens, ref
