@@ -15,6 +15,7 @@ scaling); there is no collective on the data path.
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import hashlib
 import json
 import math
@@ -57,6 +58,69 @@ def algorithmic(dims, N, K, lens):
     weights = 2 * (D * Dh + Dh * dp) * 2
     bytes_ = B * N * D * 2 + M * D * 2 + B * N * 4 + 2 * B * K * D * 2 + weights
     return flops, bytes_
+
+
+def method_as_written_flops(dims, N, K, lens):
+    """The same count with the second MLP layer and the projection as separate matrices
+    (2 Dh^2 + 2 Dh dp per token instead of 2 Dh dp), as the method is written."""
+    D, Dh, dp = dims.D, dims.Dh, dims.dp
+    per_tok = 2 * (D * Dh + Dh * Dh + Dh * dp)
+    B = len(lens)
+    M = int(np.sum(lens))
+    return B * N * per_tok + M * per_tok + 2 * M * N * dp + B * 2 * K * N * D
+
+
+def bench_qcts(mb, dev, stream, steps, hbm, cpu_on, samples=None):
+    """Question Contrastive Teacher Selection (Eq. 1-2) on LLaVA-NeXT-7B-shaped attention
+    maps: 2 samples x 32 layers x 32 heads, N = 2880, questions U[16,128] tokens and a
+    7-token reference question (1.1 GB of bf16 maps, larger than L2).  Timed with CUDA
+    events around each map_qcts call (all three of its launches)."""
+    import torch
+    wq = W.ATTENTION_WORKLOADS["q1"]
+    if samples is not None and samples != wq.B:
+        wq = dataclasses.replace(wq, B=samples)
+    attn_np, lens, ref_np = W.make_attention_batch(wq, threads=min(16, _CORES))
+    attn = torch.from_numpy(attn_np.view(np.int16)).to(dev)
+    ref = torch.from_numpy(ref_np.view(np.int16)).to(dev)
+    B, L, N = wq.B, wq.L, wq.N
+    outs = [torch.empty((B, L, N), dtype=torch.float32, device=dev) for _ in range(2)]
+    js = torch.empty((B, L), dtype=torch.float32, device=dev)
+    teacher = torch.empty(B, dtype=torch.int32, device=dev)
+    tp = torch.empty((B, N), dtype=torch.float32, device=dev)
+
+    def call():
+        mb.qcts(attn, lens, ref, L, wq.H, N, outs[0], outs[1], js, teacher, tp)
+
+    for _ in range(3):
+        call()
+    torch.cuda.synchronize()
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(steps + 1)]
+    evs[0].record(stream)
+    for i in range(steps):
+        call()
+        evs[i + 1].record(stream)
+    torch.cuda.synchronize()
+    ms = np.array([evs[i].elapsed_time(evs[i + 1]) for i in range(steps)])
+    avg_s = evs[0].elapsed_time(evs[-1]) / 1000.0 / steps
+    bytes_ = attn_np.nbytes + ref_np.nbytes + 2 * B * L * N * 4 + B * L * 4 + B * 4 + B * N * 4
+    res = {"workload": wq.name, "samples": B, "L": L, "H": wq.H, "N": N,
+           "question_len": [int(x) for x in lens], "ref_len": wq.m_ref,
+           "value": B / avg_s, "unit": "samples/s", "us_per_call_p50": float(np.percentile(ms, 50) * 1000),
+           "us_per_call_p99": float(np.percentile(ms, 99) * 1000),
+           "roofline": {"bound": "hbm", "kernel": "map_qcts (column sums, normalise + JS, teacher)",
+                        "achieved": bytes_ / avg_s / 1e9, "peak": hbm, "unit": "GB/s",
+                        "frac": bytes_ / avg_s / 1e9 / hbm, "algorithmic_bytes": int(bytes_)}}
+    if cpu_on:
+        from oracle import qcts_oracle as Q
+        one = attn_np[:L * wq.H * int(lens[0]) * N]
+        t0 = time.perf_counter()
+        Q.qcts_batch(one, lens[:1], ref_np[:1], L, wq.H, N)
+        secs = time.perf_counter() - t0
+        res["cpu_baseline"] = {"value": 1.0 / secs, "unit": "samples/s", "cores": _CORES, "kind": "oracle",
+                               "sample": f"sample 0 of the batch ({int(lens[0])} question tokens), numpy float64, "
+                                         f"{secs:.1f} s"}
+    del attn, ref
+    return res
 
 
 def measured_peaks():
@@ -248,6 +312,10 @@ def main():
     ap.add_argument("--cpu-images", type=int, default=1, help="oracle images timed for cpu_baseline")
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--no-qcts", action="store_true", help="skip the teacher-selection (QCTS) measurement")
+    ap.add_argument("--only-qcts", action="store_true",
+                    help="run only the teacher-selection measurement (for profiling), print its JSON")
+    ap.add_argument("--qcts-samples", type=int, default=W.ATTENTION_WORKLOADS["q1"].B)
     ap.add_argument("--batch", type=int, default=WORKLOAD.B, help="images per GPU (profiling on a smaller case)")
     ap.add_argument("--minimal", action="store_true",
                     help="time the steps only (no clock sampling, latency, e2e or CPU baseline): for ncu runs")
@@ -262,6 +330,12 @@ def main():
     ws, rank, local = dist_env()
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
+    if args.only_qcts:
+        if rank == 0:
+            hbm = measured_peaks()[0]
+            print(json.dumps(bench_qcts(mb, dev, torch.cuda.current_stream(), args.steps, hbm, False,
+                                        args.qcts_samples)))
+        return 0
     pg = None
     if ws > 1:
         import torch.distributed as dist
@@ -360,7 +434,7 @@ def main():
     k1 = torch.empty((1, w1.K), dtype=torch.int32, device=dev)
     s1 = torch.empty((1, w1.N), dtype=torch.float32, device=dev)
     lat = []
-    for i in range(60):
+    for i in range(1010):
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
         ctx.prune(t1, v1, [64], w1.K, o1, k1, s1)
@@ -395,6 +469,33 @@ def main():
     h2d_gbs = 3 * vis_np.nbytes / (time.perf_counter() - t0) / 1e9
     del vis_tmp
 
+    # ---------------------------------------------------------------- hand-off sequence (kept + question tokens)
+    step()
+    torch.cuda.synchronize()
+    rows = B * K + int(np.sum(lens))
+    seq = torch.empty((rows, D), dtype=torch.int16, device=dev)
+    pos = torch.empty(rows, dtype=torch.int32, device=dev)
+    for _ in range(3):
+        ctx.assemble(vis, keep, text, lens, 0, seq, pos)
+    hev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    hev[0].record(stream)
+    for _ in range(20):
+        ctx.assemble(vis, keep, text, lens, 0, seq, pos)
+    hev[1].record(stream)
+    torch.cuda.synchronize()
+    ctx.check()
+    h_s = hev[0].elapsed_time(hev[1]) / 1000.0 / 20
+    h_bytes = 2 * rows * D * 2 + rows * 4 + B * K * 4
+    handoff = {"us_per_call": h_s * 1e6, "rows": rows,
+               "roofline": {"bound": "hbm", "kernel": "assemble_kernel (kept tokens + questions, position ids)",
+                            "achieved": h_bytes / h_s / 1e9, "peak": hbm, "unit": "GB/s",
+                            "frac": h_bytes / h_s / 1e9 / hbm, "algorithmic_bytes": int(h_bytes)}}
+    del seq, pos
+
+    qcts = None
+    if rank == 0 and not args.no_qcts:
+        qcts = bench_qcts(mb, dev, stream, 20, hbm, ws == 1 and not args.no_cpu, args.qcts_samples)
+
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu:
         secs = time_oracle(args.cpu_images)
@@ -422,7 +523,10 @@ def main():
                          "peak_source": f"{peak_src} bf16 {'sustained' if sustained else 'burst'}",
                          "traffic": traffic},
             "step_roofline": {"algorithmic_gflop_per_image": flops / B / 1e9, "t_roofline_ms": t_roof * 1000,
-                              "frac": t_roof / step_s, "bound": "tensor" if flops / (bf16_burst * 1e12) >
+                              "frac": t_roof / step_s,
+                              "frac_method_as_written": max(method_as_written_flops(DIMS, N, K, lens) /
+                                                            (bf16_burst * 1e12), bytes_ / (hbm * 1e9)) / step_s,
+                              "bound": "tensor" if flops / (bf16_burst * 1e12) >
                               bytes_ / (hbm * 1e9) else "hbm", "peak_source": f"{peak_src} bf16 burst, hbm"},
             "kernel_ms_per_step": {"fv1": fv1_ms / args.steps, **{k: v[0] / args.steps for k, v in other.items()}},
             "clocks": clocks,
@@ -432,6 +536,8 @@ def main():
                     "host_to_device_gbs": round(h2d_gbs, 1)},
             "gpu_launches": int(launches),
             "cpu_baseline": cpu,
+            "handoff": handoff,
+            "qcts": qcts,
         }
         print(json.dumps(line))
     ctx.close()

@@ -93,8 +93,9 @@ int map_init(const map_config *cfg, const map_weights *w, map_ctx **out);
  *   vis_feats   bf16 [B, N, D] (device), 16-byte aligned.
  *   lens        int32 [B] HOST array: question tokens per image, each >= 1.
  *   scores      float32 [B, N] output (device).
- * B >= 1, N >= 1.  MLP outputs are rounded to bf16 after each layer; q, k, logits and
- * p_hat are fp32.
+ * B >= 1, N >= 1.  Inputs and weights are bf16; every product is accumulated in fp32,
+ * and the hidden MLP activations are kept to about 16 significant bits (a bf16 pair)
+ * rather than rounded to bf16; q, k, logits and p_hat are fp32.
  */
 int map_score(map_ctx *ctx, const void *text_feats, const void *vis_feats,
               const int32_t *lens, int B, int N, float *scores, void *stream);
@@ -131,6 +132,27 @@ int map_gather(map_ctx *ctx, const void *vis_feats, const int32_t *keep_idx, int
                int k, void *out, void *stream);
 
 /*
+ * Hand-off to the language model (last paragraph of section "Inference-Time Token
+ * Pruning"): the kept tokens, restored to their original order, keep their positional
+ * indices and are combined with the question tokens.  For image b, whose sequence starts
+ * at row o_b = b k + sum_{b' < b} lens[b'] of `seq`:
+ *   seq[o_b + j]     = vis_feats[b, keep_idx[b, j]],  pos_ids[o_b + j]     = keep_idx[b, j] + pos_offset
+ *   seq[o_b + k + m] = text_feats[t_b + m],           pos_ids[o_b + k + m] = N + m + pos_offset
+ * for j < k and m < lens[b], with t_b = sum_{b' < b} lens[b'] (the question follows the
+ * whole image, as in map_score).  pos_offset shifts every position (e.g. by the length of
+ * a system prompt placed before the image).
+ *   vis_feats  bf16 [B, N, D]; keep_idx int32 [B, k] (map_select's output);
+ *   text_feats bf16 [sum(lens), D]; lens int32 [B] HOST array, each >= 0;
+ *   seq        bf16 [sum_b (k + lens[b]), D] output; pos_ids int32 [same rows] output.
+ * Device pointers, caller-owned; vis_feats, text_feats and seq 16-byte aligned (MAP_EINVAL
+ * otherwise); 0 <= k <= N.  An index outside [0, N) is not copied: its pos_ids entry is
+ * -1 and map_status reports MAP_EINTERNAL.
+ */
+int map_assemble(map_ctx *ctx, const void *vis_feats, const int32_t *keep_idx,
+                 const void *text_feats, const int32_t *lens, int B, int N, int k,
+                 int pos_offset, void *seq, int32_t *pos_ids, void *stream);
+
+/*
  * map_select without allocating memory in the call (the paper has no counterpart; this
  * is a deployment variant of map_select).  Same arguments, results and limits as
  * map_select, but every scratch buffer is carved from one static device array of
@@ -162,6 +184,35 @@ int map_select_noalloc(map_ctx *ctx, const float *scores, const void *vis_feats,
 int map_prune(map_ctx *ctx, const void *text_feats, const void *vis_feats,
               const int32_t *lens, int B, int N, int k, void *out, int32_t *keep_idx,
               float *scores, void *stream);
+
+/*
+ * Question Contrastive Teacher Selection (section "Question Contrastive Teacher
+ * Selection", Eq. 1 and Eq. 2): the teacher layer whose attention supervises the
+ * predictor during training.  For every sample b and language-model layer l:
+ *   a^l_n     = 1/(H M_b) sum_h sum_m A^l[h, m, n]                        (Eq. 1)
+ *   p^l       = a^l / sum_n a^l_n          (l1 normalisation over visual tokens)
+ *   p_ref^l   = the same for the reference question's attention (M_ref tokens)
+ *   js[b, l]  = D_JS(p^l, p_ref^l) in nats (natural logarithm)
+ *   teacher[b] = l* = argmax_l js[b, l], ties to the lower layer               (Eq. 2)
+ * A layer whose aggregate sums to zero (M_b = 0, or attention that is all zero) gets the
+ * uniform distribution 1/N.  Context-free: it needs no map_init and no workspace.
+ *   attn       bf16, the samples' text-to-vision attention, packed in sample order: sample
+ *              b is a dense [L, H, lens[b], N] block (row (h, m) of layer l holds the
+ *              attention of question token m to the N visual tokens at head h).  Values
+ *              must be finite and non-negative (attention probabilities).
+ *   lens       int32 [B] HOST array: question tokens M_b per sample, each >= 0.
+ *   attn_ref   bf16 [B, L, H, M_ref, N]: the reference question's attention.
+ *   p, p_ref   float32 [B, L, N] outputs: the distributions p^l and p_ref^l.
+ *   js         float32 [B, L] output; teacher int32 [B] output (while the call runs it
+ *              also counts the finished layers of each sample).
+ *   teacher_p  float32 [B, N] output (p^{l*} of each sample) or NULL.
+ * All device pointers, caller-owned; attn and attn_ref 2-byte aligned (16-byte alignment
+ * with N % 8 == 0 takes the fastest path).  B, L, H, N, M_ref >= 1 (MAP_EINVAL
+ * otherwise); L <= 65535.  Asynchronous on `stream`; no device-side error conditions.
+ */
+int map_qcts(const void *attn, const int32_t *lens, const void *attn_ref, int M_ref, int B,
+             int L, int H, int N, float *p, float *p_ref, float *js, int32_t *teacher,
+             float *teacher_p, void *stream);
 
 /* Synchronises `stream` and returns the first deferred device-side error recorded by
  * this context since the last call (MAP_ETIMEOUT, MAP_EINTERNAL), clearing it; else a

@@ -49,7 +49,7 @@ from scipy.special import erf as _erf
 __all__ = [
     "bf16_bits_to_f64", "gelu", "mlp", "rope", "predict_queries",
     "predict_keys", "predicted_attention", "map_score", "resolve_k0", "select",
-    "select_replay", "gather",
+    "select_replay", "gather", "assemble",
 ]
 
 
@@ -286,3 +286,23 @@ def gather(vis_bits: np.ndarray, keep: np.ndarray) -> np.ndarray:
     """Compaction: out[b, j] = V[b, keep[b, j]] (a row copy of the bf16 bits)."""
     B = vis_bits.shape[0]
     return np.stack([vis_bits[b][np.asarray(keep[b], dtype=np.int64)] for b in range(B)])
+
+
+def assemble(vis_bits: np.ndarray, keep: np.ndarray, text_bits: np.ndarray, lens, pos_offset: int = 0):
+    """Hand-off to the language model (section "Inference-Time Token Pruning", last
+    paragraph): the kept tokens, restored to their original order, keep their positional
+    indices and are combined with the question tokens.  Per image b: its k kept visual
+    tokens (keep[b], ascending) at positions keep[b], then its M_b question tokens at
+    positions N + m (the question follows the full image), all shifted by pos_offset;
+    images one after another.  Returns (seq [sum_b (k + M_b), D] bf16 bits, pos int32)."""
+    B, N, _ = vis_bits.shape
+    rows, pos = [], []
+    o = 0
+    for b in range(B):
+        M = int(lens[b])
+        rows.append(vis_bits[b][np.asarray(keep[b], dtype=np.int64)])
+        rows.append(text_bits[o:o + M])
+        pos.append(np.asarray(keep[b], dtype=np.int64) + pos_offset)
+        pos.append(N + np.arange(M) + pos_offset)
+        o += M
+    return np.concatenate(rows, axis=0), np.concatenate(pos).astype(np.int32)

@@ -66,3 +66,26 @@ def check_selection(p: np.ndarray, V: np.ndarray, K: int, K0: int, gpu_order, gp
             return dict(ok=False, reason=f"step {s['t']}: picked {s['forced']}, oracle {s['best']} "
                                          f"(margin {s['margin']:.2e})", sub_margin_steps=subm, identical=False)
     return dict(ok=True, reason="", sub_margin_steps=subm, identical=False)
+
+
+# ----------------------------------------------------------------------------- QCTS
+# Distributions p^l, p_ref^l: elementwise relative error <= 2e-5 (fp32 sums of positive
+# bf16 values, about 1e-6 expected).  Divergences: relative error <= 1e-4 (plus 1e-7
+# absolute for near-zero values).  Teacher layer: equal to the oracle's wherever the
+# oracle's relative margin (js1 - js2) / js1 exceeds 1e-3; otherwise any layer whose
+# oracle divergence is within that margin of the largest.
+QCTS_P_RTOL, QCTS_JS_RTOL, QCTS_JS_ATOL, QCTS_LAYER_MARGIN = 2e-5, 1e-4, 1e-7, 1e-3
+
+
+def check_teacher_layer(js_oracle: np.ndarray, layer_gpu: int, margin: float = QCTS_LAYER_MARGIN) -> tuple:
+    """(ok, reason) for the GPU's teacher layer against the oracle's divergences."""
+    js = np.asarray(js_oracle, dtype=np.float64)
+    order = np.argsort(-js, kind="stable")
+    top = js[order[0]]
+    second = js[order[1]] if len(js) > 1 else -np.inf
+    rel = (top - second) / top if top > 0 else 0.0
+    if rel > margin:
+        ok = layer_gpu == int(order[0])
+        return ok, "" if ok else f"layer {layer_gpu}, oracle {int(order[0])} (margin {rel:.2e})"
+    ok = 0 <= layer_gpu < len(js) and js[layer_gpu] >= (1.0 - margin) * top
+    return ok, "" if ok else f"layer {layer_gpu} js {js[layer_gpu] if 0 <= layer_gpu < len(js) else None} vs {top}"

@@ -46,6 +46,10 @@ SIGNATURES = {
     "map_select_noalloc": (c_int, [c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_void_p, c_void_p,
                                    c_void_p]),
     "map_gather": (c_int, [c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_void_p, c_void_p]),
+    "map_qcts": (c_int, [c_void_p, POINTER(c_int32), c_void_p, c_int, c_int, c_int, c_int, c_int, c_void_p, c_void_p,
+                         c_void_p, c_void_p, c_void_p, c_void_p]),
+    "map_assemble": (c_int, [c_void_p, c_void_p, c_void_p, c_void_p, POINTER(c_int32), c_int, c_int, c_int, c_int,
+                             c_void_p, c_void_p, c_void_p]),
     "map_prune": (c_int, [c_void_p, c_void_p, c_void_p, POINTER(c_int32), c_int, c_int, c_int, c_void_p,
                           c_void_p, c_void_p, c_void_p]),
     "map_status": (c_int, [c_void_p, c_void_p]),
@@ -184,6 +188,20 @@ class Context:
         _check(lib.map_gather(self.h, _ptr(vis), _ptr(keep), B, N, k, _ptr(out), _stream(stream)), "map_gather")
         return out
 
+    def assemble(self, vis, keep, text, lens, pos_offset: int = 0, seq=None, pos=None, stream=None):
+        """map_assemble: per image, the kept tokens then the question tokens, with position ids."""
+        B, N, D = vis.shape
+        k = keep.shape[1]
+        arr, lp = _lens(lens)
+        rows = B * k + int(arr.sum())
+        if seq is None:
+            seq = torch.empty((rows, D), dtype=vis.dtype, device=vis.device)
+        if pos is None:
+            pos = torch.empty(rows, dtype=torch.int32, device=vis.device)
+        _check(lib.map_assemble(self.h, _ptr(vis), _ptr(keep), _ptr(text), lp, B, N, k, pos_offset, _ptr(seq),
+                                _ptr(pos), _stream(stream)), "map_assemble")
+        return seq, pos
+
     def prune(self, text, vis, lens, k: int, out, keep, scores=None, stream=None):
         """score + select + gather in one C call; buffers may be host (pinned or not) or device."""
         B, N = vis.shape[0], vis.shape[1]
@@ -221,3 +239,29 @@ class Context:
         ms, n = c_double(), c_longlong()
         _check(lib.map_read_timing(self.h, kid, ctypes.byref(ms), ctypes.byref(n)), "map_read_timing")
         return ms.value, n.value
+
+
+def qcts(attn, lens, attn_ref, L: int, H: int, N: int, p=None, p_ref=None, js=None, teacher=None,
+         teacher_p=None, want_teacher_p: bool = True, stream=None):
+    """map_qcts: Question Contrastive Teacher Selection on device tensors.
+
+    attn: packed bf16 (int16 storage) attention of the B samples ([L, H, lens[b], N] blocks
+    in sample order); attn_ref: [B, L, H, M_ref, N].  Returns (p, p_ref, js, teacher,
+    teacher_p); outputs not given are allocated here."""
+    arr, lp = _lens(lens)
+    B = int(arr.shape[0])
+    M_ref = int(attn_ref.shape[3])
+    dev = attn_ref.device
+    if p is None:
+        p = torch.empty((B, L, N), dtype=torch.float32, device=dev)
+    if p_ref is None:
+        p_ref = torch.empty((B, L, N), dtype=torch.float32, device=dev)
+    if js is None:
+        js = torch.empty((B, L), dtype=torch.float32, device=dev)
+    if teacher is None:
+        teacher = torch.empty(B, dtype=torch.int32, device=dev)
+    if teacher_p is None and want_teacher_p:
+        teacher_p = torch.empty((B, N), dtype=torch.float32, device=dev)
+    _check(lib.map_qcts(_ptr(attn), lp, _ptr(attn_ref), M_ref, B, L, H, N, _ptr(p), _ptr(p_ref), _ptr(js),
+                        _ptr(teacher), _ptr(teacher_p), _stream(stream)), "map_qcts")
+    return p, p_ref, js, teacher, teacher_p

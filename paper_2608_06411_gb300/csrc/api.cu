@@ -616,6 +616,26 @@ int map_gather(map_ctx* ctx, const void* vis_feats, const int32_t* keep_idx, int
   return gather_impl(ctx, vis_feats, keep_idx, B, N, k, out, static_cast<cudaStream_t>(stream));
 }
 
+int map_assemble(map_ctx* ctx, const void* vis_feats, const int32_t* keep_idx, const void* text_feats,
+                 const int32_t* lens, int B, int N, int k, int pos_offset, void* seq, int32_t* pos_ids,
+                 void* stream) {
+  if (!ctx || !vis_feats || !text_feats || !lens) return MAP_EINVAL;
+  if (B < 1 || N < 1 || k < 0 || k > N) return MAP_EINVAL;
+  long long rows = 0;
+  for (int b = 0; b < B; ++b) {
+    if (lens[b] < 0) return MAP_EINVAL;
+    rows += k + lens[b];
+  }
+  if (rows == 0) return MAP_OK;
+  if (!seq || !pos_ids || (k > 0 && !keep_idx)) return MAP_EINVAL;
+  if (!aligned16(vis_feats) || !aligned16(text_feats) || !aligned16(seq)) return MAP_EINVAL;
+  CU_TRY(cudaSetDevice(ctx->device));
+  ++ctx->counters.launches;
+  CU_TRY(mapk::launch_assemble(vis_feats, keep_idx, text_feats, lens, B, N, k, ctx->cfg.D, pos_offset, seq, pos_ids,
+                               ctx->status, static_cast<cudaStream_t>(stream)));
+  return MAP_OK;
+}
+
 int map_prune(map_ctx* ctx, const void* text_feats, const void* vis_feats, const int32_t* lens, int B, int N, int k,
               void* out, int32_t* keep_idx, float* scores, void* stream) {
   if (!ctx || !text_feats || !vis_feats || !lens || !out || !keep_idx) return MAP_EINVAL;

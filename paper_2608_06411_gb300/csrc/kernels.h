@@ -109,4 +109,10 @@ cudaError_t launch_stats_combine(const float2* part, int B, int nparts, int ld, 
 cudaError_t launch_gather(const void* V, const int32_t* idx, int B, int N, int k, int D, void* out,
                           int* status, cudaStream_t st);
 
+// Hand-off sequence per image: the kept rows V[b, idx[b, j]] (j < k), then the image's
+// lens[b] question rows of T (packed in image order); pos = the kept index or N + m, plus
+// pos_offset.  Out-of-range indices are not copied: pos = -1 and ST_BADINDEX in *status.
+cudaError_t launch_assemble(const void* V, const int32_t* idx, const void* T, const int32_t* lens, int B, int N,
+                            int k, int D, int pos_offset, void* seq, int32_t* pos, int* status, cudaStream_t st);
+
 }  // namespace mapk

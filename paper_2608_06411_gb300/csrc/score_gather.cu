@@ -126,6 +126,46 @@ __global__ void query_meta_kernel(const __grid_constant__ MetaChunk m, int32_t* 
   for (int t = threadIdx.x; t < l; t += blockDim.x) pos[o + t] = m.N + t;
 }
 
+constexpr int kAsmImages = 512;
+struct AssembleChunk {
+  int b0, count, N, k, pos_offset;
+  int32_t lens[kAsmImages];
+  long long text_row[kAsmImages];   // first question row of each image in text_feats
+  long long seq_row[kAsmImages];    // first row of each image's output sequence
+};
+
+// Hand-off sequence: row j of image b is kept token keep[b, j] (j < k) or question token
+// j - k; one CTA per output row (grid: rows of the longest sequence in the chunk x images).
+__global__ void assemble_kernel(const __grid_constant__ AssembleChunk m, const uint4* __restrict__ V,
+                                const int32_t* __restrict__ idx, const uint4* __restrict__ T, int vec_per_row,
+                                uint4* __restrict__ seq, int32_t* __restrict__ pos, int* status) {
+  pdl_enter();
+  const int i = blockIdx.y, j = blockIdx.x;
+  const long long b = m.b0 + i;
+  if (j >= m.k + m.lens[i]) return;
+  const long long r = m.seq_row[i] + j;
+  const uint4* src;
+  int p;
+  if (j < m.k) {
+    const int t = __ldg(idx + b * m.k + j);
+    if (t < 0 || t >= m.N) {
+      if (threadIdx.x == 0) {
+        atomicOr(status, ST_BADINDEX);
+        pos[r] = -1;
+      }
+      return;
+    }
+    src = V + (b * m.N + t) * vec_per_row;
+    p = t;
+  } else {
+    src = T + (m.text_row[i] + (j - m.k)) * vec_per_row;
+    p = m.N + (j - m.k);
+  }
+  if (threadIdx.x == 0) pos[r] = p + m.pos_offset;
+  uint4* d = seq + r * vec_per_row;
+  for (int v = threadIdx.x; v < vec_per_row; v += blockDim.x) d[v] = __ldg(src + v);
+}
+
 __global__ void flags_to_host_kernel(const int32_t* a, const int* b, volatile int32_t* ah, volatile int* bh) {
   pdl_enter();
   *ah = *a;
@@ -147,6 +187,35 @@ cudaError_t launch_query_meta(const int32_t* lens, const long long* offs, int B,
       m.offs[i] = static_cast<int32_t>(offs[b0 + i]);
     }
     const cudaError_t e = launch_k(query_meta_kernel, dim3(m.count), dim3(128), 0, st, m, off, len, pos);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+cudaError_t launch_assemble(const void* V, const int32_t* idx, const void* T, const int32_t* lens, int B, int N,
+                            int k, int D, int pos_offset, void* seq, int32_t* pos, int* status, cudaStream_t st) {
+  if (D % 8 != 0) return cudaErrorInvalidValue;
+  long long trow = 0, srow = 0;
+  for (int b0 = 0; b0 < B; b0 += kAsmImages) {
+    AssembleChunk m;
+    m.b0 = b0;
+    m.count = B - b0 < kAsmImages ? B - b0 : kAsmImages;
+    m.N = N;
+    m.k = k;
+    m.pos_offset = pos_offset;
+    int max_rows = 0;
+    for (int i = 0; i < m.count; ++i) {
+      m.lens[i] = lens[b0 + i];
+      m.text_row[i] = trow;
+      m.seq_row[i] = srow;
+      trow += lens[b0 + i];
+      srow += k + lens[b0 + i];
+      max_rows = std::max(max_rows, k + lens[b0 + i]);
+    }
+    if (max_rows == 0) continue;
+    const cudaError_t e = launch_k(assemble_kernel, dim3(max_rows, m.count), dim3(128), 0, st, m,
+                                   static_cast<const uint4*>(V), idx, static_cast<const uint4*>(T), D / 8,
+                                   static_cast<uint4*>(seq), pos, status);
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;

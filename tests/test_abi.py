@@ -65,3 +65,30 @@ def test_bad_arguments_are_rejected_on_the_host(mb):
     assert lib.map_status(None, None) == mb.MAP_EINVAL
     assert lib.map_get_counters(None, None) == mb.MAP_EINVAL
     lib.map_destroy(None)
+
+
+def test_qcts_bad_arguments_are_rejected_on_the_host(mb):
+    lib = mb.lib
+    lens = (ctypes.c_int32 * 2)(3, 4)
+    neg = (ctypes.c_int32 * 2)(3, -1)
+    f = 256   # a non-null stand-in; nothing is dereferenced or launched on an argument error
+    assert lib.map_qcts(None, lens, f, 2, 2, 4, 2, 8, f, f, f, f, None, None) == mb.MAP_EINVAL
+    assert lib.map_qcts(f, None, f, 2, 2, 4, 2, 8, f, f, f, f, None, None) == mb.MAP_EINVAL
+    assert lib.map_qcts(f, lens, f, 2, 2, 4, 2, 8, None, f, f, f, None, None) == mb.MAP_EINVAL
+    assert lib.map_qcts(f, lens, f, 0, 2, 4, 2, 8, f, f, f, f, None, None) == mb.MAP_EINVAL
+    assert lib.map_qcts(f, lens, f, 2, 0, 4, 2, 8, f, f, f, f, None, None) == mb.MAP_EINVAL
+    assert lib.map_qcts(f, lens, f, 2, 2, 0, 2, 8, f, f, f, f, None, None) == mb.MAP_EINVAL
+    assert lib.map_qcts(f, lens, f, 2, 2, 4, 2, 0, f, f, f, f, None, None) == mb.MAP_EINVAL
+    assert lib.map_qcts(f, neg, f, 2, 2, 4, 2, 8, f, f, f, f, None, None) == mb.MAP_EINVAL
+    assert lib.map_qcts(f + 1, lens, f, 2, 2, 4, 2, 8, f, f, f, f, None, None) == mb.MAP_EINVAL
+
+
+def test_assemble_bad_arguments_are_rejected_on_the_host(mb):
+    lib = mb.lib
+    lens = (ctypes.c_int32 * 1)(3)
+    neg = (ctypes.c_int32 * 1)(-1)
+    f = 256
+    assert lib.map_assemble(None, f, f, f, lens, 1, 8, 2, 0, f, f, None) == mb.MAP_EINVAL
+    assert lib.map_assemble(f, f, f, f, neg, 1, 8, 2, 0, f, f, None) == mb.MAP_EINVAL
+    assert lib.map_assemble(f, f, f, f, lens, 1, 8, 9, 0, f, f, None) == mb.MAP_EINVAL
+    assert lib.map_assemble(f, f, f, f, lens, 0, 8, 2, 0, f, f, None) == mb.MAP_EINVAL

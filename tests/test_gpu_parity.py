@@ -223,6 +223,38 @@ def test_gather_rejects_bad_index_without_faulting():
     assert ctx.status() == mb.MAP_OK
 
 
+def test_assemble_is_bit_exact():
+    dims = W.PredictorDims(D=512, Dh=256, dp=64)
+    ctx, _ = make_ctx(dims)
+    rng = np.random.default_rng(4)
+    B, N, K = 3, 90, 17
+    vis = rng.integers(0, 2 ** 16, size=(B, N, 512), dtype=np.uint16)
+    lens = np.array([5, 0, 12], np.int32)
+    text = rng.integers(0, 2 ** 16, size=(int(lens.sum()), 512), dtype=np.uint16)
+    keep = np.sort(np.stack([rng.choice(N, K, replace=False) for _ in range(B)]), 1).astype(np.int32)
+    for k, off in [(K, 35), (0, 0), (N, 7)]:
+        kp = keep[:, :k] if k <= K else np.tile(np.arange(N, dtype=np.int32), (B, 1))
+        seq, pos = ctx.assemble(dev_bits(vis), torch.from_numpy(np.ascontiguousarray(kp)).to(DEV), dev_bits(text),
+                                lens, pos_offset=off)
+        torch.cuda.synchronize()
+        ctx.check()
+        s_ref, p_ref = O.assemble(vis, kp, text, lens, off)
+        np.testing.assert_array_equal(seq.cpu().numpy().view(np.uint16), s_ref)
+        np.testing.assert_array_equal(pos.cpu().numpy(), p_ref)
+
+
+def test_assemble_rejects_bad_index_without_faulting():
+    dims = W.PredictorDims(D=512, Dh=256, dp=64)
+    ctx, _ = make_ctx(dims)
+    vis = torch.zeros((1, 10, 512), dtype=torch.int16, device=DEV)
+    text = torch.ones((2, 512), dtype=torch.int16, device=DEV)
+    keep = torch.tensor([[0, 12]], dtype=torch.int32, device=DEV)
+    seq, pos = ctx.assemble(vis, keep, text, [2])
+    assert ctx.status() == mb.MAP_EINTERNAL
+    assert pos.cpu().tolist() == [0, -1, 10, 11]
+    assert ctx.status() == mb.MAP_OK
+
+
 def test_prune_host_buffers_equal_device_path():
     dims = W.PredictorDims(D=512, Dh=256, dp=64)
     ctx, w = make_ctx(dims)
@@ -294,6 +326,13 @@ def _batch_parity(wl, sample, K, K0=None, **ctxkw):
     torch.cuda.synchronize()
     for b in sample:
         np.testing.assert_array_equal(out[b].cpu().numpy().view(np.uint16), vis[b][keep[b]])
+    # hand-off sequence for the whole batch (kept tokens, then questions, with positions)
+    seq, pos = ctx.assemble(vis_t, torch.from_numpy(keep).to(DEV), text_t, lens, pos_offset=35)
+    torch.cuda.synchronize()
+    ctx.check()
+    s_ref, p_ref = O.assemble(vis, keep, text, lens, 35)
+    np.testing.assert_array_equal(seq.cpu().numpy().view(np.uint16), s_ref)
+    np.testing.assert_array_equal(pos.cpu().numpy(), p_ref)
     return lens
 
 

@@ -435,3 +435,19 @@ def test_r0_ties_go_to_lower_index():
     r = O.select(p, np.eye(5), 3, 3)
     assert r["picks"].tolist() == [1, 3, 4]
     assert O.select(p, np.eye(5), 4, 4)["picks"].tolist() == [1, 3, 4, 0]
+
+
+def test_assemble_hand_example():
+    # B = 2 images of N = 4 tokens (D = 2), k = 2 kept each, question lengths 1 and 2.
+    # Image 0 keeps tokens 1, 3 then its question token; image 1 keeps 0, 2 then two tokens.
+    vis = np.arange(16, dtype=np.uint16).reshape(2, 4, 2)
+    text = np.array([[100, 101], [200, 201], [300, 301]], dtype=np.uint16)
+    seq, pos = O.assemble(vis, np.array([[1, 3], [0, 2]]), text, [1, 2], pos_offset=5)
+    np.testing.assert_array_equal(seq, [[2, 3], [6, 7], [100, 101],
+                                        [8, 9], [12, 13], [200, 201], [300, 301]])
+    # kept tokens keep their original positions; question tokens follow the whole image (N + m)
+    np.testing.assert_array_equal(pos, [6, 8, 9, 5, 7, 9, 10])
+    # an image without question tokens contributes its kept tokens only; k = 0 leaves the questions
+    seq, pos = O.assemble(vis, np.zeros((2, 0), np.int64), text, [3, 0])
+    np.testing.assert_array_equal(seq, text)
+    np.testing.assert_array_equal(pos, [4, 5, 6])
