@@ -50,21 +50,41 @@ __global__ void gather_rows_kernel(const uint4* __restrict__ V, const int32_t* _
   for (int v = threadIdx.x; v < vec_per_row; v += blockDim.x) d[v] = __ldg(s + v);
 }
 
-// (max, sum) partials of one column over all slabs -> (max, 1/sum); thread = column.
-__global__ void stats_combine_kernel(const float2* __restrict__ part, int nparts, int ld, const int* __restrict__ lens,
-                                     float2* __restrict__ fin) {
+// (max, sum) partials of one column over all slabs -> (max, 1/sum).  A block covers 32
+// columns (threadIdx.x, coalesced) with kCombY threads per column splitting the slabs; the
+// kCombY partial maxima and sums are combined in a fixed order in shared memory.
+constexpr int kCombY = 8;
+__global__ void __launch_bounds__(32 * kCombY) stats_combine_kernel(const float2* __restrict__ part, int nparts,
+                                                                    int ld, const int* __restrict__ lens,
+                                                                    float2* __restrict__ fin) {
+  __shared__ float red[kCombY][32];
   pdl_enter();
-  const int b = blockIdx.y, col = blockIdx.x * blockDim.x + threadIdx.x;
-  if (col >= lens[b]) return;
+  const int b = blockIdx.y, x = threadIdx.x, y = threadIdx.y, col = blockIdx.x * 32 + x;
+  const bool on = col < lens[b];
   const float2* p = part + static_cast<long long>(b) * nparts * ld + col;
   float m = -INFINITY;
-  for (int i = 0; i < nparts; ++i) m = fmaxf(m, p[static_cast<long long>(i) * ld].x);
+  if (on)
+    for (int i = y; i < nparts; i += kCombY) m = fmaxf(m, p[static_cast<long long>(i) * ld].x);
+  red[y][x] = m;
+  __syncthreads();
+  m = red[0][x];
+#pragma unroll
+  for (int j = 1; j < kCombY; ++j) m = fmaxf(m, red[j][x]);
+  __syncthreads();
   float sum = 0.f;
-  for (int i = 0; i < nparts; ++i) {
-    const float2 v = p[static_cast<long long>(i) * ld];
-    if (v.y > 0.f) sum += v.y * expf(v.x - m);
+  if (on)
+    for (int i = y; i < nparts; i += kCombY) {
+      const float2 v = p[static_cast<long long>(i) * ld];
+      if (v.y > 0.f) sum += v.y * expf(v.x - m);
+    }
+  red[y][x] = sum;
+  __syncthreads();
+  if (y == 0 && on) {
+    float s = red[0][x];
+#pragma unroll
+    for (int j = 1; j < kCombY; ++j) s += red[j][x];
+    fin[static_cast<long long>(b) * ld + col] = make_float2(m, 1.0f / s);
   }
-  fin[static_cast<long long>(b) * ld + col] = make_float2(m, 1.0f / sum);
 }
 
 __global__ void sum_tiles_kernel(const float* __restrict__ part, int N, int n_tiles, long long total,
@@ -236,8 +256,8 @@ cudaError_t launch_fold_weights(const void* Wp, const void* W2, const void* b2, 
 
 cudaError_t launch_stats_combine(const float2* part, int B, int nparts, int ld, const int* lens, float2* fin,
                                  cudaStream_t st) {
-  dim3 g((ld + 127) / 128, B);
-  return launch_k(stats_combine_kernel, g, dim3(128), 0, st, part, nparts, ld, lens, fin);
+  dim3 g((ld + 31) / 32, B);
+  return launch_k(stats_combine_kernel, g, dim3(32, kCombY), 0, st, part, nparts, ld, lens, fin);
 }
 
 cudaError_t launch_row_sqnorm(const void* x, long long rows, int D, float* out, cudaStream_t st) {

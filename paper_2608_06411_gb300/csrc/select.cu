@@ -260,8 +260,9 @@ __global__ void __launch_bounds__(1024) sel_choose_kernel(SelState s) {
 // row S + beta - gbase <- basis token beta for the basis vectors added since the last round.
 // kGatherCtas CTAs per image, each walking every kGatherCtas-th row; finished images exit.
 constexpr int kGatherCtas = 64;
+constexpr int kGatherThreads = 128;
 
-__global__ void __launch_bounds__(128) sel_gather_kernel(SelState s) {
+__global__ void __launch_bounds__(kGatherThreads) sel_gather_kernel(SelState s) {
   pdl_enter();
   const int b = blockIdx.y;
   if (s.done[b]) return;
@@ -276,9 +277,19 @@ __global__ void __launch_bounds__(128) sel_gather_kernel(SelState s) {
       if (beta >= lo && beta < hi) src = s.basis_tok[static_cast<long long>(b) * s.K + beta];
     }
     if (src < 0) continue;                               // uniform in the CTA
-    const uint4* V = reinterpret_cast<const uint4*>(s.V) + (static_cast<long long>(b) * s.N + src) * vec;
-    uint4* dst = reinterpret_cast<uint4*>(s.Vg) + (static_cast<long long>(b) * s.R + r) * vec;
-    for (int c = threadIdx.x; c < vec; c += blockDim.x) dst[c] = __ldg(V + c);
+    const uint4* __restrict__ V = reinterpret_cast<const uint4*>(s.V) + (static_cast<long long>(b) * s.N + src) * vec;
+    uint4* __restrict__ dst = reinterpret_cast<uint4*>(s.Vg) + (static_cast<long long>(b) * s.R + r) * vec;
+    // four 16-byte loads in flight per thread before their stores (V and Vg never overlap)
+    int c = threadIdx.x;
+    constexpr int T = kGatherThreads;
+    for (; c + 3 * T < vec; c += 4 * T) {
+      const uint4 x0 = __ldg(V + c), x1 = __ldg(V + c + T), x2 = __ldg(V + c + 2 * T), x3 = __ldg(V + c + 3 * T);
+      dst[c] = x0;
+      dst[c + T] = x1;
+      dst[c + 2 * T] = x2;
+      dst[c + 3 * T] = x3;
+    }
+    for (; c < vec; c += T) dst[c] = __ldg(V + c);
   }
 }
 
@@ -823,7 +834,7 @@ cudaError_t launch_sel_choose(const SelState& s, cudaStream_t st) {
   cudaError_t e = cudaFuncSetAttribute(sel_choose_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(sm));
   if (e != cudaSuccess) return e;
   if ((e = launch_k(sel_choose_kernel, dim3(s.B), dim3(1024), sm, st, s)) != cudaSuccess) return e;
-  return launch_k(sel_gather_kernel, dim3(kGatherCtas, s.B), dim3(128), 0, st, s);
+  return launch_k(sel_gather_kernel, dim3(kGatherCtas, s.B), dim3(kGatherThreads), 0, st, s);
 }
 
 cudaError_t launch_sel_greedy(const SelState& s, cudaStream_t st) {
@@ -867,7 +878,7 @@ cudaError_t launch_sel_proj_prep(const SelState& s, bool first, cudaStream_t st)
 }
 
 cudaError_t launch_sel_gather(const SelState& s, cudaStream_t st) {
-  return launch_k(sel_gather_kernel, dim3(kGatherCtas, s.B), dim3(128), 0, st, s);
+  return launch_k(sel_gather_kernel, dim3(kGatherCtas, s.B), dim3(kGatherThreads), 0, st, s);
 }
 
 cudaError_t launch_sel_proj_done(const SelState& s, cudaStream_t st) {

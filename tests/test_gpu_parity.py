@@ -243,6 +243,24 @@ def test_assemble_is_bit_exact():
         np.testing.assert_array_equal(pos.cpu().numpy(), p_ref)
 
 
+def test_assemble_many_images_split_over_launches():
+    # image metadata travel as launch parameters, 512 images per launch
+    dims = W.PredictorDims(D=512, Dh=256, dp=64)
+    ctx, _ = make_ctx(dims)
+    rng = np.random.default_rng(8)
+    B, N, K = 1100, 6, 2
+    vis = rng.integers(0, 2 ** 16, size=(B, N, 512), dtype=np.uint16)
+    lens = rng.integers(0, 3, size=B).astype(np.int32)
+    text = rng.integers(0, 2 ** 16, size=(int(lens.sum()), 512), dtype=np.uint16)
+    keep = np.sort(np.stack([rng.choice(N, K, replace=False) for _ in range(B)]), 1).astype(np.int32)
+    seq, pos = ctx.assemble(dev_bits(vis), torch.from_numpy(keep).to(DEV), dev_bits(text), lens, pos_offset=3)
+    torch.cuda.synchronize()
+    ctx.check()
+    s_ref, p_ref = O.assemble(vis, keep, text, lens, 3)
+    np.testing.assert_array_equal(seq.cpu().numpy().view(np.uint16), s_ref)
+    np.testing.assert_array_equal(pos.cpu().numpy(), p_ref)
+
+
 def test_assemble_rejects_bad_index_without_faulting():
     dims = W.PredictorDims(D=512, Dh=256, dp=64)
     ctx, _ = make_ctx(dims)

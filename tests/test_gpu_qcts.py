@@ -87,3 +87,14 @@ def test_qcts_llava_next_full_size(mb):
     out = _run(mb, attn, lens, ref, w.L, w.H, w.N)
     res = Q.qcts_batch(attn, lens, ref, w.L, w.H, w.N)
     _compare(res, *out)
+
+
+def test_qcts_many_layers_split_over_launches(mb):
+    # gridDim.z = samples * L is capped, so 40000 layers run one sample per launch
+    L, H, N = 40000, 1, 16
+    rng = np.random.default_rng(6)
+    lens = np.array([1, 2], np.int32)
+    attn = W.f32_to_bf16_bits(rng.random(L * H * N * 3, dtype=np.float32))
+    ref = W.f32_to_bf16_bits(rng.random((2, L, H, 1, N), dtype=np.float32))
+    out = _run(mb, attn, lens, ref, L, H, N)
+    _compare(Q.qcts_batch(attn, lens, ref, L, H, N), *out)
