@@ -123,6 +123,46 @@ def bench_qcts(mb, dev, stream, steps, hbm, cpu_on, samples=None):
     return res
 
 
+def bench_ragged(mb, dev, stream, steps, bf16_peak, hbm):
+    """Ragged batch (Qwen2.5-VL-style variable resolution): 16 images of 675-1222 tokens in
+    a batch padded to 1280, D = 3584, keep 128, through map_prune_ragged on device buffers."""
+    import torch
+    wr = W.RAGGED_WORKLOADS["c5"]
+    vis_np, text_np, lens, nv = W.make_ragged_batch(wr, threads=min(16, _CORES))
+    dims = W.PredictorDims(D=wr.D)
+    w = W.make_weights(dims)
+    ctx = mb.Context({k: torch.from_numpy(v.view(np.int16)).to(dev) for k, v in w.items()}, dims.D, dims.Dh,
+                     dims.dp)
+    vis = torch.from_numpy(vis_np.view(np.int16)).to(dev)
+    text = torch.from_numpy(text_np.view(np.int16)).to(dev)
+    B, N, K = wr.B, wr.n_max, wr.K
+    out = torch.empty((B, K, wr.D), dtype=torch.int16, device=dev)
+    keep = torch.empty((B, K), dtype=torch.int32, device=dev)
+    sc = torch.empty((B, N), dtype=torch.float32, device=dev)
+    for _ in range(3):
+        ctx.prune_ragged(text, vis, lens, nv, K, out, keep, sc)
+    torch.cuda.synchronize()
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(steps + 1)]
+    evs[0].record(stream)
+    for i in range(steps):
+        ctx.prune_ragged(text, vis, lens, nv, K, out, keep, sc)
+        evs[i + 1].record(stream)
+    torch.cuda.synchronize()
+    ctx.check()
+    ctx.close()
+    ms = np.array([evs[i].elapsed_time(evs[i + 1]) for i in range(steps)])
+    step_s = evs[0].elapsed_time(evs[-1]) / 1000.0 / steps
+    # algorithmic work of the valid tokens only (the padding rows are the layout's overhead)
+    flops = sum(algorithmic(dims, int(nv[b]), K, lens[b:b + 1])[0] for b in range(B))
+    bytes_ = sum(algorithmic(dims, int(nv[b]), K, lens[b:b + 1])[1] for b in range(B))
+    t_roof = max(flops / (bf16_peak * 1e12), bytes_ / (hbm * 1e9))
+    return {"workload": wr.name, "B": B, "n_max": N, "n_valid": [int(x) for x in nv], "D": wr.D, "k": K,
+            "value": B / step_s, "unit": "images/s", "ms_per_batch_p50": float(np.percentile(ms, 50)),
+            "ms_per_batch_p99": float(np.percentile(ms, 99)),
+            "step_roofline": {"algorithmic_gflop_per_image": flops / B / 1e9, "t_roofline_ms": t_roof * 1000,
+                              "frac": t_roof / step_s, "bound": "tensor", "peak_source": "measured bf16 burst"}}
+
+
 def measured_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -511,6 +551,8 @@ def main():
                             "frac": h_bytes / h_s / 1e9 / hbm, "algorithmic_bytes": int(h_bytes)}}
     del seq, pos
 
+    ragged = bench_ragged(mb, dev, stream, 20, bf16_burst, hbm) if rank == 0 else None
+
     qcts = None
     if rank == 0 and not args.no_qcts:
         qcts = bench_qcts(mb, dev, stream, 20, hbm, ws == 1 and not args.no_cpu, args.qcts_samples)
@@ -552,6 +594,7 @@ def main():
             "gpu_launches": int(launches),
             "cpu_baseline": cpu,
             "handoff": handoff,
+            "ragged": ragged,
             "qcts": qcts,
         }
         print(json.dumps(line))

@@ -214,6 +214,35 @@ int map_qcts(const void *attn, const int32_t *lens, const void *attn_ref, int M_
              int L, int H, int N, float *p, float *p_ref, float *js, int32_t *teacher,
              float *teacher_p, void *stream);
 
+/*
+ * Ragged batches (variable-resolution images, e.g. Qwen2.5-VL's dynamic token counts): the
+ * same three steps on a padded layout.  vis_feats is [B, N, D] with N the largest token
+ * count; image b's visual tokens are rows 0 .. n_valid[b]-1 and the rows after them are
+ * padding whose contents are never used.  n_valid int32 [B] is a HOST array with
+ * 1 <= n_valid[b] <= N (MAP_EINVAL otherwise).  Per image, the results equal those of the
+ * unpadded call on its n_valid[b] tokens: Eq. 3's softmax runs over n < n_valid[b] only and
+ * the question follows the image (positions n_valid[b] + m); scores[b, n] = 0 for padding;
+ * the selection never retains padding, so k <= min_b n_valid[b] (MAP_EINVAL otherwise).
+ * Other arguments, limits and buffer rules as for map_score / map_select / map_prune
+ * (map_prune_ragged also accepts host buffers).  The padding rows still pass through the
+ * predictor's GEMMs, so the cost is that of the padded batch.
+ */
+int map_score_ragged(map_ctx *ctx, const void *text_feats, const void *vis_feats,
+                     const int32_t *lens, const int32_t *n_valid, int B, int N, float *scores,
+                     void *stream);
+int map_select_ragged(map_ctx *ctx, const float *scores, const void *vis_feats,
+                      const int32_t *n_valid, int B, int N, int k, int32_t *keep_idx,
+                      int32_t *pick_order, void *stream);
+int map_prune_ragged(map_ctx *ctx, const void *text_feats, const void *vis_feats,
+                     const int32_t *lens, const int32_t *n_valid, int B, int N, int k, void *out,
+                     int32_t *keep_idx, float *scores, void *stream);
+/* map_assemble for a ragged batch: question token m of image b sits at position
+ * n_valid[b] + m (+ pos_offset), and kept indices must lie in [0, n_valid[b]). */
+int map_assemble_ragged(map_ctx *ctx, const void *vis_feats, const int32_t *keep_idx,
+                        const void *text_feats, const int32_t *lens, const int32_t *n_valid,
+                        int B, int N, int k, int pos_offset, void *seq, int32_t *pos_ids,
+                        void *stream);
+
 /* Synchronises `stream` and returns the first deferred device-side error recorded by
  * this context since the last call (MAP_ETIMEOUT, MAP_EINTERNAL), clearing it; else a
  * CUDA error as MAP_ECUDA; else MAP_OK. */

@@ -288,21 +288,25 @@ def gather(vis_bits: np.ndarray, keep: np.ndarray) -> np.ndarray:
     return np.stack([vis_bits[b][np.asarray(keep[b], dtype=np.int64)] for b in range(B)])
 
 
-def assemble(vis_bits: np.ndarray, keep: np.ndarray, text_bits: np.ndarray, lens, pos_offset: int = 0):
+def assemble(vis_bits: np.ndarray, keep: np.ndarray, text_bits: np.ndarray, lens, pos_offset: int = 0,
+             n_valid=None):
     """Hand-off to the language model (section "Inference-Time Token Pruning", last
     paragraph): the kept tokens, restored to their original order, keep their positional
     indices and are combined with the question tokens.  Per image b: its k kept visual
     tokens (keep[b], ascending) at positions keep[b], then its M_b question tokens at
     positions N + m (the question follows the full image), all shifted by pos_offset;
-    images one after another.  Returns (seq [sum_b (k + M_b), D] bf16 bits, pos int32)."""
+    images one after another.  With n_valid (ragged batch: image b has n_valid[b] tokens,
+    the rest of its rows are padding) the question follows the image's own tokens: N_b + m.
+    Returns (seq [sum_b (k + M_b), D] bf16 bits, pos int32)."""
     B, N, _ = vis_bits.shape
     rows, pos = [], []
     o = 0
     for b in range(B):
         M = int(lens[b])
+        Nb = N if n_valid is None else int(n_valid[b])
         rows.append(vis_bits[b][np.asarray(keep[b], dtype=np.int64)])
         rows.append(text_bits[o:o + M])
         pos.append(np.asarray(keep[b], dtype=np.int64) + pos_offset)
-        pos.append(N + np.arange(M) + pos_offset)
+        pos.append(Nb + np.arange(M) + pos_offset)
         o += M
     return np.concatenate(rows, axis=0), np.concatenate(pos).astype(np.int32)

@@ -50,6 +50,14 @@ SIGNATURES = {
                          c_void_p, c_void_p, c_void_p, c_void_p]),
     "map_assemble": (c_int, [c_void_p, c_void_p, c_void_p, c_void_p, POINTER(c_int32), c_int, c_int, c_int, c_int,
                              c_void_p, c_void_p, c_void_p]),
+    "map_score_ragged": (c_int, [c_void_p, c_void_p, c_void_p, POINTER(c_int32), POINTER(c_int32), c_int, c_int,
+                                 c_void_p, c_void_p]),
+    "map_select_ragged": (c_int, [c_void_p, c_void_p, c_void_p, POINTER(c_int32), c_int, c_int, c_int, c_void_p,
+                                  c_void_p, c_void_p]),
+    "map_prune_ragged": (c_int, [c_void_p, c_void_p, c_void_p, POINTER(c_int32), POINTER(c_int32), c_int, c_int,
+                                 c_int, c_void_p, c_void_p, c_void_p, c_void_p]),
+    "map_assemble_ragged": (c_int, [c_void_p, c_void_p, c_void_p, c_void_p, POINTER(c_int32), POINTER(c_int32),
+                                    c_int, c_int, c_int, c_int, c_void_p, c_void_p, c_void_p]),
     "map_prune": (c_int, [c_void_p, c_void_p, c_void_p, POINTER(c_int32), c_int, c_int, c_int, c_void_p,
                           c_void_p, c_void_p, c_void_p]),
     "map_status": (c_int, [c_void_p, c_void_p]),
@@ -200,6 +208,52 @@ class Context:
             pos = torch.empty(rows, dtype=torch.int32, device=vis.device)
         _check(lib.map_assemble(self.h, _ptr(vis), _ptr(keep), _ptr(text), lp, B, N, k, pos_offset, _ptr(seq),
                                 _ptr(pos), _stream(stream)), "map_assemble")
+        return seq, pos
+
+    # -- ragged batches (padded layout, n_valid tokens per image) ---------------------------
+    def score_ragged(self, text, vis, lens, n_valid, scores=None, stream=None):
+        B, N = vis.shape[0], vis.shape[1]
+        if scores is None:
+            scores = torch.empty((B, N), dtype=torch.float32, device=vis.device)
+        arr, lp = _lens(lens)
+        nva, nvp = _lens(n_valid)
+        _check(lib.map_score_ragged(self.h, _ptr(text), _ptr(vis), lp, nvp, B, N, _ptr(scores), _stream(stream)),
+               "map_score_ragged")
+        return scores
+
+    def select_ragged(self, scores, vis, n_valid, k: int, keep=None, order=None, want_order: bool = True,
+                      stream=None):
+        B, N = vis.shape[0], vis.shape[1]
+        if keep is None:
+            keep = torch.empty((B, k), dtype=torch.int32, device=vis.device)
+        if order is None and want_order:
+            order = torch.empty((B, k), dtype=torch.int32, device=vis.device)
+        nva, nvp = _lens(n_valid)
+        _check(lib.map_select_ragged(self.h, _ptr(scores), _ptr(vis), nvp, B, N, k, _ptr(keep), _ptr(order),
+                                     _stream(stream)), "map_select_ragged")
+        return keep, order
+
+    def prune_ragged(self, text, vis, lens, n_valid, k: int, out, keep, scores=None, stream=None):
+        B, N = vis.shape[0], vis.shape[1]
+        arr, lp = _lens(lens)
+        nva, nvp = _lens(n_valid)
+        _check(lib.map_prune_ragged(self.h, _ptr(text), _ptr(vis), lp, nvp, B, N, k, _ptr(out), _ptr(keep),
+                                    _ptr(scores), _stream(stream)), "map_prune_ragged")
+        return out, keep
+
+    def assemble_ragged(self, vis, keep, text, lens, n_valid, pos_offset: int = 0, seq=None, pos=None,
+                        stream=None):
+        B, N, D = vis.shape
+        k = keep.shape[1]
+        arr, lp = _lens(lens)
+        nva, nvp = _lens(n_valid)
+        rows = B * k + int(arr.sum())
+        if seq is None:
+            seq = torch.empty((rows, D), dtype=vis.dtype, device=vis.device)
+        if pos is None:
+            pos = torch.empty(rows, dtype=torch.int32, device=vis.device)
+        _check(lib.map_assemble_ragged(self.h, _ptr(vis), _ptr(keep), _ptr(text), lp, nvp, B, N, k, pos_offset,
+                                       _ptr(seq), _ptr(pos), _stream(stream)), "map_assemble_ragged")
         return seq, pos
 
     def prune(self, text, vis, lens, k: int, out, keep, scores=None, stream=None):

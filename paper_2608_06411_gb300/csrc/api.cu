@@ -39,7 +39,7 @@ struct map_ctx {
   // [hi | hi | lo] of W_Q W_T2 / W_K W_V2 ([dp, 3 Dh]) and fp32 biases W_Q b_T2 / W_K b_V2
   void* wqt = nullptr; void* wkv = nullptr; float* bqt = nullptr; float* bkv = nullptr;
   DevBuf rope;  int rope_rows = 0;
-  DevBuf h1, kb, th1, qb, stats, qoff, post, sqn, pmean;
+  DevBuf h1, kb, th1, qb, stats, qoff, post, sqn, pmean, snv;
   // selection
   DevBuf sU, sr2, scstep, sstate, sEc, spicks, sr0, sbt, srn, ssmall, stheta, saslot, sVg, sG;
   // map_prune staging
@@ -220,10 +220,15 @@ int predictor_branch(map_ctx* c, const void* x, long long rows, const void* w1, 
   return MAP_OK;
 }
 
-int score_impl(map_ctx* c, const void* text, const void* vis, const int32_t* lens, int B, int N, float* scores,
-               float* q_out, float* k_out, cudaStream_t st) {
+// nv (host, B entries, or nullptr = every image has N tokens): valid visual tokens per image;
+// rows at or past nv[b] are padding, excluded from Eq. 3 (their score is 0).
+int score_impl(map_ctx* c, const void* text, const void* vis, const int32_t* lens, const int32_t* nv, int B, int N,
+               float* scores, float* q_out, float* k_out, cudaStream_t st) {
   if (!c || !text || !vis || !lens || !scores) return MAP_EINVAL;
   if (B < 1 || N < 1) return MAP_EINVAL;
+  if (nv)
+    for (int b = 0; b < B; ++b)
+      if (nv[b] < 1 || nv[b] > N) return MAP_EINVAL;
   if (!aligned16(text) || !aligned16(vis)) return MAP_EINVAL;
   long long total_m = 0;
   int max_m = 0;
@@ -239,18 +244,20 @@ int score_impl(map_ctx* c, const void* text, const void* vis, const int32_t* len
   // per-image query offsets, lengths and question-token positions N + m, written on the device
   const size_t off_bytes = static_cast<size_t>(B + 1) * 4, len_bytes = static_cast<size_t>(B) * 4;
   const size_t pos_bytes = static_cast<size_t>(total_m) * 4;
-  MAP_TRY(ensure(c->qoff, off_bytes + len_bytes));
+  MAP_TRY(ensure(c->qoff, off_bytes + 2 * len_bytes));
   MAP_TRY(ensure(c->post, pos_bytes));
   {
     std::vector<long long> offs(B);
     long long acc = 0;
     for (int b = 0; b < B; ++b) { offs[b] = acc; acc += lens[b]; }
     int32_t* qo = static_cast<int32_t*>(c->qoff.p);
-    CU_TRY(mapk::launch_query_meta(lens, offs.data(), B, N, qo, qo + (B + 1), static_cast<int32_t*>(c->post.p), st));
+    CU_TRY(mapk::launch_query_meta(lens, offs.data(), B, N, qo, qo + (B + 1), static_cast<int32_t*>(c->post.p), nv,
+                                   nv ? qo + (2 * B + 1) : nullptr, st));
     c->counters.launches += (B + 1023) / 1024;
   }
   const int* d_off = static_cast<const int*>(c->qoff.p);
   const int* d_len = d_off + (B + 1);
+  const int* d_nv = nv ? d_off + (2 * B + 1) : nullptr;
 
   const long long vrows = static_cast<long long>(B) * N;
   const int dp3 = 3 * g.dp;
@@ -273,6 +280,7 @@ int score_impl(map_ctx* c, const void* text, const void* vis, const int32_t* len
   d.A = c->kb.p; d.a_rows_total = vrows; d.a_row_stride = N;
   d.B = c->qb.p; d.b_rows_total = total_m; d.b_row_stride = 0; d.b_off = d_off;
   d.M = N; d.N = max_m; d.K = dp3; d.batch = B; d.n_limit = d_len; d.col_count = d_len;
+  d.m_limit = d_nv;
   d.status = c->status;
   float* mean_out = scores;
   if (n_tiles > 1) {
@@ -304,10 +312,14 @@ T* carve(char*& p, size_t n) {
   return r;
 }
 
-int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, int K, int32_t* keep,
-                int32_t* order, cudaStream_t st) {
+// nv as for score_impl: tokens at or past nv[b] are never retained (K <= every nv[b]).
+int select_impl(map_ctx* c, const float* scores, const void* vis, const int32_t* nv, int B, int N, int K,
+                int32_t* keep, int32_t* order, cudaStream_t st) {
   if (!c || !scores || !vis) return MAP_EINVAL;
   if (B < 1 || N < 1 || K < 0 || K > N) return MAP_EINVAL;
+  if (nv)
+    for (int b = 0; b < B; ++b)
+      if (nv[b] < 1 || nv[b] > N || K > nv[b]) return MAP_EINVAL;
   if (K == 0) return MAP_OK;
   if (!keep) return MAP_EINVAL;
   if (K > kMaxK || N > kMaxN) return MAP_EUNSUPPORTED;
@@ -331,6 +343,12 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, int B, int N, 
   s.B = B; s.N = N; s.D = g.D; s.K = K; s.K0 = K0; s.S = S; s.R = R; s.KP = KP;
   s.lambda = g.lambda; s.tau = g.tau;
   s.scores = scores; s.V = vis; s.status = c->status;
+  if (nv) {                                      // valid tokens per image, on the device
+    MAP_TRY(ensure(c->snv, static_cast<size_t>(B) * 4));
+    c->counters.launches += (B + 2047) / 2048;
+    CU_TRY(mapk::launch_put_ints(nv, B, static_cast<int32_t*>(c->snv.p), st));
+    s.nvalid = static_cast<const int32_t*>(c->snv.p);
+  }
   // per-token arrays
   MAP_TRY(ensure(c->sqn, BN * 4));
   MAP_TRY(ensure(c->sU, BN * 4));
@@ -502,6 +520,27 @@ int gather_impl(map_ctx* c, const void* vis, const int32_t* keep, int B, int N, 
   return MAP_OK;
 }
 
+int assemble_impl(map_ctx* ctx, const void* vis_feats, const int32_t* keep_idx, const void* text_feats,
+                  const int32_t* lens, const int32_t* nv, int B, int N, int k, int pos_offset, void* seq,
+                  int32_t* pos_ids, cudaStream_t st) {
+  if (!ctx || !vis_feats || !text_feats || !lens) return MAP_EINVAL;
+  if (B < 1 || N < 1 || k < 0 || k > N) return MAP_EINVAL;
+  long long rows = 0;
+  for (int b = 0; b < B; ++b) {
+    if (lens[b] < 0) return MAP_EINVAL;
+    if (nv && (nv[b] < 1 || nv[b] > N || k > nv[b])) return MAP_EINVAL;
+    rows += k + lens[b];
+  }
+  if (rows == 0) return MAP_OK;
+  if (!seq || !pos_ids || (k > 0 && !keep_idx)) return MAP_EINVAL;
+  if (!aligned16(vis_feats) || !aligned16(text_feats) || !aligned16(seq)) return MAP_EINVAL;
+  CU_TRY(cudaSetDevice(ctx->device));
+  ++ctx->counters.launches;
+  CU_TRY(mapk::launch_assemble(vis_feats, keep_idx, text_feats, lens, nv, B, N, k, ctx->cfg.D, pos_offset, seq,
+                               pos_ids, ctx->status, st));
+  return MAP_OK;
+}
+
 bool is_device_ptr(const void* p) {
   cudaPointerAttributes a;
   if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
@@ -598,17 +637,20 @@ int map_init(const map_config* cfg, const map_weights* w, map_ctx** out) {
 
 int map_score(map_ctx* ctx, const void* text_feats, const void* vis_feats, const int32_t* lens, int B, int N,
               float* scores, void* stream) {
-  return score_impl(ctx, text_feats, vis_feats, lens, B, N, scores, nullptr, nullptr, static_cast<cudaStream_t>(stream));
+  return score_impl(ctx, text_feats, vis_feats, lens, nullptr, B, N, scores, nullptr, nullptr,
+                    static_cast<cudaStream_t>(stream));
 }
 
 int map_score_debug(map_ctx* ctx, const void* text_feats, const void* vis_feats, const int32_t* lens, int B, int N,
                     float* scores, float* q_out, float* k_out, void* stream) {
-  return score_impl(ctx, text_feats, vis_feats, lens, B, N, scores, q_out, k_out, static_cast<cudaStream_t>(stream));
+  return score_impl(ctx, text_feats, vis_feats, lens, nullptr, B, N, scores, q_out, k_out,
+                    static_cast<cudaStream_t>(stream));
 }
 
 int map_select(map_ctx* ctx, const float* scores, const void* vis_feats, int B, int N, int k, int32_t* keep_idx,
                int32_t* pick_order, void* stream) {
-  return select_impl(ctx, scores, vis_feats, B, N, k, keep_idx, pick_order, static_cast<cudaStream_t>(stream));
+  return select_impl(ctx, scores, vis_feats, nullptr, B, N, k, keep_idx, pick_order,
+                     static_cast<cudaStream_t>(stream));
 }
 
 int map_gather(map_ctx* ctx, const void* vis_feats, const int32_t* keep_idx, int B, int N, int k, void* out,
@@ -619,27 +661,28 @@ int map_gather(map_ctx* ctx, const void* vis_feats, const int32_t* keep_idx, int
 int map_assemble(map_ctx* ctx, const void* vis_feats, const int32_t* keep_idx, const void* text_feats,
                  const int32_t* lens, int B, int N, int k, int pos_offset, void* seq, int32_t* pos_ids,
                  void* stream) {
-  if (!ctx || !vis_feats || !text_feats || !lens) return MAP_EINVAL;
-  if (B < 1 || N < 1 || k < 0 || k > N) return MAP_EINVAL;
-  long long rows = 0;
-  for (int b = 0; b < B; ++b) {
-    if (lens[b] < 0) return MAP_EINVAL;
-    rows += k + lens[b];
-  }
-  if (rows == 0) return MAP_OK;
-  if (!seq || !pos_ids || (k > 0 && !keep_idx)) return MAP_EINVAL;
-  if (!aligned16(vis_feats) || !aligned16(text_feats) || !aligned16(seq)) return MAP_EINVAL;
-  CU_TRY(cudaSetDevice(ctx->device));
-  ++ctx->counters.launches;
-  CU_TRY(mapk::launch_assemble(vis_feats, keep_idx, text_feats, lens, B, N, k, ctx->cfg.D, pos_offset, seq, pos_ids,
-                               ctx->status, static_cast<cudaStream_t>(stream)));
-  return MAP_OK;
+  return assemble_impl(ctx, vis_feats, keep_idx, text_feats, lens, nullptr, B, N, k, pos_offset, seq, pos_ids,
+                       static_cast<cudaStream_t>(stream));
 }
 
-int map_prune(map_ctx* ctx, const void* text_feats, const void* vis_feats, const int32_t* lens, int B, int N, int k,
-              void* out, int32_t* keep_idx, float* scores, void* stream) {
+int map_assemble_ragged(map_ctx* ctx, const void* vis_feats, const int32_t* keep_idx, const void* text_feats,
+                        const int32_t* lens, const int32_t* n_valid, int B, int N, int k, int pos_offset, void* seq,
+                        int32_t* pos_ids, void* stream) {
+  if (!n_valid) return MAP_EINVAL;
+  return assemble_impl(ctx, vis_feats, keep_idx, text_feats, lens, n_valid, B, N, k, pos_offset, seq, pos_ids,
+                       static_cast<cudaStream_t>(stream));
+}
+
+}  // extern "C"
+
+namespace {
+int prune_impl(map_ctx* ctx, const void* text_feats, const void* vis_feats, const int32_t* lens, const int32_t* nv,
+               int B, int N, int k, void* out, int32_t* keep_idx, float* scores, void* stream) {
   if (!ctx || !text_feats || !vis_feats || !lens || !out || !keep_idx) return MAP_EINVAL;
   if (B < 1 || N < 1 || k < 0 || k > N) return MAP_EINVAL;
+  if (nv)
+    for (int b = 0; b < B; ++b)
+      if (nv[b] < 1 || nv[b] > N || k > nv[b]) return MAP_EINVAL;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   map_ctx* c = ctx;
   CU_TRY(cudaSetDevice(c->device));
@@ -727,8 +770,9 @@ int map_prune(map_ctx* ctx, const void* text_feats, const void* vis_feats, const
     float* spc = sp + static_cast<size_t>(b0) * N;
     int32_t* kpc = kp + static_cast<size_t>(b0) * k;
     void* oc = static_cast<char*>(o) + static_cast<size_t>(b0) * k * D * 2;
-    int rc = score_impl(c, tc, vc, lens + b0, Bc, N, spc, nullptr, nullptr, st);
-    if (rc == MAP_OK) rc = select_impl(c, spc, vc, Bc, N, k, kpc, nullptr, st);
+    const int32_t* nvc = nv ? nv + b0 : nullptr;
+    int rc = score_impl(c, tc, vc, lens + b0, nvc, Bc, N, spc, nullptr, nullptr, st);
+    if (rc == MAP_OK) rc = select_impl(c, spc, vc, nvc, Bc, N, k, kpc, nullptr, st);
     if (rc == MAP_OK) rc = gather_impl(c, vc, kpc, Bc, N, k, oc, st);
     if (rc != MAP_OK) return finish(rc);
     if (host_io) {
@@ -757,6 +801,35 @@ int map_prune(map_ctx* ctx, const void* text_feats, const void* vis_feats, const
   }
   return finish(MAP_OK);
 }
+}  // namespace
+
+extern "C" {
+
+int map_prune(map_ctx* ctx, const void* text_feats, const void* vis_feats, const int32_t* lens, int B, int N, int k,
+              void* out, int32_t* keep_idx, float* scores, void* stream) {
+  return prune_impl(ctx, text_feats, vis_feats, lens, nullptr, B, N, k, out, keep_idx, scores, stream);
+}
+
+int map_prune_ragged(map_ctx* ctx, const void* text_feats, const void* vis_feats, const int32_t* lens,
+                     const int32_t* n_valid, int B, int N, int k, void* out, int32_t* keep_idx, float* scores,
+                     void* stream) {
+  if (!n_valid) return MAP_EINVAL;
+  return prune_impl(ctx, text_feats, vis_feats, lens, n_valid, B, N, k, out, keep_idx, scores, stream);
+}
+
+int map_score_ragged(map_ctx* ctx, const void* text_feats, const void* vis_feats, const int32_t* lens,
+                     const int32_t* n_valid, int B, int N, float* scores, void* stream) {
+  if (!n_valid) return MAP_EINVAL;
+  return score_impl(ctx, text_feats, vis_feats, lens, n_valid, B, N, scores, nullptr, nullptr,
+                    static_cast<cudaStream_t>(stream));
+}
+
+int map_select_ragged(map_ctx* ctx, const float* scores, const void* vis_feats, const int32_t* n_valid, int B, int N,
+                      int k, int32_t* keep_idx, int32_t* pick_order, void* stream) {
+  if (!n_valid) return MAP_EINVAL;
+  return select_impl(ctx, scores, vis_feats, n_valid, B, N, k, keep_idx, pick_order,
+                     static_cast<cudaStream_t>(stream));
+}
 
 int map_status(map_ctx* ctx, void* stream) {
   if (!ctx) return MAP_EINVAL;
@@ -782,7 +855,7 @@ void map_destroy(map_ctx* ctx) {
   for (void* p : {ctx->wqt, ctx->wkv, static_cast<void*>(ctx->bqt), static_cast<void*>(ctx->bkv)})
     if (p) cudaFree(p);
   DevBuf* bufs[] = {&ctx->rope, &ctx->h1, &ctx->kb, &ctx->th1, &ctx->qb, &ctx->stats,
-                    &ctx->qoff, &ctx->post, &ctx->sqn, &ctx->pmean, &ctx->sU, &ctx->sr2, &ctx->scstep, &ctx->sstate,
+                    &ctx->qoff, &ctx->post, &ctx->sqn, &ctx->pmean, &ctx->snv, &ctx->sU, &ctx->sr2, &ctx->scstep, &ctx->sstate,
                     &ctx->sEc, &ctx->spicks, &ctx->sr0, &ctx->sbt, &ctx->srn, &ctx->ssmall, &ctx->stheta,
                     &ctx->saslot, &ctx->sVg, &ctx->sG, &ctx->pvis, &ctx->ptext, &ctx->pout, &ctx->pkeep,
                     &ctx->pscores};

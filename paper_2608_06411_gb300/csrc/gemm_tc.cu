@@ -53,6 +53,7 @@ struct KArgs {
   int split3;
   const float* biasf;
   const int* blist; const int* bcount;
+  const int* m_limit;
 };
 
 __device__ __forceinline__ float gelu_erf(float x) {
@@ -322,7 +323,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       if (!mbar_wait(&tfull[acc], acc_phase, a.status, abort_flag)) break;
       tc_fence_after();
       const int row = c.m_blk * kBM + r_in_tile;
-      const bool row_ok = row < a.M;
+      const bool row_ok = row < (a.m_limit ? min(a.M, __ldg(a.m_limit + c.b)) : a.M);
       const int lim = a.n_limit ? min(a.N, __ldg(a.n_limit + c.b)) : a.N;
       const int col0 = c.n_blk * BN;
       const uint32_t tbase = tmem_base + (static_cast<uint32_t>(lane_grp * 32) << 16) + acc * BN;
@@ -533,9 +534,10 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             }
           }
         }
-        if (row_ok) {
+        if (row < a.M) {   // rows past the image's valid tokens (m_limit) get 0
           float* out = reinterpret_cast<float*>(a.C) + static_cast<long long>(c.b) * a.c_batch_stride;
-          out[static_cast<long long>(c.n_blk) * a.M + row] = acc_p / static_cast<float>(ncol > 0 ? ncol : 1);
+          out[static_cast<long long>(c.n_blk) * a.M + row] =
+              row_ok ? acc_p / static_cast<float>(ncol > 0 ? ncol : 1) : 0.f;
         }
       } else if constexpr (EPI == EPI_PROJECT) {
         // Cholesky coordinates of token `row` on the R0 basis by forward substitution,
@@ -865,6 +867,7 @@ cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t st) {
   ka.b_base = d.b_base; ka.proj = d.proj;
   ka.a_kwrap = d.a_kwrap; ka.biasf = d.biasf; ka.split3 = d.split3;
   ka.blist = d.blist; ka.bcount = d.blist ? d.bcount : nullptr;
+  ka.m_limit = d.m_limit;
   if (d.blist && !d.bcount) return cudaErrorInvalidValue;
   switch (d.epi) {
     case EPI_GELU_BF16:

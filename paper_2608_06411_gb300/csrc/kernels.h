@@ -73,6 +73,9 @@ struct GemmDesc {
   // Batch entries to process (device): blist[0 .. *bcount) instead of 0 .. batch-1, so that a
   // launch over a few active images spreads their tiles over all SMs (grid sized for batch)
   const int* blist = nullptr; const int* bcount = nullptr;
+  // Per-batch number of valid A rows (device) or nullptr: rows at or past it are treated as
+  // absent (EPI_SM_STATS: excluded from the column statistics; EPI_SM_MEAN: output 0)
+  const int* m_limit = nullptr;
 };
 
 // Returns cudaSuccess, or an error for an unsupported shape (cudaErrorInvalidValue).
@@ -89,8 +92,12 @@ cudaError_t launch_fold_weights(const void* Wp, const void* W2, const void* b2, 
 // (no host-to-device copy, so nothing queues behind bulk input copies on the copy engines):
 // off[b] = first query row of image b (off[B] = total), len[b], pos[row] = N + m for the
 // m-th question token of its image.  lens has B entries; offs are their exclusive prefix sums.
+// With nv (host, B entries: valid visual tokens per image) the positions are nv[b] + m and
+// nvalid[b] = nv[b] is written too (nvalid may be nullptr).
 cudaError_t launch_query_meta(const int32_t* lens, const long long* offs, int B, int N, int32_t* off, int32_t* len,
-                              int32_t* pos, cudaStream_t st);
+                              int32_t* pos, const int32_t* nv, int32_t* nvalid, cudaStream_t st);
+// dst[0 .. n) = host[0 .. n), passed as kernel parameters (no copy engine).
+cudaError_t launch_put_ints(const int32_t* host, int n, int32_t* dst, cudaStream_t st);
 // Copies two device ints into host-mapped memory (device aliases of pinned host words).
 cudaError_t launch_flags_to_host(const int32_t* a, const int* b, int32_t* a_host_dev, int* b_host_dev, cudaStream_t st);
 
@@ -110,9 +117,11 @@ cudaError_t launch_gather(const void* V, const int32_t* idx, int B, int N, int k
                           int* status, cudaStream_t st);
 
 // Hand-off sequence per image: the kept rows V[b, idx[b, j]] (j < k), then the image's
-// lens[b] question rows of T (packed in image order); pos = the kept index or N + m, plus
-// pos_offset.  Out-of-range indices are not copied: pos = -1 and ST_BADINDEX in *status.
-cudaError_t launch_assemble(const void* V, const int32_t* idx, const void* T, const int32_t* lens, int B, int N,
-                            int k, int D, int pos_offset, void* seq, int32_t* pos, int* status, cudaStream_t st);
+// lens[b] question rows of T (packed in image order); pos = the kept index or n_b + m, plus
+// pos_offset, with n_b = nv[b] (host; nullptr: N).  Indices outside [0, n_b) are not copied:
+// pos = -1 and ST_BADINDEX in *status.
+cudaError_t launch_assemble(const void* V, const int32_t* idx, const void* T, const int32_t* lens, const int32_t* nv,
+                            int B, int N, int k, int D, int pos_offset, void* seq, int32_t* pos, int* status,
+                            cudaStream_t st);
 
 }  // namespace mapk

@@ -127,29 +127,45 @@ __global__ void fold_weights_kernel(const __nv_bfloat16* __restrict__ Wp, const 
 
 constexpr int kMetaImages = 1024;
 struct MetaChunk {
-  int b0, count, N, last;
+  int b0, count, N, last, has_nv;
   int32_t lens[kMetaImages];
   int32_t offs[kMetaImages];
+  int32_t nv[kMetaImages];       // valid visual tokens per image (has_nv), else N
 };
 
 // One CTA per image of the chunk.
 __global__ void query_meta_kernel(const __grid_constant__ MetaChunk m, int32_t* __restrict__ off,
-                                  int32_t* __restrict__ len, int32_t* __restrict__ pos) {
+                                  int32_t* __restrict__ len, int32_t* __restrict__ pos,
+                                  int32_t* __restrict__ nvalid) {
   pdl_enter();
   const int i = blockIdx.x, b = m.b0 + i;
   const int o = m.offs[i], l = m.lens[i];
+  const int n = m.has_nv ? m.nv[i] : m.N;
   if (threadIdx.x == 0) {
     off[b] = o;
     len[b] = l;
+    if (nvalid) nvalid[b] = n;
     if (m.last && i == m.count - 1) off[b + 1] = o + l;
   }
-  for (int t = threadIdx.x; t < l; t += blockDim.x) pos[o + t] = m.N + t;
+  for (int t = threadIdx.x; t < l; t += blockDim.x) pos[o + t] = n + t;
+}
+
+constexpr int kPutInts = 2048;
+struct IntChunk {
+  int n;
+  int32_t v[kPutInts];
+};
+
+__global__ void put_ints_kernel(const __grid_constant__ IntChunk c, int32_t* __restrict__ dst) {
+  pdl_enter();
+  for (int i = threadIdx.x; i < c.n; i += blockDim.x) dst[i] = c.v[i];
 }
 
 constexpr int kAsmImages = 512;
 struct AssembleChunk {
   int b0, count, N, k, pos_offset;
   int32_t lens[kAsmImages];
+  int32_t nv[kAsmImages];           // valid visual tokens per image (N without padding)
   long long text_row[kAsmImages];   // first question row of each image in text_feats
   long long seq_row[kAsmImages];    // first row of each image's output sequence
 };
@@ -164,11 +180,12 @@ __global__ void assemble_kernel(const __grid_constant__ AssembleChunk m, const u
   const long long b = m.b0 + i;
   if (j >= m.k + m.lens[i]) return;
   const long long r = m.seq_row[i] + j;
+  const int nv = m.nv[i];
   const uint4* src;
   int p;
   if (j < m.k) {
     const int t = __ldg(idx + b * m.k + j);
-    if (t < 0 || t >= m.N) {
+    if (t < 0 || t >= nv) {
       if (threadIdx.x == 0) {
         atomicOr(status, ST_BADINDEX);
         pos[r] = -1;
@@ -179,7 +196,7 @@ __global__ void assemble_kernel(const __grid_constant__ AssembleChunk m, const u
     p = t;
   } else {
     src = T + (m.text_row[i] + (j - m.k)) * vec_per_row;
-    p = m.N + (j - m.k);
+    p = nv + (j - m.k);
   }
   if (threadIdx.x == 0) pos[r] = p + m.pos_offset;
   uint4* d = seq + r * vec_per_row;
@@ -194,26 +211,40 @@ __global__ void flags_to_host_kernel(const int32_t* a, const int* b, volatile in
 
 }  // namespace
 
+cudaError_t launch_put_ints(const int32_t* host, int n, int32_t* dst, cudaStream_t st) {
+  for (int i0 = 0; i0 < n; i0 += kPutInts) {
+    IntChunk c;
+    c.n = n - i0 < kPutInts ? n - i0 : kPutInts;
+    for (int i = 0; i < c.n; ++i) c.v[i] = host[i0 + i];
+    const cudaError_t e = launch_k(put_ints_kernel, dim3(1), dim3(256), 0, st, c, dst + i0);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
 cudaError_t launch_query_meta(const int32_t* lens, const long long* offs, int B, int N, int32_t* off, int32_t* len,
-                              int32_t* pos, cudaStream_t st) {
+                              int32_t* pos, const int32_t* nv, int32_t* nvalid, cudaStream_t st) {
   for (int b0 = 0; b0 < B; b0 += kMetaImages) {
     MetaChunk m;
     m.b0 = b0;
     m.count = B - b0 < kMetaImages ? B - b0 : kMetaImages;
     m.N = N;
     m.last = b0 + m.count == B;
+    m.has_nv = nv != nullptr;
     for (int i = 0; i < m.count; ++i) {
       m.lens[i] = lens[b0 + i];
       m.offs[i] = static_cast<int32_t>(offs[b0 + i]);
+      m.nv[i] = nv ? nv[b0 + i] : N;
     }
-    const cudaError_t e = launch_k(query_meta_kernel, dim3(m.count), dim3(128), 0, st, m, off, len, pos);
+    const cudaError_t e = launch_k(query_meta_kernel, dim3(m.count), dim3(128), 0, st, m, off, len, pos, nvalid);
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;
 }
 
-cudaError_t launch_assemble(const void* V, const int32_t* idx, const void* T, const int32_t* lens, int B, int N,
-                            int k, int D, int pos_offset, void* seq, int32_t* pos, int* status, cudaStream_t st) {
+cudaError_t launch_assemble(const void* V, const int32_t* idx, const void* T, const int32_t* lens, const int32_t* nv,
+                            int B, int N, int k, int D, int pos_offset, void* seq, int32_t* pos, int* status,
+                            cudaStream_t st) {
   if (D % 8 != 0) return cudaErrorInvalidValue;
   long long trow = 0, srow = 0;
   for (int b0 = 0; b0 < B; b0 += kAsmImages) {
@@ -226,6 +257,7 @@ cudaError_t launch_assemble(const void* V, const int32_t* idx, const void* T, co
     int max_rows = 0;
     for (int i = 0; i < m.count; ++i) {
       m.lens[i] = lens[b0 + i];
+      m.nv[i] = nv ? nv[b0 + i] : N;
       m.text_row[i] = trow;
       m.seq_row[i] = srow;
       trow += lens[b0 + i];

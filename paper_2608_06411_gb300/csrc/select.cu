@@ -168,7 +168,16 @@ __global__ void __launch_bounds__(1024) sel_init_kernel(SelState s) {
   const long long base = static_cast<long long>(b) * s.N;
   __shared__ uint32_t hist[256], bc[4];
   __shared__ int cnt;
+  const int nv = s.nvalid ? s.nvalid[b] : s.N;
   for (int i = threadIdx.x; i < s.N; i += blockDim.x) {
+    if (i >= nv) {                       // padding: never a candidate, key below every token's
+      s.U[base + i] = 0.f;
+      s.r2[base + i] = 0.f;
+      s.cstep[base + i] = 0;
+      s.state[base + i] = 2;
+      sh64[i] = 0ull;
+      continue;
+    }
     const float p = s.scores[base + i], sq = s.sqn ? s.sqn[base + i] : 0.f;
     s.U[base + i] = sel_value(p, sq, sq, s.lambda, s.tau);
     s.r2[base + i] = sq;

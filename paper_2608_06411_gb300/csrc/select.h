@@ -19,7 +19,7 @@ struct SelState {
   float* U;                       // [B, N] squared value bound / exact squared value (sel_value)
   float* r2;                      // [B, N] residual^2 as of cstep
   int32_t* cstep;                 // [B, N] basis coordinates cached
-  uint8_t* state;                 // [B, N] 0 candidate, 1 retained
+  uint8_t* state;                 // [B, N] 0 candidate, 1 retained, 2 padding (never a candidate)
   float* Ec;                      // [B, N, KP] cached coordinates e_beta[i]
   int32_t* picks;                 // [B, K] pick order
   int32_t* r0;                    // [B, K] R0 in p_hat order (first K0 used)
@@ -43,6 +43,7 @@ struct SelState {
   // flips bc_par after each producer's consumer.
   int32_t* blist; int32_t* bcount; int bc_par;
   int* status;
+  const int32_t* nvalid;          // [B] valid tokens per image (nullptr: all N); the rest are padding
 };
 
 size_t sel_init_smem(int N, int K0);

@@ -291,3 +291,69 @@ def make_attention_batch(w: AttentionWorkload, B: int | None = None, lens=None, 
     attn = np.concatenate(blocks) if blocks else np.zeros(0, np.uint16)
     ref = np.stack([make_attention(w, b, w.m_ref, True, L, H, N, threads) for b in range(B)])
     return attn, lens, ref
+
+
+# ----------------------------------------------------------------------------- ragged batches
+
+@dataclasses.dataclass(frozen=True)
+class RaggedWorkload:
+    """Variable-resolution images (Qwen2.5-VL-style dynamic token counts) in a padded batch:
+    image b has n_valid[b] tokens on its own rows x cols grid, at most n_max."""
+    name: str
+    config_id: int
+    B: int
+    n_max: int
+    n_lo: int           # smallest token count drawn
+    D: int
+    centroids: int      # per image, on an 8 x 8 block grid over its token grid
+    noise: float
+    m_lo: int
+    m_hi: int
+    K: int
+
+
+RAGGED_WORKLOADS = {
+    # Qwen2.5-VL-7B width (D = 3584), up to 1280 visual tokens per image, keep 128
+    "c5": RaggedWorkload("c5_ragged16_nmax1280_k128", 5, 16, 1280, 640, 3584, 64, 0.3, 16, 128, 128),
+}
+
+
+def make_ragged_image(w: RaggedWorkload, image: int, D: int | None = None):
+    """(bits [n_max, D], n_valid): a rows x cols token grid (rows in [20, 32], n_valid =
+    rows * cols drawn near U[n_lo, n_max]) of clustered features (centroid of the token's
+    block on an 8 x 8 block grid + N(0, noise^2)); the padding rows after n_valid hold
+    unrelated N(0, 5^2) values, which no result may depend on."""
+    D = D or w.D
+    rng = np.random.Generator(np.random.PCG64(1000 * w.config_id + image))
+    rows = int(rng.integers(20, 33))
+    target = int(rng.integers(w.n_lo, w.n_max + 1))
+    cols = max(1, min(target // rows, w.n_max // rows))
+    nv = rows * cols
+    r = np.arange(rows)[:, None] * 8 // rows
+    c = np.arange(cols)[None, :] * 8 // cols
+    cid = (r * 8 + c).reshape(-1) % w.centroids
+    cent = rng.standard_normal((w.centroids, D), dtype=np.float32)
+    x = np.empty((w.n_max, D), dtype=np.float32)
+    x[:nv] = cent[cid] + rng.standard_normal((nv, D), dtype=np.float32) * np.float32(w.noise)
+    x[nv:] = rng.standard_normal((w.n_max - nv, D), dtype=np.float32) * np.float32(5.0)
+    return f32_to_bf16_bits(x), nv
+
+
+def make_ragged_batch(w: RaggedWorkload, B: int | None = None, threads: int = 8, D: int | None = None):
+    """(vis [B, n_max, D] u16, text [sum(lens), D] u16, lens [B] int32, n_valid [B] int32)."""
+    B = B or w.B
+    D = D or w.D
+    rng = np.random.Generator(np.random.PCG64(1000 * w.config_id + 999_999))
+    lens = rng.integers(w.m_lo, w.m_hi + 1, size=B).astype(np.int32)
+    vis = np.empty((B, w.n_max, D), dtype=np.uint16)
+    nv = np.empty(B, dtype=np.int32)
+    texts = [None] * B
+
+    def one(b):
+        vis[b], nv[b] = make_ragged_image(w, b, D)
+        trng = np.random.Generator(np.random.PCG64(1000 * w.config_id + b + 1_000_000))
+        texts[b] = f32_to_bf16_bits(trng.standard_normal((int(lens[b]), D), dtype=np.float32))
+
+    with ThreadPoolExecutor(max_workers=max(1, threads)) as ex:
+        list(ex.map(one, range(B)))
+    return vis, np.concatenate(texts, axis=0), lens, nv

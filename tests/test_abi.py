@@ -92,3 +92,20 @@ def test_assemble_bad_arguments_are_rejected_on_the_host(mb):
     assert lib.map_assemble(f, f, f, f, neg, 1, 8, 2, 0, f, f, None) == mb.MAP_EINVAL
     assert lib.map_assemble(f, f, f, f, lens, 1, 8, 9, 0, f, f, None) == mb.MAP_EINVAL
     assert lib.map_assemble(f, f, f, f, lens, 0, 8, 2, 0, f, f, None) == mb.MAP_EINVAL
+
+
+def test_ragged_bad_arguments_are_rejected_on_the_host(mb):
+    lib = mb.lib
+    lens = (ctypes.c_int32 * 2)(3, 4)
+    nv_ok = (ctypes.c_int32 * 2)(8, 5)
+    nv_big = (ctypes.c_int32 * 2)(9, 5)
+    nv_zero = (ctypes.c_int32 * 2)(8, 0)
+    f = 256
+    assert lib.map_score_ragged(None, f, f, lens, nv_ok, 2, 8, f, None) == mb.MAP_EINVAL
+    assert lib.map_score_ragged(f, f, f, lens, None, 2, 8, f, None) == mb.MAP_EINVAL
+    assert lib.map_select_ragged(f, f, f, None, 2, 8, 2, f, None, None) == mb.MAP_EINVAL
+    assert lib.map_prune_ragged(f, f, f, lens, None, 2, 8, 2, f, f, None, None) == mb.MAP_EINVAL
+    # sizes checked before the context is touched
+    assert lib.map_prune_ragged(f, f, f, lens, nv_big, 2, 8, 2, f, f, None, None) == mb.MAP_EINVAL
+    assert lib.map_prune_ragged(f, f, f, lens, nv_zero, 2, 8, 2, f, f, None, None) == mb.MAP_EINVAL
+    assert lib.map_prune_ragged(f, f, f, lens, nv_ok, 2, 8, 6, f, f, None, None) == mb.MAP_EINVAL

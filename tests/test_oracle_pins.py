@@ -447,6 +447,9 @@ def test_assemble_hand_example():
                                         [8, 9], [12, 13], [200, 201], [300, 301]])
     # kept tokens keep their original positions; question tokens follow the whole image (N + m)
     np.testing.assert_array_equal(pos, [6, 8, 9, 5, 7, 9, 10])
+    # ragged batch: image 1 has 3 valid tokens, so its question starts at position 3
+    _, pos = O.assemble(vis, np.array([[1, 3], [0, 2]]), text, [1, 2], n_valid=[4, 3])
+    np.testing.assert_array_equal(pos, [1, 3, 4, 0, 2, 3, 4])
     # an image without question tokens contributes its kept tokens only; k = 0 leaves the questions
     seq, pos = O.assemble(vis, np.zeros((2, 0), np.int64), text, [3, 0])
     np.testing.assert_array_equal(seq, text)
