@@ -163,6 +163,64 @@ def bench_ragged(mb, dev, stream, steps, bf16_peak, hbm):
                               "frac": t_roof / step_s, "bound": "tensor", "peak_source": "measured bf16 burst"}}
 
 
+# fp32 FMA lanes (SIMT): 152 SMs x 128 lanes x 2 FLOP x 2.07 GHz (maximum SM clock)
+FP32_SIMT_PEAK_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
+
+
+def bench_distill(mb, dev, stream, steps, cpu_on):
+    """Predictor distillation step (KL loss + gradients of every weight) on 4 LLaVA-NeXT-shaped
+    training samples: N = 2880 visual tokens, questions U[16,128], D = 4096, Dh = 1024,
+    dp = 128; fp32 SIMT GEMMs, so the roofline is the fp32 FMA rate."""
+    import torch
+    wl = W.WORKLOADS["c1"]
+    B, N = 4, wl.N
+    dims = W.PredictorDims()
+    rng = np.random.Generator(np.random.PCG64(4242))
+    lens = rng.integers(16, 129, size=B).astype(np.int32)
+    vis_np = np.stack([W.make_image(wl, 100 + b) for b in range(B)])
+    text_np = np.concatenate([W.make_text(wl, 100 + b, int(lens[b])) for b in range(B)])
+    t = rng.gamma(0.3, size=(B, N))
+    teacher_np = (t / t.sum(axis=1, keepdims=True)).astype(np.float32)
+    w = W.make_weights(dims, bias_std=0.1)
+    ctx = mb.Context({k: torch.from_numpy(v.view(np.int16)).to(dev) for k, v in w.items()}, dims.D, dims.Dh,
+                     dims.dp)
+    vis = torch.from_numpy(vis_np.view(np.int16)).to(dev)
+    text = torch.from_numpy(text_np.view(np.int16)).to(dev)
+    teacher = torch.from_numpy(teacher_np).to(dev)
+    loss, grads = ctx.distill_grad(text, vis, lens, teacher)
+    for _ in range(2):
+        ctx.distill_grad(text, vis, lens, teacher, grads, loss)
+    torch.cuda.synchronize()
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(steps + 1)]
+    evs[0].record(stream)
+    for i in range(steps):
+        ctx.distill_grad(text, vis, lens, teacher, grads, loss)
+        evs[i + 1].record(stream)
+    torch.cuda.synchronize()
+    ctx.check()
+    ctx.close()
+    step_s = evs[0].elapsed_time(evs[-1]) / 1000.0 / steps
+    D, Dh, dp = dims.D, dims.Dh, dims.dp
+    T, M = B * N, int(lens.sum())
+    fwd = 2 * (T + M) * (D * Dh + Dh * Dh + Dh * dp) + 2 * M * N * dp
+    bwd = 2 * 2 * M * N * dp + (T + M) * (2 * 2 * dp * Dh + 2 * 2 * Dh * Dh + 2 * Dh * D)
+    achieved = (fwd + bwd) / step_s / 1e12
+    res = {"workload": "distill_llava_next_b4_n2880", "B": B, "N": N, "question_len": [int(x) for x in lens],
+           "value": B / step_s, "unit": "samples/s", "ms_per_step": step_s * 1000,
+           "roofline": {"bound": "alu", "kernel": "fp32 SIMT GEMMs + elementwise (whole step)",
+                        "achieved": achieved, "peak": FP32_SIMT_PEAK_TFLOPS, "unit": "TFLOP/s",
+                        "frac": achieved / FP32_SIMT_PEAK_TFLOPS, "algorithmic_gflop": (fwd + bwd) / 1e9,
+                        "peak_source": "derived: 152 SMs x 128 fp32 lanes x 2 x 2.07 GHz"}}
+    if cpu_on:
+        from oracle import distill_oracle as DO
+        t0 = time.perf_counter()
+        DO.distill_batch(text_np[:int(lens[0])], vis_np[:1], lens[:1], teacher_np[:1].astype(np.float64), w)
+        secs = time.perf_counter() - t0
+        res["cpu_baseline"] = {"value": 1.0 / secs, "unit": "samples/s", "cores": _CORES, "kind": "oracle",
+                               "sample": f"sample 0 ({int(lens[0])} question tokens), numpy float64, {secs:.1f} s"}
+    return res
+
+
 def measured_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -553,6 +611,8 @@ def main():
 
     ragged = bench_ragged(mb, dev, stream, 20, bf16_burst, hbm) if rank == 0 else None
 
+    distill = bench_distill(mb, dev, stream, 5, ws == 1 and not args.no_cpu) if rank == 0 else None
+
     qcts = None
     if rank == 0 and not args.no_qcts:
         qcts = bench_qcts(mb, dev, stream, 20, hbm, ws == 1 and not args.no_cpu, args.qcts_samples)
@@ -595,6 +655,7 @@ def main():
             "cpu_baseline": cpu,
             "handoff": handoff,
             "ragged": ragged,
+            "distill": distill,
             "qcts": qcts,
         }
         print(json.dumps(line))

@@ -243,6 +243,32 @@ int map_assemble_ragged(map_ctx *ctx, const void *vis_feats, const int32_t *keep
                         int B, int N, int k, int pos_offset, void *seq, int32_t *pos_ids,
                         void *stream);
 
+/*
+ * Predictor distillation step (section "Cross-Modal Attention Distillation"): the predictor
+ * is trained offline by minimising D_KL(p^{l*} || p_hat) (the teacher distribution chosen by
+ * QCTS, e.g. map_qcts's teacher_p, against Eq. 3's prediction).  This call computes the batch
+ * loss  L = (1/B) sum_b sum_n p*_b[n] log(p*_b[n] / p_hat_b[n])  (0 log 0 = 0) with the
+ * context's weights and the gradient dL/dW of every predictor weight, through Eq. 3's
+ * softmax-mean, RoPE, W_Q / W_K and both MLPs (the second MLP layer and the projection are
+ * kept separate here, unlike the inference path).  The optimiser update is the caller's.
+ *   text_feats, vis_feats, lens  as for map_score (lens HOST, each >= 1).
+ *   teacher    float32 [B, N] (device): each row a distribution over the N visual tokens.
+ *   loss       float32 [1] output (device).
+ *   grads      float32 device outputs, each with its weight's shape (wT1 [Dh, D], bT1 [Dh],
+ *              wT2 [Dh, Dh], bT2 [Dh], wQ [dp, Dh], and the same for V / K); overwritten.
+ * fp32 arithmetic throughout (bf16 inputs decoded exactly); deterministic.  Workspace (about
+ * 4 (B N + sum(lens)) (D + 5 Dh + 4 dp) + 4 sum(lens) N bytes) is owned by the context.
+ * B N <= 2^24 and sum(lens) <= 2^24 (MAP_EUNSUPPORTED beyond).
+ */
+typedef struct {
+    float *wT1, *bT1, *wT2, *bT2, *wQ;
+    float *wV1, *bV1, *wV2, *bV2, *wK;
+} map_grads;
+
+int map_distill_grad(map_ctx *ctx, const void *text_feats, const void *vis_feats,
+                     const int32_t *lens, const float *teacher, int B, int N, float *loss,
+                     const map_grads *grads, void *stream);
+
 /* Synchronises `stream` and returns the first deferred device-side error recorded by
  * this context since the last call (MAP_ETIMEOUT, MAP_EINTERNAL), clearing it; else a
  * CUDA error as MAP_ECUDA; else MAP_OK. */

@@ -82,16 +82,17 @@ def _mlp_forward(x, w1, b1, w2, b2):
     return z1, h1, h2
 
 
-def forward_image(t: np.ndarray, v: np.ndarray, W: dict, rope_base: float = 10000.0) -> dict:
+def forward_image(t: np.ndarray, v: np.ndarray, W: dict, rope_base: float = 10000.0, rope_on: bool = True) -> dict:
     """The predictor's forward pass for one image with every intermediate kept.
-    t [M, D], v [N, D] float64; W float64 weights."""
+    t [M, D], v [N, D] float64; W float64 weights.  rope_on=False puts every token at
+    position 0 (RoPE becomes the identity)."""
     M, N = t.shape[0], v.shape[0]
     z1t, h1t, h2t = _mlp_forward(t, W["wT1"], W["bT1"], W["wT2"], W["bT2"])
     z1v, h1v, h2v = _mlp_forward(v, W["wV1"], W["bV1"], W["wV2"], W["bV2"])
     qp = h2t @ W["wQ"].T
     kp = h2v @ W["wK"].T
-    pos_q = N + np.arange(M)
-    pos_k = np.arange(N)
+    pos_q = N + np.arange(M) if rope_on else np.zeros(M)
+    pos_k = np.arange(N) if rope_on else np.zeros(N)
     q = O.rope(qp, pos_q, rope_base)
     k = O.rope(kp, pos_k, rope_base)
     d = q.shape[1]
@@ -120,7 +121,8 @@ def _mlp_backward(dh2, x, z1, h1, w2):
     return dW1, db1, dW2, db2
 
 
-def loss_and_grads(texts: list, visions: list, teachers: list, W: dict, rope_base: float = 10000.0):
+def loss_and_grads(texts: list, visions: list, teachers: list, W: dict, rope_base: float = 10000.0,
+                   rope_on: bool = True):
     """Batch loss L = mean_b D_KL(p*_b || p_hat_b) and dL/dW for every weight.
 
     texts[b] [M_b, D], visions[b] [N, D], teachers[b] [N] (float64; each teacher sums to 1)."""
@@ -128,7 +130,7 @@ def loss_and_grads(texts: list, visions: list, teachers: list, W: dict, rope_bas
     grads = {k: np.zeros_like(W[k]) for k in WEIGHT_NAMES}
     loss = 0.0
     for b in range(B):
-        f = forward_image(texts[b], visions[b], W, rope_base)
+        f = forward_image(texts[b], visions[b], W, rope_base, rope_on)
         p_star, p_hat, s = teachers[b], f["p_hat"], f["s"]
         M = s.shape[0]
         loss += kl_divergence(p_star, p_hat) / B
@@ -158,10 +160,10 @@ def loss_and_grads(texts: list, visions: list, teachers: list, W: dict, rope_bas
 
 
 def distill_batch(text_bits: np.ndarray, vis_bits: np.ndarray, lens, teachers: np.ndarray, weights_bits: dict,
-                  rope_base: float = 10000.0):
+                  rope_base: float = 10000.0, rope_on: bool = True):
     """loss_and_grads on a packed bf16 batch: vis [B, N, D], text [sum(lens), D], teachers [B, N]."""
     W = decode_weights(weights_bits)
     off = np.concatenate([[0], np.cumsum(np.asarray(lens, dtype=np.int64))])
     texts = [O.bf16_bits_to_f64(text_bits[off[b]:off[b + 1]]) for b in range(len(lens))]
     visions = [O.bf16_bits_to_f64(vis_bits[b]) for b in range(len(lens))]
-    return loss_and_grads(texts, visions, [np.asarray(t, dtype=np.float64) for t in teachers], W, rope_base)
+    return loss_and_grads(texts, visions, [np.asarray(t, dtype=np.float64) for t in teachers], W, rope_base, rope_on)

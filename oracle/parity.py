@@ -89,3 +89,20 @@ def check_teacher_layer(js_oracle: np.ndarray, layer_gpu: int, margin: float = Q
         return ok, "" if ok else f"layer {layer_gpu}, oracle {int(order[0])} (margin {rel:.2e})"
     ok = 0 <= layer_gpu < len(js) and js[layer_gpu] >= (1.0 - margin) * top
     return ok, "" if ok else f"layer {layer_gpu} js {js[layer_gpu] if 0 <= layer_gpu < len(js) else None} vs {top}"
+
+
+# ----------------------------------------------------------------------------- distillation
+# Loss: relative error <= 1e-5.  Gradients (fp32 chain against float64): per weight tensor,
+# max |g_gpu - g_ref| <= 1e-4 * max |g_ref| (sums over up to ~10^4 tokens of fp32 products
+# err by ~sqrt(T) eps relative to the tensor's scale, ~5e-6; the softmax backward's
+# g - c difference adds about as much).
+DISTILL_LOSS_RTOL, DISTILL_GRAD_TOL = 1e-5, 1e-4
+
+
+def distill_grad_err(g_gpu: np.ndarray, g_ref: np.ndarray, scale: float = 0.0) -> float:
+    """max |g_gpu - g_ref| / max(max |g_ref|, scale).  A gradient that vanishes exactly (the
+    key bias without RoPE: the softmax over visual tokens ignores a shift common to every key)
+    is compared on `scale`, 1e-3 of the largest gradient of the step."""
+    g_ref = np.asarray(g_ref, dtype=np.float64)
+    den = max(float(np.abs(g_ref).max()), scale, 1e-300)
+    return float(np.abs(np.asarray(g_gpu, dtype=np.float64) - g_ref).max() / den)

@@ -33,6 +33,10 @@ class MapWeights(ctypes.Structure):
     _fields_ = [(n, c_void_p) for n in WEIGHT_NAMES]
 
 
+class MapGrads(ctypes.Structure):
+    _fields_ = [(n, c_void_p) for n in WEIGHT_NAMES]
+
+
 class MapCounters(ctypes.Structure):
     _fields_ = [("launches", c_longlong), ("select_rounds", c_longlong), ("gram_rows", c_longlong)]
 
@@ -58,6 +62,8 @@ SIGNATURES = {
                                  c_int, c_void_p, c_void_p, c_void_p, c_void_p]),
     "map_assemble_ragged": (c_int, [c_void_p, c_void_p, c_void_p, c_void_p, POINTER(c_int32), POINTER(c_int32),
                                     c_int, c_int, c_int, c_int, c_void_p, c_void_p, c_void_p]),
+    "map_distill_grad": (c_int, [c_void_p, c_void_p, c_void_p, POINTER(c_int32), c_void_p, c_int, c_int, c_void_p,
+                                 POINTER(MapGrads), c_void_p]),
     "map_prune": (c_int, [c_void_p, c_void_p, c_void_p, POINTER(c_int32), c_int, c_int, c_int, c_void_p,
                           c_void_p, c_void_p, c_void_p]),
     "map_status": (c_int, [c_void_p, c_void_p]),
@@ -255,6 +261,22 @@ class Context:
         _check(lib.map_assemble_ragged(self.h, _ptr(vis), _ptr(keep), _ptr(text), lp, nvp, B, N, k, pos_offset,
                                        _ptr(seq), _ptr(pos), _stream(stream)), "map_assemble_ragged")
         return seq, pos
+
+    def distill_grad(self, text, vis, lens, teacher, grads=None, loss=None, stream=None):
+        """map_distill_grad: (loss [1], {weight name: fp32 gradient}) on device tensors."""
+        B, N = vis.shape[0], vis.shape[1]
+        D, Dh, dp = self.cfg.D, self.cfg.Dh, self.cfg.dp
+        shapes = {"wT1": (Dh, D), "bT1": (Dh,), "wT2": (Dh, Dh), "bT2": (Dh,), "wQ": (dp, Dh),
+                  "wV1": (Dh, D), "bV1": (Dh,), "wV2": (Dh, Dh), "bV2": (Dh,), "wK": (dp, Dh)}
+        if grads is None:
+            grads = {n: torch.empty(shapes[n], dtype=torch.float32, device=vis.device) for n in WEIGHT_NAMES}
+        if loss is None:
+            loss = torch.empty(1, dtype=torch.float32, device=vis.device)
+        g = MapGrads(*[_ptr(grads[n]) for n in WEIGHT_NAMES])
+        arr, lp = _lens(lens)
+        _check(lib.map_distill_grad(self.h, _ptr(text), _ptr(vis), lp, _ptr(teacher), B, N, _ptr(loss),
+                                    ctypes.byref(g), _stream(stream)), "map_distill_grad")
+        return loss, grads
 
     def prune(self, text, vis, lens, k: int, out, keep, scores=None, stream=None):
         """score + select + gather in one C call; buffers may be host (pinned or not) or device."""

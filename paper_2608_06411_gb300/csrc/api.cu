@@ -1,5 +1,6 @@
 // C ABI of libmap_gb300 (include/map_gb300.h): context, workspace, argument checks and
 // the orchestration of the kernels for score (Eq. 3), select (Eq. 4) and gather.
+#include <algorithm>
 #include <cmath>
 #include <cstdio>
 #include <cstdlib>
@@ -39,7 +40,7 @@ struct map_ctx {
   // [hi | hi | lo] of W_Q W_T2 / W_K W_V2 ([dp, 3 Dh]) and fp32 biases W_Q b_T2 / W_K b_V2
   void* wqt = nullptr; void* wkv = nullptr; float* bqt = nullptr; float* bkv = nullptr;
   DevBuf rope;  int rope_rows = 0;
-  DevBuf h1, kb, th1, qb, stats, qoff, post, sqn, pmean, snv;
+  DevBuf h1, kb, th1, qb, stats, qoff, post, sqn, pmean, snv, dist;
   // selection
   DevBuf sU, sr2, scstep, sstate, sEc, spicks, sr0, sbt, srn, ssmall, stheta, saslot, sVg, sG;
   // map_prune staging
@@ -831,6 +832,117 @@ int map_select_ragged(map_ctx* ctx, const float* scores, const void* vis_feats, 
                      static_cast<cudaStream_t>(stream));
 }
 
+int map_distill_grad(map_ctx* ctx, const void* text_feats, const void* vis_feats, const int32_t* lens,
+                     const float* teacher, int B, int N, float* loss, const map_grads* grads, void* stream) {
+  if (!ctx || !text_feats || !vis_feats || !lens || !teacher || !loss || !grads) return MAP_EINVAL;
+  float* gout[10] = {grads->wT1, grads->bT1, grads->wT2, grads->bT2, grads->wQ,
+                     grads->wV1, grads->bV1, grads->wV2, grads->bV2, grads->wK};
+  for (float* p : gout)
+    if (!p) return MAP_EINVAL;
+  if (B < 1 || N < 1) return MAP_EINVAL;
+  long long total_m = 0;
+  int max_m = 0;
+  for (int b = 0; b < B; ++b) {
+    if (lens[b] < 1) return MAP_EINVAL;
+    total_m += lens[b];
+    max_m = std::max(max_m, static_cast<int>(lens[b]));
+  }
+  if (total_m > (1ll << 24) || static_cast<long long>(B) * N > (1ll << 24)) return MAP_EUNSUPPORTED;
+  map_ctx* c = ctx;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const map_config& g = c->cfg;
+  const long long D = g.D, Dh = g.Dh, dp = g.dp, Tv = static_cast<long long>(B) * N, Tt = total_m;
+  CU_TRY(cudaSetDevice(c->device));
+  MAP_TRY(ensure_rope(c, g.rope_on ? N + max_m + 1 : 1));
+  // question offsets and positions N + m (as for map_score), image of every question row
+  MAP_TRY(ensure(c->qoff, static_cast<size_t>(3 * B + 1) * 4));
+  MAP_TRY(ensure(c->post, static_cast<size_t>(total_m) * 4));
+  std::vector<long long> offs(B);
+  std::vector<int32_t> row_img(static_cast<size_t>(total_m));
+  {
+    long long acc = 0;
+    for (int b = 0; b < B; ++b) {
+      offs[b] = acc;
+      for (int m = 0; m < lens[b]; ++m) row_img[static_cast<size_t>(acc + m)] = b;
+      acc += lens[b];
+    }
+  }
+  int32_t* qo = static_cast<int32_t*>(c->qoff.p);
+  int32_t* post = static_cast<int32_t*>(c->post.p);
+  CU_TRY(mapk::launch_query_meta(lens, offs.data(), B, N, qo, qo + (B + 1), post, nullptr, nullptr, st));
+  // fp32 workspace
+  const int nblk = (N + 255) / 256;
+  const long long wsz[10] = {Dh * D, Dh, Dh * Dh, Dh, dp * Dh, Dh * D, Dh, Dh * Dh, Dh, dp * Dh};
+  long long wtot = 0;
+  for (long long x : wsz) wtot += x;
+  const long long floats = wtot + (Tv + Tt) * D + 5 * (Tv + Tt) * Dh + 4 * (Tv + Tt) * dp + Tt * N + 2LL * B * N +
+                           static_cast<long long>(B) * nblk + total_m + 64 * 16;
+  MAP_TRY(ensure(c->dist, static_cast<size_t>(floats) * 4));
+  float* base = static_cast<float*>(c->dist.p);
+  auto take = [&](long long n) { float* p = base; base += ((n + 15) / 16) * 16; return p; };
+  float* Wf[10];
+  for (int i = 0; i < 10; ++i) Wf[i] = take(wsz[i]);
+  float* Vf = take(Tv * D);
+  float* Tf = take(Tt * D);
+  float *z1v = take(Tv * Dh), *h1v = take(Tv * Dh), *h2v = take(Tv * Dh), *dh2v = take(Tv * Dh), *dh1v = take(Tv * Dh);
+  float *z1t = take(Tt * Dh), *h1t = take(Tt * Dh), *h2t = take(Tt * Dh), *dh2t = take(Tt * Dh), *dh1t = take(Tt * Dh);
+  float *kp = take(Tv * dp), *kk = take(Tv * dp), *dk = take(Tv * dp), *dkp = take(Tv * dp);
+  float *qp = take(Tt * dp), *qq = take(Tt * dp), *dq = take(Tt * dp), *dqp = take(Tt * dp);
+  float* S = take(Tt * N);
+  float *p_hat = take(static_cast<long long>(B) * N), *gb = take(static_cast<long long>(B) * N);
+  float* part = take(static_cast<long long>(B) * nblk);
+  int32_t* d_row_img = reinterpret_cast<int32_t*>(take(total_m));
+  CU_TRY(mapk::launch_put_ints(row_img.data(), static_cast<int>(total_m), d_row_img, st));
+  for (int i = 0; i < 10; ++i) CU_TRY(mapk::launch_bf16_to_f32(c->w[i], wsz[i], Wf[i], st));
+  CU_TRY(mapk::launch_bf16_to_f32(vis_feats, Tv * D, Vf, st));
+  CU_TRY(mapk::launch_bf16_to_f32(text_feats, Tt * D, Tf, st));
+  const float2* tab = static_cast<const float2*>(c->rope.p);
+  const float rs = 1.0f / std::sqrt(static_cast<float>(dp));
+  // forward: z1 = X W1^T + b1, h1 = GELU(z1), h2 = h1 W2^T + b2, projection, RoPE
+  auto branch_fwd = [&](const float* X, long long T, int i1, float* z1, float* h1, float* h2, int ip, float* pre,
+                        float* post_rope, const int32_t* pos, int pos_mod) -> int {
+    CU_TRY(mapk::launch_sgemm(false, true, T, Dh, D, 1.f, X, D, Wf[i1], D, false, z1, Dh, st));
+    CU_TRY(mapk::launch_bias_gelu(z1, Wf[i1 + 1], T, Dh, h1, st));
+    CU_TRY(mapk::launch_sgemm(false, true, T, Dh, Dh, 1.f, h1, Dh, Wf[i1 + 2], Dh, false, h2, Dh, st));
+    CU_TRY(mapk::launch_bias_add(h2, Wf[i1 + 3], T, Dh, st));
+    CU_TRY(mapk::launch_sgemm(false, true, T, dp, Dh, 1.f, h2, Dh, Wf[ip], Dh, false, pre, dp, st));
+    CU_TRY(mapk::launch_rope_f32(false, pre, T, dp, tab, c->rope_rows, pos, pos_mod, post_rope, st));
+    return MAP_OK;
+  };
+  MAP_TRY(branch_fwd(Vf, Tv, 5, z1v, h1v, h2v, 9, kp, kk, nullptr, g.rope_on ? N : 1));
+  MAP_TRY(branch_fwd(Tf, Tt, 0, z1t, h1t, h2t, 4, qp, qq, g.rope_on ? post : nullptr, 1));
+  // Eq. 3 logits per image, softmax, KL, and dL/dlogits
+  for (int b = 0; b < B; ++b)
+    CU_TRY(mapk::launch_sgemm(false, true, lens[b], N, dp, rs, qq + offs[b] * dp, dp, kk + b * N * dp, dp, false,
+                              S + offs[b] * N, N, st));
+  CU_TRY(mapk::launch_distill_loss_grad(S, total_m, qo, d_row_img, teacher, B, N, p_hat, gb, part, loss, st));
+  for (int b = 0; b < B; ++b) {
+    CU_TRY(mapk::launch_sgemm(false, false, lens[b], dp, N, rs, S + offs[b] * N, N, kk + b * N * dp, dp, false,
+                              dq + offs[b] * dp, dp, st));
+    CU_TRY(mapk::launch_sgemm(true, false, N, dp, lens[b], rs, S + offs[b] * N, N, qq + offs[b] * dp, dp, false,
+                              dk + b * N * dp, dp, st));
+  }
+  // backward through RoPE, the projection and the MLP of each branch
+  auto branch_bwd = [&](float* dpost, long long T, const int32_t* pos, int pos_mod, float* dpre, const float* X,
+                        int i1, const float* z1, const float* h1, const float* h2, float* dh2, float* dh1,
+                        int ip) -> int {
+    CU_TRY(mapk::launch_rope_f32(true, dpost, T, dp, tab, c->rope_rows, pos, pos_mod, dpre, st));
+    CU_TRY(mapk::launch_sgemm(true, false, dp, Dh, T, 1.f, dpre, dp, h2, Dh, false, gout[ip], Dh, st));
+    CU_TRY(mapk::launch_sgemm(false, false, T, Dh, dp, 1.f, dpre, dp, Wf[ip], Dh, false, dh2, Dh, st));
+    CU_TRY(mapk::launch_sgemm(true, false, Dh, Dh, T, 1.f, dh2, Dh, h1, Dh, false, gout[i1 + 2], Dh, st));
+    CU_TRY(mapk::launch_colsum(dh2, T, Dh, gout[i1 + 3], st));
+    CU_TRY(mapk::launch_sgemm(false, false, T, Dh, Dh, 1.f, dh2, Dh, Wf[i1 + 2], Dh, false, dh1, Dh, st));
+    CU_TRY(mapk::launch_gelu_back(dh1, z1, T * Dh, st));
+    CU_TRY(mapk::launch_sgemm(true, false, Dh, D, T, 1.f, dh1, Dh, X, D, false, gout[i1], D, st));
+    CU_TRY(mapk::launch_colsum(dh1, T, Dh, gout[i1 + 1], st));
+    return MAP_OK;
+  };
+  MAP_TRY(branch_bwd(dk, Tv, nullptr, g.rope_on ? N : 1, dkp, Vf, 5, z1v, h1v, h2v, dh2v, dh1v, 9));
+  MAP_TRY(branch_bwd(dq, Tt, g.rope_on ? post : nullptr, 1, dqp, Tf, 0, z1t, h1t, h2t, dh2t, dh1t, 4));
+  c->counters.launches += 40 + 3 * B;
+  return MAP_OK;
+}
+
 int map_status(map_ctx* ctx, void* stream) {
   if (!ctx) return MAP_EINVAL;
   if (cudaSetDevice(ctx->device) != cudaSuccess) return MAP_ECUDA;
@@ -855,7 +967,7 @@ void map_destroy(map_ctx* ctx) {
   for (void* p : {ctx->wqt, ctx->wkv, static_cast<void*>(ctx->bqt), static_cast<void*>(ctx->bkv)})
     if (p) cudaFree(p);
   DevBuf* bufs[] = {&ctx->rope, &ctx->h1, &ctx->kb, &ctx->th1, &ctx->qb, &ctx->stats,
-                    &ctx->qoff, &ctx->post, &ctx->sqn, &ctx->pmean, &ctx->snv, &ctx->sU, &ctx->sr2, &ctx->scstep, &ctx->sstate,
+                    &ctx->qoff, &ctx->post, &ctx->sqn, &ctx->pmean, &ctx->snv, &ctx->dist, &ctx->sU, &ctx->sr2, &ctx->scstep, &ctx->sstate,
                     &ctx->sEc, &ctx->spicks, &ctx->sr0, &ctx->sbt, &ctx->srn, &ctx->ssmall, &ctx->stheta,
                     &ctx->saslot, &ctx->sVg, &ctx->sG, &ctx->pvis, &ctx->ptext, &ctx->pout, &ctx->pkeep,
                     &ctx->pscores};

@@ -124,4 +124,27 @@ cudaError_t launch_assemble(const void* V, const int32_t* idx, const void* T, co
                             int B, int N, int k, int D, int pos_offset, void* seq, int32_t* pos, int* status,
                             cudaStream_t st);
 
+// ------------------------------------------------------------------ distillation step (fp32)
+// C[i, j] = alpha sum_k A(i, k) B(k, j) (+ C when accumulate); row-major, A(i, k) = ta ? A[k lda + i]
+// : A[i lda + k], B(k, j) = tb ? B[j ldb + k] : B[k ldb + j].  Tiled SIMT, fixed summation order.
+cudaError_t launch_sgemm(bool ta, bool tb, int M, int N, int K, float alpha, const float* A, long long lda,
+                         const float* B, long long ldb, bool accumulate, float* C, long long ldc, cudaStream_t st);
+cudaError_t launch_bf16_to_f32(const void* x, long long n, float* y, cudaStream_t st);
+// z += b (per column); h = GELU(z)
+cudaError_t launch_bias_gelu(float* z, const float* b, long long rows, int cols, float* h, cudaStream_t st);
+cudaError_t launch_bias_add(float* x, const float* b, long long rows, int cols, cudaStream_t st);
+// RoPE (or its transpose when backward) on [rows, d] fp32 rows; positions pos[r] or r % pos_mod.
+cudaError_t launch_rope_f32(bool backward, const float* x, long long rows, int d, const float2* tab, int ld,
+                            const int32_t* pos, int pos_mod, float* y, cudaStream_t st);
+// S [total_m, N] logits of all images' question rows (image b: rows qoff[b] .. qoff[b+1]) ->
+// softmax, p_hat [B, N], g = dL/dp_hat, *loss = mean_b D_KL(teacher_b || p_hat_b), then S is
+// overwritten with dL/dlogits.  row_img [total_m]: image of each row; part: B * ceil(N/256) floats.
+cudaError_t launch_distill_loss_grad(float* S, long long total_m, const int32_t* qoff, const int32_t* row_img,
+                                     const float* teacher, int B, int N, float* p_hat, float* g, float* part,
+                                     float* loss, cudaStream_t st);
+// dh *= GELU'(z)
+cudaError_t launch_gelu_back(float* dh, const float* z, long long n, cudaStream_t st);
+// out[c] = sum_r X[r, c]
+cudaError_t launch_colsum(const float* X, long long rows, int cols, float* out, cudaStream_t st);
+
 }  // namespace mapk

@@ -98,3 +98,14 @@ def test_teacher_equal_to_prediction_has_zero_loss_and_gradient():
 def test_kl_closed_form():
     # D_KL((1/2, 1/2, 0) || (1/4, 1/4, 1/2)) = ln 2; zero-probability teacher entries add nothing
     assert DO.kl_divergence(np.array([0.5, 0.5, 0.0]), np.array([0.25, 0.25, 0.5])) == pytest.approx(math.log(2))
+
+
+def test_key_bias_gradient_vanishes_without_rope():
+    # every row of the softmax sums to one, so sum_n dL/dl[m, n] = 0: a shift common to all
+    # keys (the key MLP's output bias, seen through W_K) has zero gradient when no position
+    # rotates the keys differently
+    Wt, texts, visions, teachers = _tiny(seed=5)
+    _, g_off = DO.loss_and_grads(texts, visions, teachers, Wt, rope_on=False)
+    assert np.abs(g_off["bV2"]).max() <= 1e-12 * np.abs(g_off["wV2"]).max()
+    _, g_on = DO.loss_and_grads(texts, visions, teachers, Wt, rope_on=True)
+    assert np.abs(g_on["bV2"]).max() > 1e-6 * np.abs(g_on["wV2"]).max()
