@@ -576,7 +576,7 @@ def main():
     e2e_s = max_over_ranks(e2e_s, dev)
     e2e_value = B * args.e2e_steps * ws / e2e_s
     ctx.check()
-    # context for the end-to-end figure: this box's plain pinned host -> device copy rate
+    # context for the end-to-end figure: this machine's plain pinned host -> device copy rate
     vis_tmp = torch.empty_like(vis)
     torch.cuda.synchronize()
     t0 = time.perf_counter()

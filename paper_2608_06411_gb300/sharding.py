@@ -2,7 +2,9 @@
 
 Images are independent units of the pruning path, so a batch is split into contiguous
 blocks of images, one block per rank, and nothing is exchanged on the data path.  The
-only collective is the max over ranks of a scalar (elapsed time) for reporting.
+only collective there is the max over ranks of a scalar (elapsed time) for reporting.
+Data-parallel training of the predictor (the distillation step) has a real exchange: the
+gradients of every rank's samples are averaged over all ranks (allreduce_mean_grads).
 """
 from __future__ import annotations
 
@@ -27,3 +29,30 @@ def max_over_ranks(value: float, device=None) -> float:
     t = torch.tensor([float(value)], dtype=torch.float64, device=device)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def allreduce_mean_grads(grads: dict, local_samples: int, loss=None) -> int:
+    """Data-parallel distillation step (the one place where ranks exchange data): each rank
+    holds the loss and gradients of the mean over its own samples (map_distill_grad); after
+    this call every rank holds those of the mean over all ranks' samples.  Each rank's
+    tensors are weighted by its share of the samples, then summed over ranks: one all-reduce
+    per tensor, in a fixed name order, in place.  Returns the total number of samples."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()):
+        return int(local_samples)
+    names = sorted(grads)
+    dev = grads[names[0]].device if names else None
+    n = torch.tensor([float(local_samples)], dtype=torch.float64, device=dev)
+    dist.all_reduce(n, op=dist.ReduceOp.SUM)
+    total = int(n.item())
+    if total == 0:
+        return 0
+    share = float(local_samples) / total
+    for name in names:
+        grads[name].mul_(share)
+        dist.all_reduce(grads[name], op=dist.ReduceOp.SUM)
+    if loss is not None:
+        loss.mul_(share)
+        dist.all_reduce(loss, op=dist.ReduceOp.SUM)
+    return total

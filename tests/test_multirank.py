@@ -50,3 +50,53 @@ def test_two_gloo_ranks_shard_and_reduce():
         got, t = out[r]
         assert got == [(0, 64), (64, 64)]
         assert t == 2.5
+
+
+def _grad_worker(rank, world, port, out):
+    import numpy as np
+    from oracle import distill_oracle as DO
+    from paper_2608_06411_gb300.sharding import allreduce_mean_grads
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    W, texts, visions, teachers = _tiny_problem()
+    first, n = image_range(len(texts), world, rank)           # 3 samples: 2 on rank 0, 1 on rank 1
+    loss, g = DO.loss_and_grads(texts[first:first + n], visions[first:first + n], teachers[first:first + n], W)
+    grads = {k: torch.tensor(v) for k, v in g.items()}
+    lt = torch.tensor([loss], dtype=torch.float64)
+    total = allreduce_mean_grads(grads, n, lt)
+    out[rank] = (total, float(lt.item()), {k: v.numpy() for k, v in grads.items()})
+    dist.barrier()
+    dist.destroy_process_group()
+
+
+def _tiny_problem():
+    import numpy as np
+    rng = np.random.default_rng(21)
+    D, Dh, dp, N = 8, 6, 4, 5
+    W = {"wT1": rng.standard_normal((Dh, D)), "bT1": rng.standard_normal(Dh), "wT2": rng.standard_normal((Dh, Dh)),
+         "bT2": rng.standard_normal(Dh), "wQ": rng.standard_normal((dp, Dh)), "wV1": rng.standard_normal((Dh, D)),
+         "bV1": rng.standard_normal(Dh), "wV2": rng.standard_normal((Dh, Dh)), "bV2": rng.standard_normal(Dh),
+         "wK": rng.standard_normal((dp, Dh))}
+    W = {k: v / 3.0 for k, v in W.items()}
+    texts = [rng.standard_normal((m, D)) for m in (3, 2, 4)]
+    visions = [rng.standard_normal((N, D)) for _ in range(3)]
+    teachers = [t / t.sum() for t in (rng.gamma(1.0, size=N) for _ in range(3))]
+    return W, texts, visions, teachers
+
+
+def test_two_gloo_ranks_average_distillation_gradients():
+    import numpy as np
+    from oracle import distill_oracle as DO
+    world = 2
+    mgr = mp.get_context("spawn").Manager()
+    out = mgr.dict()
+    mp.start_processes(_grad_worker, args=(world, _free_port(), out), nprocs=world, start_method="spawn", join=True)
+    W, texts, visions, teachers = _tiny_problem()
+    loss, g = DO.loss_and_grads(texts, visions, teachers, W)   # the whole batch on one process
+    for r in range(world):
+        total, lr, gr = out[r]
+        assert total == 3
+        assert lr == pytest.approx(loss, rel=1e-12)
+        for k in g:
+            np.testing.assert_allclose(gr[k], g[k], rtol=1e-10, atol=1e-14)
