@@ -121,6 +121,24 @@ def _mlp_backward(dh2, x, z1, h1, w2):
     return dW1, db1, dW2, db2
 
 
+def _softmax_mean_backward(s: np.ndarray, g: np.ndarray) -> np.ndarray:
+    """dL/dl from dL/dp_hat = g, through p_hat = mean_m softmax_n(l[m, :]) (s = the softmax)."""
+    M = s.shape[0]
+    ds = np.broadcast_to(g / M, s.shape)                 # dL/ds
+    return s * (ds - (s * ds).sum(axis=1, keepdims=True))
+
+
+def _logits_backward(dl: np.ndarray, q: np.ndarray, k: np.ndarray):
+    """(dq, dk) through l = q k^T / sqrt(d)."""
+    d = q.shape[1]
+    return dl @ k / math.sqrt(d), dl.T @ q / math.sqrt(d)
+
+
+def _teacher_grad(p_star: np.ndarray, p_hat: np.ndarray, B: int) -> np.ndarray:
+    """dL/dp_hat of L = (1/B) sum_b D_KL(p*_b || p_hat_b)."""
+    return -p_star / (B * p_hat)
+
+
 def loss_and_grads(texts: list, visions: list, teachers: list, W: dict, rope_base: float = 10000.0,
                    rope_on: bool = True):
     """Batch loss L = mean_b D_KL(p*_b || p_hat_b) and dL/dW for every weight.
@@ -132,14 +150,10 @@ def loss_and_grads(texts: list, visions: list, teachers: list, W: dict, rope_bas
     for b in range(B):
         f = forward_image(texts[b], visions[b], W, rope_base, rope_on)
         p_star, p_hat, s = teachers[b], f["p_hat"], f["s"]
-        M = s.shape[0]
         loss += kl_divergence(p_star, p_hat) / B
-        g = -p_star / (B * p_hat)                           # dL/dp_hat
-        ds = np.broadcast_to(g / M, s.shape)                # dL/ds
-        dl = s * (ds - (s * ds).sum(axis=1, keepdims=True))  # softmax backward
-        d = f["q"].shape[1]
-        dq = dl @ f["k"] / math.sqrt(d)
-        dk = dl.T @ f["q"] / math.sqrt(d)
+        g = _teacher_grad(p_star, p_hat, B)
+        dl = _softmax_mean_backward(s, g)
+        dq, dk = _logits_backward(dl, f["q"], f["k"])
         dqp = _rope_backward(dq, f["pos_q"], rope_base)
         dkp = _rope_backward(dk, f["pos_k"], rope_base)
         grads["wQ"] += dqp.T @ f["h2t"]

@@ -1,0 +1,235 @@
+"""Planted-mistake sweep: each test plants one plausible mistake in an oracle (on the CPU,
+by replacing one of its functions for the duration of the test) and requires that at least
+one pin of that oracle then fails.  This shows the pins tie each oracle to the paper rather
+than to itself: a dropped term, a wrong sign, index or axis, or a transposed operand is
+caught.  CPU only."""
+import inspect
+import math
+
+import numpy as np
+import pytest
+
+from oracle import distill_oracle as DO
+from oracle import map_oracle as O
+from oracle import qcts_oracle as Q
+
+import test_distill_pins
+import test_golden
+import test_oracle_pins
+import test_qcts_pins
+
+
+def _some_pin_fails(*modules) -> bool:
+    """Runs the modules' pin functions (every parameter set of a parametrized one) until one
+    raises; True if one did."""
+    for mod in modules:
+        for name, fn in inspect.getmembers(mod, inspect.isfunction):
+            if not name.startswith("test_") or fn.__module__ != mod.__name__:
+                continue
+            marks = [m for m in getattr(fn, "pytestmark", []) if m.name == "parametrize"]
+            if marks:
+                argnames, values = marks[0].args[0], marks[0].args[1]
+                names = [a.strip() for a in argnames.split(",")] if isinstance(argnames, str) else list(argnames)
+                calls = [dict(zip(names, v if len(names) > 1 else (v,))) for v in values]
+            else:
+                if inspect.signature(fn).parameters:
+                    continue                        # needs a fixture: not a pure pin
+                calls = [{}]
+            for kw in calls:
+                try:
+                    fn(**kw)
+                except Exception:
+                    return True
+    return False
+
+
+def test_pins_pass_unmodified():
+    assert not _some_pin_fails(test_oracle_pins, test_golden, test_qcts_pins, test_distill_pins)
+
+
+# ------------------------------------------------------------------ scoring and selection oracle
+
+def _rope_sign_flipped(x, pos, base=10000.0):
+    n, d = x.shape
+    half = d // 2
+    freq = base ** (-2.0 * np.arange(half) / d)
+    ang = np.asarray(pos, dtype=np.float64)[:, None] * freq[None, :]
+    c, s = np.cos(ang), np.sin(ang)
+    x1, x2 = x[:, :half], x[:, half:]
+    return np.concatenate([x1 * c + x2 * s, x2 * c - x1 * s], axis=1)
+
+
+def _rope_adjacent_pairs(x, pos, base=10000.0):
+    n, d = x.shape
+    freq = base ** (-2.0 * np.arange(d // 2) / d)
+    ang = np.asarray(pos, dtype=np.float64)[:, None] * freq[None, :]
+    c, s = np.cos(ang), np.sin(ang)
+    x1, x2 = x[:, 0::2], x[:, 1::2]
+    out = np.empty_like(x)
+    out[:, 0::2] = x1 * c - x2 * s
+    out[:, 1::2] = x2 * c + x1 * s
+    return out
+
+
+def _attention_unscaled(q, k):
+    logits = q @ k.T
+    logits = logits - logits.max(axis=1, keepdims=True)
+    e = np.exp(logits)
+    return (e / e.sum(axis=1, keepdims=True)).mean(axis=0)
+
+
+def _attention_softmax_of_mean(q, k):
+    logits = (q @ k.T).mean(axis=0) / math.sqrt(q.shape[1])
+    e = np.exp(logits - logits.max())
+    return e / e.sum()
+
+
+def _mlp_without_gelu(x, w1, b1, w2, b2):
+    return (x @ w1.T + b1) @ w2.T + b2
+
+
+def _mlp_without_biases(x, w1, b1, w2, b2):
+    return O.gelu(x @ w1.T) @ w2.T
+
+
+def _top_order_ties_high(p):
+    p = np.asarray(p, dtype=np.float64)
+    order = np.argsort(-p[::-1], kind="stable")
+    return (len(p) - 1 - order)
+
+
+def _values_without_diversity(p, rho, lam):
+    return p.astype(np.float64).copy()
+
+
+def _add_without_update(self, j):
+    rj = self.res[j]
+    if not float(rj @ rj) > self.tau * self.sq[j]:
+        return False
+    self.size += 1
+    return True
+
+
+_orig_predict_queries = O.predict_queries
+
+
+def _queries_at_own_positions(text_bits, N, weights, rope_on=True, rope_base=10000.0, pos=None):
+    M = len(text_bits)
+    return _orig_predict_queries(text_bits, N, weights, rope_on, rope_base, np.arange(M) if pos is None else pos)
+
+
+@pytest.mark.parametrize("attr,bad", [
+    ("rope", _rope_sign_flipped),
+    ("rope", _rope_adjacent_pairs),
+    ("predicted_attention", _attention_unscaled),
+    ("predicted_attention", _attention_softmax_of_mean),
+    ("mlp", _mlp_without_gelu),
+    ("mlp", _mlp_without_biases),
+    ("_top_order", _top_order_ties_high),
+    ("_values", _values_without_diversity),
+    ("predict_queries", _queries_at_own_positions),
+])
+def test_scoring_and_selection_mistakes_are_caught(monkeypatch, attr, bad):
+    monkeypatch.setattr(O, attr, bad)
+    assert _some_pin_fails(test_oracle_pins, test_golden)
+
+
+def test_missing_basis_update_is_caught(monkeypatch):
+    monkeypatch.setattr(O._Basis, "add", _add_without_update)
+    assert _some_pin_fails(test_oracle_pins, test_golden)
+
+
+# ------------------------------------------------------------------ QCTS oracle
+
+def _js_without_halves(p, q):
+    p = np.asarray(p, dtype=np.float64)
+    q = np.asarray(q, dtype=np.float64)
+    m = 0.5 * (p + q)
+    return Q._kl(p, m) + Q._kl(q, m)
+
+
+_orig_js = Q.js_divergence
+
+
+def _js_log2(p, q):
+    return _orig_js(p, q) / math.log(2.0)
+
+
+def _aggregate_rows_normalised_first(A):
+    A = np.asarray(A, dtype=np.float64)
+    s = A.sum(axis=-1, keepdims=True)
+    return (A / np.where(s > 0, s, 1.0)).mean(axis=(1, 2))
+
+
+def _aggregate_first_head_only(A):
+    A = np.asarray(A, dtype=np.float64)
+    return A[:, 0].mean(axis=1)
+
+
+def _teacher_argmin(js):
+    return int(np.argmin(np.asarray(js, dtype=np.float64)))
+
+
+def _teacher_ties_high(js):
+    js = np.asarray(js, dtype=np.float64)
+    return int(len(js) - 1 - np.argmax(js[::-1]))
+
+
+@pytest.mark.filterwarnings("ignore::RuntimeWarning")
+@pytest.mark.parametrize("attr,bad", [
+    ("js_divergence", _js_without_halves),
+    ("js_divergence", _js_log2),
+    ("aggregate_attention", _aggregate_rows_normalised_first),
+    ("aggregate_attention", _aggregate_first_head_only),
+    ("select_teacher_layer", _teacher_argmin),
+    ("select_teacher_layer", _teacher_ties_high),
+])
+def test_qcts_mistakes_are_caught(monkeypatch, attr, bad):
+    monkeypatch.setattr(Q, attr, bad)
+    assert _some_pin_fails(test_qcts_pins)
+
+
+# ------------------------------------------------------------------ distillation oracle
+
+def _softmax_back_without_centering(s, g):
+    return s * np.broadcast_to(g / s.shape[0], s.shape)
+
+
+def _logits_back_unscaled_keys(dl, q, k):
+    return dl @ k / math.sqrt(q.shape[1]), dl.T @ q
+
+
+def _teacher_grad_without_batch_mean(p_star, p_hat, B):
+    return -p_star / p_hat
+
+
+def _rope_back_forward_rotation(dy, pos, base):
+    half = dy.shape[1] // 2
+    c, s = DO._rope_angles(pos, dy.shape[1], base)
+    d1, d2 = dy[:, :half], dy[:, half:]
+    return np.concatenate([d1 * c - d2 * s, d2 * c + d1 * s], axis=1)
+
+
+def _gelu_grad_phi_only(x):
+    return 0.5 * (1.0 + np.vectorize(math.erf)(x / math.sqrt(2.0)))
+
+
+_orig_mlp_backward = DO._mlp_backward
+
+
+def _mlp_backward_mean_bias(dh2, x, z1, h1, w2):
+    dW1, db1, dW2, db2 = _orig_mlp_backward(dh2, x, z1, h1, w2)
+    return dW1, db1, dW2, db2 / dh2.shape[0]
+
+
+@pytest.mark.parametrize("attr,bad", [
+    ("_softmax_mean_backward", _softmax_back_without_centering),
+    ("_logits_backward", _logits_back_unscaled_keys),
+    ("_teacher_grad", _teacher_grad_without_batch_mean),
+    ("_rope_backward", _rope_back_forward_rotation),
+    ("_gelu_grad", _gelu_grad_phi_only),
+    ("_mlp_backward", _mlp_backward_mean_bias),
+])
+def test_distillation_mistakes_are_caught(monkeypatch, attr, bad):
+    monkeypatch.setattr(DO, attr, bad)
+    assert _some_pin_fails(test_distill_pins)
