@@ -39,3 +39,30 @@ def test_near_duplicate_images_repeat_crop_zero():
     assert rel < 0.1
     lens = W.make_lens(w)
     assert lens.min() >= 16 and lens.max() <= 256 and len(lens) == 64
+
+
+def test_attention_generator_rows_are_partial_distributions():
+    w = W.AttentionWorkload("t", 80, 2, 6, 3, 2, 12, 4, 9, 5)
+    a = W.bf16_bits_to_f32(W.make_attention(w, 0, 7)).astype(np.float64)
+    assert a.shape == (6, 3, 7, w.N) and np.all(a >= 0)
+    rows = a.sum(axis=-1)
+    assert rows.min() > 0.04 and rows.max() < 0.51          # visual share U(0.05, 0.5), bf16-rounded
+    np.testing.assert_array_equal(W.make_attention(w, 0, 7), W.make_attention(w, 0, 7, threads=1))
+    assert not np.array_equal(W.make_attention(w, 0, 7), W.make_attention(w, 1, 7))
+    attn, lens, ref = W.make_attention_batch(w)
+    assert attn.size == w.L * w.H * w.N * int(lens.sum()) and ref.shape == (2, 6, 3, 5, w.N)
+    assert lens.min() >= 4 and lens.max() <= 9
+
+
+def test_ragged_generator_shapes_and_padding():
+    w = W.RaggedWorkload("t", 81, 5, 300, 100, 64, 16, 0.3, 2, 9, 10)
+    vis, text, lens, nv = W.make_ragged_batch(w)
+    assert vis.shape == (5, 300, 64) and text.shape == (int(lens.sum()), 64)
+    assert np.all(nv >= 20) and np.all(nv <= 300)
+    v = W.bf16_bits_to_f32(vis).astype(np.float64)
+    for b in range(5):
+        # clustered tokens have norms near sqrt(D) (centroid N(0,1) + noise); padding N(0, 5^2) is far larger
+        assert np.linalg.norm(v[b, :nv[b]], axis=1).mean() < 12
+        if nv[b] < 300:
+            assert np.linalg.norm(v[b, nv[b]:], axis=1).mean() > 30
+    np.testing.assert_array_equal(W.make_ragged_batch(w)[0], vis)
