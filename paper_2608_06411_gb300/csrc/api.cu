@@ -939,7 +939,9 @@ int map_distill_grad(map_ctx* ctx, const void* text_feats, const void* vis_feats
   };
   MAP_TRY(branch_bwd(dk, Tv, nullptr, g.rope_on ? N : 1, dkp, Vf, 5, z1v, h1v, h2v, dh2v, dh1v, 9));
   MAP_TRY(branch_bwd(dq, Tt, g.rope_on ? post : nullptr, 1, dqp, Tf, 0, z1t, h1t, h2t, dh2t, dh1t, 4));
-  c->counters.launches += 40 + 3 * B;
+  // query metadata, question-row images, 12 conversions, 2 x 6 forward, B logits, 4 loss /
+  // softmax-backward kernels, 2B logits backward, 2 x 9 branch backward
+  c->counters.launches += (B + 1023) / 1024 + (total_m + 2047) / 2048 + 12 + 12 + 3LL * B + 4 + 18;
   return MAP_OK;
 }
 
