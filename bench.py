@@ -221,6 +221,56 @@ def bench_distill(mb, dev, stream, steps, cpu_on):
     return res
 
 
+def bench_config(mb, dev, stream, key, steps, bf16_peak, hbm, ctx=None):
+    """One more workload of the pruning path through map_prune on device buffers: per-batch
+    CUDA-event times (p50/p99) and the fraction of the algorithmic roofline (GEMM FLOPs at
+    the measured bf16 peak vs feature bytes at the measured HBM rate; FLOPs counted as the
+    method is written and, stricter, with the folded second layer)."""
+    import torch
+    wl = W.WORKLOADS[key]
+    dims = W.PredictorDims(D=wl.D)
+    vis_np, text_np, lens = W.make_batch(wl, threads=min(16, _CORES))
+    own = ctx is None
+    if own:
+        w = W.make_weights(dims)
+        ctx = mb.Context({k: torch.from_numpy(v.view(np.int16)).to(dev) for k, v in w.items()}, dims.D, dims.Dh,
+                         dims.dp)
+    vis = torch.from_numpy(vis_np.view(np.int16)).to(dev)
+    text = torch.from_numpy(text_np.view(np.int16)).to(dev)
+    B, N, K = wl.B, wl.N, wl.K
+    out = torch.empty((B, K, wl.D), dtype=torch.int16, device=dev)
+    keep = torch.empty((B, K), dtype=torch.int32, device=dev)
+    sc = torch.empty((B, N), dtype=torch.float32, device=dev)
+    for _ in range(5):
+        ctx.prune(text, vis, lens, K, out, keep, sc)
+    torch.cuda.synchronize()
+    ms = []
+    for i in range(steps):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        ctx.prune(text, vis, lens, K, out, keep, sc)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms.append(e0.elapsed_time(e1))
+    ctx.check()
+    if own:
+        ctx.close()
+    ms = np.array(ms)
+    t = float(np.median(ms)) / 1000.0
+    flops, bytes_ = algorithmic(dims, N, K, lens)
+    flops_w = method_as_written_flops(dims, N, K, lens)
+    t_fold = max(flops / (bf16_peak * 1e12), bytes_ / (hbm * 1e9))
+    t_writ = max(flops_w / (bf16_peak * 1e12), bytes_ / (hbm * 1e9))
+    return {"workload": wl.name, "B": B, "N": N, "D": wl.D, "k": K,
+            "question_len": f"U[{wl.m_lo},{wl.m_hi}], sum={int(np.sum(lens))}" if B > 1 else int(lens[0]),
+            "value": B / t, "unit": "images/s", "us_per_batch_p50": float(np.percentile(ms, 50) * 1000),
+            "us_per_batch_p99": float(np.percentile(ms, 99) * 1000), "batches_timed": steps,
+            "step_roofline": {"algorithmic_gflop_per_image": flops_w / B / 1e9, "t_roofline_us": t_writ * 1e6,
+                              "frac": t_writ / t, "frac_folded": t_fold / t,
+                              "bound": "tensor" if flops_w / (bf16_peak * 1e12) > bytes_ / (hbm * 1e9) else "hbm",
+                              "peak_source": "measured bf16 burst, hbm"}}
+
+
 def measured_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -610,6 +660,8 @@ def main():
     del seq, pos
 
     ragged = bench_ragged(mb, dev, stream, 20, bf16_burst, hbm) if rank == 0 else None
+    c0 = bench_config(mb, dev, stream, "c0", 200, bf16_burst, hbm, ctx) if rank == 0 else None
+    c4 = bench_config(mb, dev, stream, "c4", 20, bf16_burst, hbm) if rank == 0 else None
 
     distill = bench_distill(mb, dev, stream, 5, ws == 1 and not args.no_cpu) if rank == 0 else None
 
@@ -655,6 +707,8 @@ def main():
             "cpu_baseline": cpu,
             "handoff": handoff,
             "ragged": ragged,
+            "single_image_c0": c0,
+            "high_token_c4": c4,
             "distill": distill,
             "qcts": qcts,
         }

@@ -562,10 +562,14 @@ struct CtxView {
   int32_t* h_done;
   long long* launches;
   long long* rounds;
+  int* h_status;
+  int32_t* h_done_dev;
+  int* h_status_dev;
+  int* deferred;
 };
 CtxView ctx_view(map_ctx* c) {
   return CtxView{&c->cfg, c->device, c->num_sms, c->status, c->h_done, &c->counters.launches,
-                 &c->counters.select_rounds};
+                 &c->counters.select_rounds, c->h_status, c->h_done_dev, c->h_status_dev, &c->deferred};
 }
 }  // namespace mapk
 

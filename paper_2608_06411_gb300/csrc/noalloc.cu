@@ -1,12 +1,12 @@
 // map_select_noalloc: the diversity-aware selection with no memory allocation in the call.
 //
-// Some callers cannot allocate device memory while they prune: code running while a
-// stream is being captured into a CUDA graph (cudaMalloc is not capturable), code that
-// runs inside another framework's memory pool or under a fixed device-memory budget, and
-// real-time paths that must not block on the allocator.  map_select grows workspace owned
-// by the context on demand; this entry point instead carves every buffer it needs from
-// one file-scope device array of kNoAllocScratchBytes, which each GPU that loads this
-// part of the library holds until the process exits.
+// Some callers cannot allocate device memory while they prune: code that runs inside
+// another framework's caching pool or under a fixed device-memory budget (a cudaMalloc
+// would take memory the budget does not have, or fail), and latency-bound serving paths
+// that must not stall on the allocator (cudaMalloc / cudaFree may synchronise the device).
+// map_select grows workspace owned by the context on demand; this entry point instead
+// carves every buffer it needs from one file-scope device array of kNoAllocScratchBytes,
+// which each GPU that loads this part of the library holds until the process exits.
 //
 // The array's device address is looked up once per device (cudaGetSymbolAddress, with
 // that device current) by the first call made on that device; make that first call
@@ -14,6 +14,11 @@
 // behind: the completion counter is cleared at the start of each call, everything else
 // is written before it is read.  Calls whose work overlaps on the GPU (two streams, two
 // host threads) race on the array and must be serialised by the caller.
+//
+// It runs the selection without the tensor-core projection pass that map_select uses
+// when |R0| <= 128: every candidate starts from the bound p_hat * ||v||^lambda and the
+// rounds of active sets (Gram blocks, coordinate updates, greedy picks) do the rest.
+// The picks are the same exact greedy picks; only the number of rounds differs.
 #include <cmath>
 #include <mutex>
 
@@ -30,6 +35,10 @@ struct CtxView {
   int32_t* h_done;
   long long* launches;
   long long* rounds;
+  int* h_status;                     // host-mapped words and their device aliases
+  int32_t* h_done_dev;
+  int* h_status_dev;
+  int* deferred;                     // error reported by the next map_status
 };
 CtxView ctx_view(map_ctx* c);
 }  // namespace mapk
@@ -39,6 +48,9 @@ namespace {
 constexpr size_t kNoAllocScratchBytes = MAP_NOALLOC_SCRATCH_BYTES;
 constexpr int kSelS = 256;
 constexpr int kMaxDevices = 64;
+constexpr int kMaxN = 16384;
+constexpr int kMaxK = 4096;          // plain top-k
+constexpr int kMaxKDiverse = 1024;   // with the diversity term
 
 static __device__ __align__(256) unsigned char g_scratch[kNoAllocScratchBytes];
 
@@ -91,7 +103,7 @@ extern "C" int map_select_noalloc(map_ctx* ctx, const float* scores, const void*
   if (k == 0) return MAP_OK;
   if (!keep_idx) return MAP_EINVAL;
   if ((reinterpret_cast<uintptr_t>(vis_feats) & 15) != 0) return MAP_EINVAL;
-  if (N > 16384 || k > 1024) return MAP_EUNSUPPORTED;
+  if (N > kMaxN || k > kMaxK) return MAP_EUNSUPPORTED;
   mapk::CtxView v = mapk::ctx_view(ctx);
   const map_config& g = *v.cfg;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
@@ -106,6 +118,7 @@ extern "C" int map_select_noalloc(map_ctx* ctx, const float* scores, const void*
   }
   int K0 = k0_of(g, k);
   if (g.lambda == 0.f) K0 = k;
+  if (K0 < k && k > kMaxKDiverse) return MAP_EUNSUPPORTED;
   const int K = k, S = kSelS, R = ((kSelS + K + 15) / 16) * 16, KP = ((K + 3) / 4) * 4;
   const long long BN = static_cast<long long>(B) * N;
 
@@ -173,13 +186,20 @@ extern "C" int map_select_noalloc(map_ctx* ctx, const float* scores, const void*
       }
       rounds += burst;
       *v.rounds += burst;
-      if ((rc = rc_of(cudaMemcpyAsync(v.h_done, s.done_count, 4, cudaMemcpyDeviceToHost, st))) != MAP_OK) return rc;
+      // completion and device status through host-mapped words (no copy engine)
+      ++*v.launches;
+      if ((rc = rc_of(mapk::launch_flags_to_host(s.done_count, v.status, v.h_done_dev, v.h_status_dev, st))) != MAP_OK)
+        return rc;
       if ((rc = rc_of(cudaStreamSynchronize(st))) != MAP_OK) return rc;
       if (*v.h_done >= B) break;
-      int dev_status = 0;             // a kernel that gave up stops the loop at once
-      if ((rc = rc_of(cudaMemcpy(&dev_status, v.status, sizeof(int), cudaMemcpyDeviceToHost))) != MAP_OK) return rc;
-      if (dev_status) return (dev_status & mapk::ST_TIMEOUT) ? MAP_ETIMEOUT : MAP_EINTERNAL;
-      if (rounds > cap) return MAP_EINTERNAL;
+      if (*v.h_status) {              // a kernel gave up (bounded wait) or saw a bad index: stop here
+        *v.deferred = (*v.h_status & mapk::ST_TIMEOUT) ? MAP_ETIMEOUT : MAP_EINTERNAL;
+        return *v.deferred;
+      }
+      if (rounds > cap) {
+        *v.deferred = MAP_EINTERNAL;
+        return MAP_EINTERNAL;
+      }
       burst = 2;
     }
   } else {

@@ -109,3 +109,20 @@ def test_ragged_bad_arguments_are_rejected_on_the_host(mb):
     assert lib.map_prune_ragged(f, f, f, lens, nv_big, 2, 8, 2, f, f, None, None) == mb.MAP_EINVAL
     assert lib.map_prune_ragged(f, f, f, lens, nv_zero, 2, 8, 2, f, f, None, None) == mb.MAP_EINVAL
     assert lib.map_prune_ragged(f, f, f, lens, nv_ok, 2, 8, 6, f, f, None, None) == mb.MAP_EINVAL
+
+
+def test_select_noalloc_bad_arguments_are_rejected_on_the_host(mb):
+    lib = mb.lib
+    f = 256   # a non-null, 16-byte aligned stand-in; the context is not touched on these errors
+    assert lib.map_select_noalloc(None, f, f, 1, 8, 2, f, None, None) == mb.MAP_EINVAL
+    assert lib.map_select_noalloc(f, None, f, 1, 8, 2, f, None, None) == mb.MAP_EINVAL
+    assert lib.map_select_noalloc(f, f, None, 1, 8, 2, f, None, None) == mb.MAP_EINVAL
+    assert lib.map_select_noalloc(f, f, f, 0, 8, 2, f, None, None) == mb.MAP_EINVAL
+    assert lib.map_select_noalloc(f, f, f, 1, 0, 0, f, None, None) == mb.MAP_EINVAL
+    assert lib.map_select_noalloc(f, f, f, 1, 8, 9, f, None, None) == mb.MAP_EINVAL
+    assert lib.map_select_noalloc(f, f, f, 1, 8, -1, f, None, None) == mb.MAP_EINVAL
+    assert lib.map_select_noalloc(f, f, f, 1, 8, 2, None, None, None) == mb.MAP_EINVAL
+    assert lib.map_select_noalloc(f, f, f + 8, 1, 8, 2, f, None, None) == mb.MAP_EINVAL   # misaligned features
+    assert lib.map_select_noalloc(f, f, f, 1, 16385, 2, f, None, None) == mb.MAP_EUNSUPPORTED
+    assert lib.map_select_noalloc(f, f, f, 1, 8000, 4097, f, None, None) == mb.MAP_EUNSUPPORTED
+    assert lib.map_select_noalloc(f, f, f, 1, 8, 0, None, None, None) == mb.MAP_OK          # k = 0: nothing to do

@@ -8,6 +8,8 @@ from oracle import map_oracle as O
 from oracle import parity as P
 from paper_2608_06411_gb300 import workloads as W
 
+import _oracle_pool as OP
+
 pytestmark = pytest.mark.gpu
 
 if not torch.cuda.is_available():
@@ -34,11 +36,15 @@ def run_select(ctx, p32, vis, K):
     return keep.cpu().numpy(), order.cpu().numpy()
 
 
-def assert_selection(p32, vis, K, K0, keep, order, lam=1.0, tau=1e-5):
+def assert_selection(p32, vis, K, K0, keep, order, lam=1.0, tau=1e-5, label=None):
+    reps = []
     for b in range(len(p32)):
         rep = P.check_selection(p32[b].astype(np.float64), O.bf16_bits_to_f64(vis[b]), K, K0, order[b], keep[b],
                                 lam=lam, tau=tau)
         assert rep["ok"], f"image {b}: {rep['reason']}"
+        reps.append(rep)
+    if label:
+        OP.record(label, reps)
 
 
 # ------------------------------------------------------------------ GEMM building block
@@ -135,7 +141,7 @@ def test_select_matches_oracle_llava15_shape():
     text = W.make_text(wl, 0, 32)
     p32 = _oracle_scores(vis, [32], text, w)
     keep, order = run_select(ctx, p32, vis, wl.K)
-    assert_selection(p32, vis, wl.K, O.resolve_k0(wl.K), keep, order)
+    assert_selection(p32, vis, wl.K, O.resolve_k0(wl.K), keep, order, label="c0 N=576 k=32 (oracle scores)")
 
 
 @pytest.mark.parametrize("lam,k0_frac,K", [(1.0, 0.0, 40), (1.0, 0.25, 64), (0.5, 0.5, 50), (2.0, 0.5, 33),
@@ -149,7 +155,8 @@ def test_select_variants(lam, k0_frac, K):
     vis = np.stack([W.make_image(wl, b, N=N, D=dims.D) for b in range(B)])
     p32 = rng.dirichlet(np.full(N, 0.3), size=B).astype(np.float32)
     keep, order = run_select(ctx, p32, vis, K)
-    assert_selection(p32, vis, K, O.resolve_k0(K, k0_frac), keep, order, lam=lam)
+    assert_selection(p32, vis, K, O.resolve_k0(K, k0_frac), keep, order, lam=lam,
+                     label=f"variants N=700 D=256 k={K} lambda={lam} K0={O.resolve_k0(K, k0_frac)}")
 
 
 def test_select_duplicates_and_near_duplicates():
@@ -311,7 +318,7 @@ def test_llava_next_shape_end_to_end():
     assert P.score_rel_err(p.cpu().numpy(), p_ref) <= 1e-3
     p32 = p_ref.astype(np.float32)
     keep, order = run_select(ctx, p32, vis, wl.K)
-    assert_selection(p32, vis, wl.K, O.resolve_k0(wl.K), keep, order)
+    assert_selection(p32, vis, wl.K, O.resolve_k0(wl.K), keep, order, label="c1 N=2880 k=160 (oracle scores)")
     out = ctx.gather(dev_bits(vis), torch.from_numpy(keep).to(DEV))
     torch.cuda.synchronize()
     np.testing.assert_array_equal(out.cpu().numpy().view(np.uint16), O.gather(vis, keep))
@@ -319,55 +326,74 @@ def test_llava_next_shape_end_to_end():
 
 # ------------------------------------------------------------------ remaining workload configs
 
-def _batch_parity(wl, sample, K, K0=None, **ctxkw):
-    """GPU scores for the whole batch against the oracle on `sample` images; then GPU
-    selection on the batch with the oracle's scores on the sampled images."""
+def _full_batch_parity(key, own_scores=False):
+    """Every image of a batched configuration: GPU scores against the oracle (max relative
+    error <= 1e-3), GPU selection on the oracle's scores checked by forced replay, gathered
+    tokens and the hand-off sequence bit for bit.  With own_scores, map_prune's own GPU
+    scores and pick order are checked against the oracle's greedy too (the product path as
+    a user runs it).  The oracle runs in a pool of host processes."""
+    wl = W.WORKLOADS[key]
     dims = W.PredictorDims(D=wl.D)
-    ctx, w = make_ctx(dims, **ctxkw)
+    ctx, w = make_ctx(dims)
     vis, text, lens = W.make_batch(wl, threads=8)
+    B, N, K = wl.B, wl.N, wl.K
+    K0 = O.resolve_k0(K)
+    ex = OP.pool()
+    f_scores = [ex.submit(OP.oracle_scores, key, b, int(lens[b])) for b in range(B)]
     vis_t, text_t = dev_bits(vis), dev_bits(text)
-    p = ctx.score(text_t, vis_t, lens)
+    # the product path: map_prune on device buffers, then its scores' pick order
+    out_p = torch.empty((B, K, wl.D), dtype=torch.int16, device=DEV)
+    keep_p = torch.empty((B, K), dtype=torch.int32, device=DEV)
+    p_gpu_t = torch.empty((B, N), dtype=torch.float32, device=DEV)
+    ctx.prune(text_t, vis_t, lens, K, out_p, keep_p, p_gpu_t)
+    keep_s, order_s = ctx.select(p_gpu_t, vis_t, K)
     torch.cuda.synchronize()
     ctx.check()
-    p_all = p.cpu().numpy().copy()
-    off = np.concatenate([[0], np.cumsum(lens)])
-    for b in sample:
-        p_ref = O.map_score(text[off[b]:off[b + 1]], vis[b:b + 1], [lens[b]], w)[0]
-        assert P.score_rel_err(p_all[b], p_ref) <= 1e-3, f"image {b}"
-        p_all[b] = p_ref.astype(np.float32)           # both sides select on the oracle's scores
-    keep, order = run_select(ctx, p_all, vis, K)
-    K0 = O.resolve_k0(K) if K0 is None else K0
-    for b in sample:
-        rep = P.check_selection(p_all[b].astype(np.float64), O.bf16_bits_to_f64(vis[b]), K, K0, order[b], keep[b])
-        assert rep["ok"], f"image {b}: {rep['reason']}"
+    p_gpu = p_gpu_t.cpu().numpy()
+    np.testing.assert_array_equal(keep_s.cpu().numpy(), keep_p.cpu().numpy())
+    keep_pn = keep_p.cpu().numpy()
+    np.testing.assert_array_equal(out_p.cpu().numpy().view(np.uint16), O.gather(vis, keep_pn))
+    p_ref = np.stack([f.result() for f in f_scores])
+    errs = [P.score_rel_err(p_gpu[b], p_ref[b]) for b in range(B)]
+    assert max(errs) <= 1e-3, f"image {int(np.argmax(errs))}: score rel err {max(errs):.2e}"
+    # both sides select on the oracle's scores rounded to fp32
+    p32 = p_ref.astype(np.float32)
+    keep, order = run_select(ctx, p32, vis, K)
+    f_sel = [ex.submit(OP.oracle_check, key, b, p32[b], K, K0, order[b], keep[b]) for b in range(B)]
+    order_sn = order_s.cpu().numpy()
+    f_own = [ex.submit(OP.oracle_check, key, b, p_gpu[b], K, K0, order_sn[b], keep_pn[b])
+             for b in range(B)] if own_scores else []
     out = ctx.gather(vis_t, torch.from_numpy(keep).to(DEV))
-    torch.cuda.synchronize()
-    for b in sample:
-        np.testing.assert_array_equal(out[b].cpu().numpy().view(np.uint16), vis[b][keep[b]])
-    # hand-off sequence for the whole batch (kept tokens, then questions, with positions)
     seq, pos = ctx.assemble(vis_t, torch.from_numpy(keep).to(DEV), text_t, lens, pos_offset=35)
     torch.cuda.synchronize()
     ctx.check()
-    s_ref, p_ref = O.assemble(vis, keep, text, lens, 35)
+    np.testing.assert_array_equal(out.cpu().numpy().view(np.uint16), O.gather(vis, keep))
+    s_ref, pos_ref = O.assemble(vis, keep, text, lens, 35)
     np.testing.assert_array_equal(seq.cpu().numpy().view(np.uint16), s_ref)
-    np.testing.assert_array_equal(pos.cpu().numpy(), p_ref)
-    return lens
+    np.testing.assert_array_equal(pos.cpu().numpy(), pos_ref)
+    reps = [f.result() for f in f_sel]
+    bad = [(b, r["reason"]) for b, r in enumerate(reps) if not r["ok"]]
+    assert not bad, f"selection on the oracle's scores: {bad[:3]}"
+    OP.record(f"{key} all {B} images (oracle scores)", reps, max(errs))
+    if own_scores:
+        reps = [f.result() for f in f_own]
+        bad = [(b, r["reason"]) for b, r in enumerate(reps) if not r["ok"]]
+        assert not bad, f"selection on the GPU's own scores: {bad[:3]}"
+        OP.record(f"{key} all {B} images (map_prune's own GPU scores)", reps, max(errs))
+    ctx.close()
 
 
-def test_batched_serving_config_sampled():
-    """64 images, N = 2880, k = 160, ragged questions, near-duplicate images (b % 10 == 0)."""
-    wl = W.WORKLOADS["c3"]
-    _batch_parity(wl, sample=[0, 7, 63], K=wl.K)
+def test_batched_serving_config_every_image():
+    """64 images, N = 2880, k = 160, ragged questions, near-duplicate images (b % 10 == 0):
+    every image, on the oracle's scores and on map_prune's own scores."""
+    _full_batch_parity("c3", own_scores=True)
 
 
-def test_high_token_config_sampled():
+def test_high_token_config_every_image():
     """16 images, N = 7290, D = 3584, k = 405, questions up to 512 tokens (two column tiles
     in Eq. 3) and K0 = 202 (no projection pass; coordinates in global memory)."""
-    wl = W.WORKLOADS["c4"]
-    lens = W.make_lens(wl)
-    long_q = int(np.argmax(lens))
-    assert lens[long_q] > 256
-    _batch_parity(wl, sample=sorted({0, long_q}), K=wl.K)
+    assert W.make_lens(W.WORKLOADS["c4"]).max() > 256
+    _full_batch_parity("c4")
 
 
 _SWEEP = {}
@@ -393,4 +419,5 @@ def test_retention_sweep_config(K, lam, k0_frac):
     ctx, w = make_ctx(dims, lam=lam, k0_frac=k0_frac)
     vis, p32 = _sweep_inputs()
     keep, order = run_select(ctx, p32, vis, K)
-    assert_selection(p32, vis, K, O.resolve_k0(K, k0_frac), keep, order, lam=lam)
+    assert_selection(p32, vis, K, O.resolve_k0(K, k0_frac), keep, order, lam=lam,
+                     label=f"c2 N=2880 k={K} lambda={lam} K0={O.resolve_k0(K, k0_frac)}")

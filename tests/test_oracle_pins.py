@@ -12,6 +12,7 @@ import scipy.special
 import torch
 
 from oracle import map_oracle as O
+from oracle import parity as P
 from paper_2608_06411_gb300 import workloads as W
 
 
@@ -454,3 +455,79 @@ def test_assemble_hand_example():
     seq, pos = O.assemble(vis, np.zeros((2, 0), np.int64), text, [3, 0])
     np.testing.assert_array_equal(seq, text)
     np.testing.assert_array_equal(pos, [4, 5, 6])
+
+
+# ------------------------------------------------------------------ the forced-replay parity checker
+# The GPU selection is accepted by oracle/parity.py::check_selection: a pick must be the
+# oracle's argmax wherever the oracle's margin (v1 - v2) / v1 exceeds 1e-4; below that margin
+# any near-best token is valid and the check continues from it.  These cases feed the checker
+# pick orders that did not come from the oracle, built by hand on orthogonal tokens whose
+# values p_i * ||residual_i|| are known in closed form.
+
+def _orthogonal_case():
+    """Eight orthonormal tokens, value_i = p_i at every step.  K0 = 1, K = 6.  Greedy order
+    by p: 0 (R0), 1, 2, then 4 (0.100004) over 3 (0.1) with margin 4e-5 (below 1e-4), 7, 5."""
+    p = np.array([0.30, 0.20, 0.15, 0.10, 0.100004, 0.05, 0.04, 0.056])
+    return p, np.eye(8), 6, 1
+
+
+def test_checker_accepts_the_oracle_order_and_counts_its_near_tie():
+    p, V, K, K0 = _orthogonal_case()
+    order = [0, 1, 2, 4, 3, 7]
+    assert O.select(p, V, K, K0)["picks"].tolist() == order
+    rep = P.check_selection(p, V, K, K0, order, sorted(order))
+    assert rep["ok"] and rep["identical"] and rep["sub_margin_steps"] == 1
+
+
+def test_checker_accepts_a_swap_below_the_margin():
+    p, V, K, K0 = _orthogonal_case()
+    rep = P.check_selection(p, V, K, K0, [0, 1, 2, 3, 4, 7], [0, 1, 2, 3, 4, 7])
+    assert rep["ok"] and not rep["identical"] and rep["sub_margin_steps"] == 1
+
+
+def test_checker_rejects_a_wrong_pick_above_the_margin():
+    p, V, K, K0 = _orthogonal_case()
+    rep = P.check_selection(p, V, K, K0, [0, 1, 7, 2, 4, 3], [0, 1, 2, 3, 4, 7])
+    assert not rep["ok"] and "picked 7" in rep["reason"]
+    # the same set in another order is still wrong: token 2 must come before 4 and 3
+    assert not P.check_selection(p, V, K, K0, [0, 1, 4, 2, 3, 7])["ok"]
+
+
+def test_checker_rejects_repeated_out_of_range_and_unsorted_picks():
+    p, V, K, K0 = _orthogonal_case()
+    assert not P.check_selection(p, V, K, K0, [0, 1, 2, 4, 4, 7])["ok"]
+    assert not P.check_selection(p, V, K, K0, [0, 1, 2, 4, 3, 8])["ok"]
+    assert not P.check_selection(p, V, K, K0, [0, 1, 2, 4, 3])["ok"]
+    assert not P.check_selection(p, V, K, K0, [0, 1, 2, 4, 3, 7], [0, 1, 2, 3, 7, 4])["ok"]
+
+
+def test_checker_rejects_a_wrong_r0():
+    p, V, K, K0 = _orthogonal_case()
+    # the top-1 set is {0}, with a wide boundary margin (0.30 vs 0.20)
+    rep = P.check_selection(p, V, K, K0, [1, 0, 2, 4, 3, 7], [0, 1, 2, 3, 4, 7])
+    assert not rep["ok"] and "R0" in rep["reason"]
+    assert not P.check_selection(p, V, 6, 2, [0, 2, 1, 4, 3, 7])["ok"]     # R0 out of p order
+
+
+def _divergent_case():
+    """Tokens 0 = e1 and 1 = (cos .3, sin .3, 0, 0) tie below the margin (values 1 and
+    0.99995).  After picking 0 the best next token is 2 = e2 (0.6 against 0.59 for 3 = e3);
+    after picking 1 instead, e2 keeps a residual of cos .3, so 2 is worth 0.6 cos .3 = 0.573
+    and 3 (0.59) wins.  Both paths are valid; they keep different sets."""
+    t = 0.3
+    V = np.array([[1.0, 0, 0, 0], [math.cos(t), math.sin(t), 0, 0], [0, 1.0, 0, 0], [0, 0, 1.0, 0]])
+    p = np.array([1.0, 0.99995, 0.6, 0.59])
+    return p, V, 2, 0
+
+
+def test_checker_follows_the_gpu_path_after_a_near_tie():
+    p, V, K, K0 = _divergent_case()
+    assert O.select(p, V, K, K0)["picks"].tolist() == [0, 2]
+    rep = P.check_selection(p, V, K, K0, [1, 3], [1, 3])
+    assert rep["ok"] and rep["sub_margin_steps"] == 1 and not rep["identical"]
+    # the replay evaluates step 1 with token 1 (not the oracle's 0) in the basis
+    steps = O.select_replay(p, V, K, K0, [1, 3])["steps"]
+    assert [s["best"] for s in steps] == [0, 3]
+    assert abs(steps[1]["v_best"] - 0.59) < 1e-12
+    # continuing from 1, token 2 is no longer the best: [1, 2] is a wrong pick above the margin
+    assert not P.check_selection(p, V, K, K0, [1, 2])["ok"]

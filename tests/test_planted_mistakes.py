@@ -11,6 +11,7 @@ import pytest
 
 from oracle import distill_oracle as DO
 from oracle import map_oracle as O
+from oracle import parity as P
 from oracle import qcts_oracle as Q
 
 import test_distill_pins
@@ -137,6 +138,64 @@ def test_scoring_and_selection_mistakes_are_caught(monkeypatch, attr, bad):
 def test_missing_basis_update_is_caught(monkeypatch):
     monkeypatch.setattr(O._Basis, "add", _add_without_update)
     assert _some_pin_fails(test_oracle_pins, test_golden)
+
+
+# ------------------------------------------------------------------ the forced-replay checker
+
+def _replay_from_own_best(p, V, K, K0, forced, lam=1.0, tau=1e-5):
+    """select_replay that records the forced pick but continues from its own argmax."""
+    p = np.asarray(p, dtype=np.float64)
+    K0 = max(0, min(K0, K))
+    basis = O._Basis(V, tau)
+    alive = np.ones(len(p), dtype=bool)
+    steps = []
+    for t, j in enumerate(int(x) for x in forced):
+        if t < K0:
+            alive[j] = False
+            basis.add(j)
+            continue
+        vals = O._values(p, basis.rho(), lam)
+        vals[~alive] = -np.inf
+        best = int(np.argmax(vals))
+        steps.append(dict(t=t, forced=j, best=best, v_forced=float(vals[j]), v_best=float(vals[best]),
+                          margin=O._margin(vals), forced_alive=bool(alive[j])))
+        alive[best] = False
+        basis.add(best)
+    return dict(r0=O._top_order(p)[:K0], steps=steps)
+
+
+def _checker_accepts_anything(p, V, K, K0, gpu_order, gpu_keep=None, lam=1.0, tau=1e-5, margin=1e-4):
+    return dict(ok=True, reason="", sub_margin_steps=0, identical=True)
+
+
+_orig_check_selection = P.check_selection
+
+
+def _checker_without_r0(p, V, K, K0, gpu_order, gpu_keep=None, lam=1.0, tau=1e-5, margin=1e-4):
+    return _orig_check_selection(p, V, K, 0, gpu_order, gpu_keep, lam, tau, margin)
+
+
+def _checker_ignores_repeats(p, V, K, K0, gpu_order, gpu_keep=None, lam=1.0, tau=1e-5, margin=1e-4):
+    order = list(dict.fromkeys(int(x) for x in np.asarray(gpu_order).reshape(-1)))
+    if len(order) < K:
+        return dict(ok=True, reason="", sub_margin_steps=0, identical=False)
+    return _orig_check_selection(p, V, K, K0, order, None, lam, tau, margin)
+
+
+def _checker_without_value_bound(p, V, K, K0, gpu_order, gpu_keep=None, lam=1.0, tau=1e-5, margin=1e-4):
+    return _orig_check_selection(p, V, K, K0, gpu_order, gpu_keep, lam, tau, margin=1.0)
+
+
+@pytest.mark.parametrize("target,attr,bad", [
+    (O, "select_replay", _replay_from_own_best),
+    (P, "check_selection", _checker_accepts_anything),
+    (P, "check_selection", _checker_without_r0),
+    (P, "check_selection", _checker_ignores_repeats),
+    (P, "check_selection", _checker_without_value_bound),
+])
+def test_parity_checker_mistakes_are_caught(monkeypatch, target, attr, bad):
+    monkeypatch.setattr(target, attr, bad)
+    assert _some_pin_fails(test_oracle_pins)
 
 
 # ------------------------------------------------------------------ QCTS oracle
