@@ -115,8 +115,11 @@ int map_score(map_ctx *ctx, const void *text_feats, const void *vis_feats,
  * k == N keeps every token (keep_idx = pick_order = 0..N-1); k == 0 is a no-op;
  * k > N is MAP_EINVAL.  Supported: N <= 16384; k <= 4096 for plain top-k (lambda = 0 or
  * K0 = k), k <= 1024 with the diversity term (MAP_EUNSUPPORTED beyond).
- * Runs a few selection rounds per host synchronisation: the call returns after the
- * selection has finished on the device (the final gather of indices is still queued).
+ * Asynchronous like the other calls: after its first rounds the selection runs as a
+ * device-side loop (a CUDA graph whose WHILE node repeats two rounds while an image still
+ * selects; built on the first call of a shape and workspace, then cached in the context), so
+ * the host never waits for it.  A device-side failure (a bounded wait that ran out, or the
+ * loop's iteration cap, which no input reaches) is reported by map_status.
  */
 int map_select(map_ctx *ctx, const float *scores, const void *vis_feats, int B, int N,
                int k, int32_t *keep_idx, int32_t *pick_order, void *stream);
@@ -296,6 +299,8 @@ typedef struct {
     long long gram_rows;      /* Gram-block rows evaluated by the selection */
 } map_counters;
 
+/* The launches of the selection's device-side loop are counted on the device: this call reads
+ * that count (a synchronous copy), so it includes the loop iterations that have completed. */
 int map_get_counters(map_ctx *ctx, map_counters *out);
 
 /* Kernel ids for timing. */
@@ -322,6 +327,12 @@ int map_read_timing(map_ctx *ctx, int id, double *total_ms, long long *count);
  * Device pointers; x, w bf16; K % 64 == 0, Nout % 64 == 0. */
 int map_linear(map_ctx *ctx, const void *x, const void *w, const void *b, int M, int K,
                int Nout, int epi, void *y, void *stream);
+
+/* Limit, in ns, of every wait inside the tensor-core GEMM kernels that this context launches
+ * (ns <= 0 restores the default of 2 s).  A wait that runs out makes the kernel stop issuing
+ * work, let the copies and MMAs already in flight land, release its tensor memory and exit;
+ * map_status then reports MAP_ETIMEOUT.  For tests of that path; MAP_EINVAL for NULL. */
+int map_set_wait_limit(map_ctx *ctx, long long ns);
 
 /* map_score that also writes q [sum(lens), dp] and k [B*N, dp] (fp32, after RoPE). */
 int map_score_debug(map_ctx *ctx, const void *text_feats, const void *vis_feats,

@@ -71,6 +71,7 @@ SIGNATURES = {
     "map_strerror": (ctypes.c_char_p, [c_int]),
     "map_get_counters": (c_int, [c_void_p, POINTER(MapCounters)]),
     "map_set_timing": (c_int, [c_void_p, c_int]),
+    "map_set_wait_limit": (c_int, [c_void_p, c_longlong]),
     "map_read_timing": (c_int, [c_void_p, c_int, POINTER(c_double), POINTER(c_longlong)]),
     "map_linear": (c_int, [c_void_p, c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_int, c_void_p, c_void_p]),
     "map_score_debug": (c_int, [c_void_p, c_void_p, c_void_p, POINTER(c_int32), c_int, c_int, c_void_p, c_void_p,
@@ -307,6 +308,10 @@ class Context:
         c = MapCounters()
         _check(lib.map_get_counters(self.h, ctypes.byref(c)), "map_get_counters")
         return {"launches": c.launches, "select_rounds": c.select_rounds, "gram_rows": c.gram_rows}
+
+    def set_wait_limit(self, ns: int) -> None:
+        """Limit of the GEMM kernels' waits in ns (<= 0: the 2 s default); for tests."""
+        _check(lib.map_set_wait_limit(self.h, int(ns)), "map_set_wait_limit")
 
     def set_timing(self, enable: bool) -> None:
         _check(lib.map_set_timing(self.h, int(bool(enable))), "map_set_timing")

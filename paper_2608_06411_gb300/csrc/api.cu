@@ -40,7 +40,7 @@ struct map_ctx {
   // [hi | hi | lo] of W_Q W_T2 / W_K W_V2 ([dp, 3 Dh]) and fp32 biases W_Q b_T2 / W_K b_V2
   void* wqt = nullptr; void* wkv = nullptr; float* bqt = nullptr; float* bkv = nullptr;
   DevBuf rope;  int rope_rows = 0;
-  DevBuf h1, kb, th1, qb, stats, qoff, post, sqn, pmean, snv, dist;
+  DevBuf h1, kb, th1, qb, stats, qoff, post, sqn, pmean, snv, dist, dsa, dsb;
   // selection
   DevBuf sU, sr2, scstep, sstate, sEc, spicks, sr0, sbt, srn, ssmall, stheta, saslot, sVg, sG;
   // map_prune staging
@@ -50,6 +50,8 @@ struct map_ctx {
   int32_t* h_done = nullptr;        // pinned, mapped
   int* h_status_dev = nullptr; int32_t* h_done_dev = nullptr;   // their device aliases
   cudaStream_t s_in = nullptr, s_out = nullptr;   // map_prune copy streams (host buffers)
+  cudaStream_t s_aux = nullptr;     // question branch of the predictor, concurrent with the visual one
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
   bool timing = false;
   std::vector<TimedPair> pairs;
   std::vector<cudaEvent_t> free_events;
@@ -57,6 +59,9 @@ struct map_ctx {
   long long t_n[MAP_K_NUM] = {};
   map_counters counters{};
   int deferred = MAP_OK;
+  long long wait_ns = 0;            // GEMM role-wait limit (0: the kernels' default)
+  mapk::SelLoopCache* loops = nullptr;   // cached graphs of the selection's device-side round loop
+  long long* loop_iters_total = nullptr; // device: loop iterations run so far (two rounds each)
 };
 
 namespace {
@@ -167,7 +172,9 @@ int ensure_rope(map_ctx* c, int rows_needed) {
 
 int gemm(map_ctx* c, const GemmDesc& d, cudaStream_t st) {
   ++c->counters.launches;
-  cudaError_t e = mapk::launch_gemm(d, c->num_sms, st);
+  GemmDesc dd = d;
+  dd.wait_ns = c->wait_ns;
+  cudaError_t e = mapk::launch_gemm(dd, c->num_sms, st);
   if (e == cudaErrorInvalidValue) return MAP_EUNSUPPORTED;
   return cuda_err(e);
 }
@@ -264,11 +271,20 @@ int score_impl(map_ctx* c, const void* text, const void* vis, const int32_t* len
   const int dp3 = 3 * g.dp;
   MAP_TRY(ensure(c->kb, static_cast<size_t>(vrows) * dp3 * 2));
   MAP_TRY(ensure(c->qb, static_cast<size_t>(total_m) * dp3 * 2));
-  MAP_TRY(predictor_branch(c, vis, vrows, c->w[5], c->w[6], c->wkv, c->bkv, c->h1, c->kb.p, 0, 1.0f, k_out, nullptr,
-                           N, st, MAP_K_GEMM_FV1, MAP_K_GEMM_WK));
+  // The two branches are independent until Eq. 3: the question branch runs on a second stream
+  // (it fills SMs that a small batch's visual GEMMs leave idle), joined before the logits.
+  if (!c->s_aux) CU_TRY(cudaStreamCreateWithFlags(&c->s_aux, cudaStreamNonBlocking));
+  if (!c->ev_fork) CU_TRY(cudaEventCreateWithFlags(&c->ev_fork, cudaEventDisableTiming));
+  if (!c->ev_join) CU_TRY(cudaEventCreateWithFlags(&c->ev_join, cudaEventDisableTiming));
+  CU_TRY(cudaEventRecord(c->ev_fork, st));
+  CU_TRY(cudaStreamWaitEvent(c->s_aux, c->ev_fork, 0));
   MAP_TRY(predictor_branch(c, text, total_m, c->w[0], c->w[1], c->wqt, c->bqt, c->th1, c->qb.p, 1,
                            1.0f / std::sqrt(static_cast<float>(g.dp)), q_out, static_cast<const int*>(c->post.p), 1,
-                           st, MAP_K_GEMM_TEXT, MAP_K_GEMM_TEXT));
+                           c->s_aux, MAP_K_GEMM_TEXT, MAP_K_GEMM_TEXT));
+  CU_TRY(cudaEventRecord(c->ev_join, c->s_aux));
+  MAP_TRY(predictor_branch(c, vis, vrows, c->w[5], c->w[6], c->wkv, c->bkv, c->h1, c->kb.p, 0, 1.0f, k_out, nullptr,
+                           N, st, MAP_K_GEMM_FV1, MAP_K_GEMM_WK));
+  CU_TRY(cudaStreamWaitEvent(st, c->ev_join, 0));
   // Eq. 3 on the tensor cores: logits tile [visual tokens x question tokens] of one image,
   // pass 1 -> per-slab column (max, sum exp), combine -> (max, 1/sum), pass 2 -> mean.
   const int m_tiles = (N + 127) / 128, nparts = 4 * m_tiles;
@@ -360,7 +376,7 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, const int32_t*
   MAP_TRY(ensure(c->sr0, static_cast<size_t>(B) * K * 4));
   MAP_TRY(ensure(c->sbt, static_cast<size_t>(B) * K * 4));
   MAP_TRY(ensure(c->srn, static_cast<size_t>(B) * K * 4));
-  MAP_TRY(ensure(c->ssmall, static_cast<size_t>(B) * 4 * 16 + 20 * 256));
+  MAP_TRY(ensure(c->ssmall, static_cast<size_t>(B) * 4 * 16 + 24 * 256));
   static_assert(mapk::kReprojMax <= kProjMaxBasis, "re-projection basis limit");
   MAP_TRY(ensure(c->stheta, static_cast<size_t>(B) * 8));
   MAP_TRY(ensure(c->saslot, static_cast<size_t>(B) * S * 4));
@@ -387,6 +403,8 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, const int32_t*
   s.blist = carve<int32_t>(sm, B);
   s.bcount = carve<int32_t>(sm, 2);
   s.done_count = carve<int32_t>(sm, 1);
+  s.uptr = carve<const void*>(sm, 2);
+  int32_t* loop_iters = carve<int32_t>(sm, 1);
   s.theta = static_cast<uint64_t*>(c->stheta.p);
   s.aslot = static_cast<int32_t*>(c->saslot.p);
 
@@ -421,9 +439,7 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, const int32_t*
     d.blist = s.blist;                           // images still selecting (built by choose)
     // the GEMM after a list producer reads the count that producer appended through
     auto take_list = [&](GemmDesc& g) { g.bcount = s.bcount + s.bc_par; s.bc_par ^= 1; };
-    const long long cap = 8LL * (K + N / S) + 64;
-    long long rounds = 0;
-    int burst = (K0 + S - 1) / S + 6;   // rounds queued per host check; finished images skip
+    const long long cap = 8LL * (K + N / S) + 64;   // rounds; far above what any input needs
     if (project) {
       // R0: gather its rows, G[R0, R0] on the tensor cores, then its Cholesky factor.
       c->counters.launches += 3;
@@ -435,7 +451,6 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, const int32_t*
         MAP_TRY(gemm(c, d0, st));
       }
       CU_TRY(mapk::launch_sel_chol(s, st));
-      ++rounds;
       ++c->counters.select_rounds;
       // every candidate's exact value: one tensor-core pass over V against the R0 basis
       GemmDesc pd{};
@@ -469,36 +484,18 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, const int32_t*
       take_list(d);
       MAP_TRY(gemm(c, d, st));
       CU_TRY(mapk::launch_sel_greedy(s, st));
-      ++rounds;
       ++c->counters.select_rounds;
       MAP_TRY(project_all(false));
-      burst = 2;
     }
-    for (;;) {
-      for (int r = 0; r < burst; ++r) {
-        c->counters.launches += 4;
-        CU_TRY(mapk::launch_sel_choose(s, st));
-        take_list(d);
-        MAP_TRY(gemm(c, d, st));
-        CU_TRY(mapk::launch_sel_greedy(s, st));
-      }
-      rounds += burst;
-      c->counters.select_rounds += burst;
-      // through host-mapped words (no copy engine: bulk copies on other streams do not delay it)
-      CU_TRY(mapk::launch_flags_to_host(s.done_count, c->status, c->h_done_dev, c->h_status_dev, st));
-      ++c->counters.launches;
-      CU_TRY(cudaStreamSynchronize(st));
-      if (*c->h_done >= B) break;
-      if (*c->h_status) {               // a kernel gave up (bounded wait) or saw a bad index: stop here
-        c->deferred = dev_status_error(*c->h_status);
-        return c->deferred;
-      }
-      if (rounds > cap) {
-        c->deferred = MAP_EINTERNAL;
-        return MAP_EINTERNAL;
-      }
-      burst = 2;
-    }
+    // The remaining rounds run as a device-side loop (a CUDA graph whose WHILE node repeats two
+    // rounds while an image still selects): the host never waits for them.
+    if (!c->loops) c->loops = mapk::sel_loop_cache_create();
+    if (!c->loops) return MAP_ENOMEM;
+    GemmDesc dl = d;
+    dl.wait_ns = c->wait_ns;
+    ++c->counters.launches;            // the test kernel ahead of the loop; iterations are counted on the device
+    CU_TRY(mapk::launch_sel_loop(c->loops, s, dl, c->num_sms, static_cast<int>((cap + 1) / 2), loop_iters,
+                                 c->loop_iters_total, st));
   } else {
     ++c->counters.launches;
     CU_TRY(mapk::launch_sel_copy_r0(s.r0, B, K, s.picks, st));
@@ -621,6 +618,11 @@ int map_init(const map_config* cfg, const map_weights* w, map_ctx** out) {
       rc = MAP_ECUDA;
       break;
     }
+    if (cudaMalloc(reinterpret_cast<void**>(&c->loop_iters_total), sizeof(long long)) != cudaSuccess) {
+      rc = MAP_ENOMEM;
+      break;
+    }
+    if (cudaMemset(c->loop_iters_total, 0, sizeof(long long)) != cudaSuccess) { rc = MAP_ECUDA; break; }
     if (cudaMalloc(&c->status, sizeof(int)) != cudaSuccess) { rc = MAP_ENOMEM; break; }
     if (cudaMemset(c->status, 0, sizeof(int)) != cudaSuccess) { rc = MAP_ECUDA; break; }
     if (cudaHostAlloc(&c->h_status, sizeof(int), cudaHostAllocMapped) != cudaSuccess) { rc = MAP_ENOMEM; break; }
@@ -874,78 +876,119 @@ int map_distill_grad(map_ctx* ctx, const void* text_feats, const void* vis_feats
   int32_t* qo = static_cast<int32_t*>(c->qoff.p);
   int32_t* post = static_cast<int32_t*>(c->post.p);
   CU_TRY(mapk::launch_query_meta(lens, offs.data(), B, N, qo, qo + (B + 1), post, nullptr, nullptr, st));
-  // fp32 workspace
+  // fp32 workspace (the features and weights stay bf16: the tensor-core GEMMs read them as exact
+  // operands; only the biases are needed in fp32)
   const int nblk = (N + 255) / 256;
-  const long long wsz[10] = {Dh * D, Dh, Dh * Dh, Dh, dp * Dh, Dh * D, Dh, Dh * Dh, Dh, dp * Dh};
-  long long wtot = 0;
-  for (long long x : wsz) wtot += x;
-  const long long floats = wtot + (Tv + Tt) * D + 5 * (Tv + Tt) * Dh + 4 * (Tv + Tt) * dp + Tt * N + 2LL * B * N +
+  const long long Np = (N + 3) / 4 * 4;              // logits row stride: 16-byte aligned rows
+  const int bias_idx[4] = {1, 3, 6, 8};
+  const long long floats = 4 * Dh + 5 * (Tv + Tt) * Dh + 4 * (Tv + Tt) * dp + Tt * Np + 2LL * B * N +
                            static_cast<long long>(B) * nblk + total_m + 64 * 16;
   MAP_TRY(ensure(c->dist, static_cast<size_t>(floats) * 4));
   float* base = static_cast<float*>(c->dist.p);
   auto take = [&](long long n) { float* p = base; base += ((n + 15) / 16) * 16; return p; };
-  float* Wf[10];
-  for (int i = 0; i < 10; ++i) Wf[i] = take(wsz[i]);
-  float* Vf = take(Tv * D);
-  float* Tf = take(Tt * D);
+  float* Wb[10] = {};
+  for (int i : bias_idx) Wb[i] = take(Dh);
   float *z1v = take(Tv * Dh), *h1v = take(Tv * Dh), *h2v = take(Tv * Dh), *dh2v = take(Tv * Dh), *dh1v = take(Tv * Dh);
   float *z1t = take(Tt * Dh), *h1t = take(Tt * Dh), *h2t = take(Tt * Dh), *dh2t = take(Tt * Dh), *dh1t = take(Tt * Dh);
   float *kp = take(Tv * dp), *kk = take(Tv * dp), *dk = take(Tv * dp), *dkp = take(Tv * dp);
   float *qp = take(Tt * dp), *qq = take(Tt * dp), *dq = take(Tt * dp), *dqp = take(Tt * dp);
-  float* S = take(Tt * N);
+  float* S = take(Tt * Np);
   float *p_hat = take(static_cast<long long>(B) * N), *gb = take(static_cast<long long>(B) * N);
   float* part = take(static_cast<long long>(B) * nblk);
   int32_t* d_row_img = reinterpret_cast<int32_t*>(take(total_m));
-  CU_TRY(mapk::launch_put_ints(row_img.data(), static_cast<int>(total_m), d_row_img, st));
-  for (int i = 0; i < 10; ++i) CU_TRY(mapk::launch_bf16_to_f32(c->w[i], wsz[i], Wf[i], st));
-  CU_TRY(mapk::launch_bf16_to_f32(vis_feats, Tv * D, Vf, st));
-  CU_TRY(mapk::launch_bf16_to_f32(text_feats, Tt * D, Tf, st));
-  const float2* tab = static_cast<const float2*>(c->rope.p);
   const float rs = 1.0f / std::sqrt(static_cast<float>(dp));
+  // Every contraction of the step, in order: C = alpha A(M x K) B(K x N) with A(i, k) = ta ? A[k lda
+  // + i] : A[i lda + k], B(k, j) = tb ? B[j ldb + k] : B[k ldb + j]; bf16 operands are exact.
+  struct Mm { bool ta, tb; long long M, N, K; float alpha; const void* A; bool abf; long long lda;
+              const void* Bm; bool bbf; long long ldb; float* C; long long ldc; };
+  std::vector<Mm> fwd, mid, bwd;
+  auto branch_fwd = [&](const void* X, long long T, int i1, float* z1, float* h1, float* h2, int ip, float* pre) {
+    fwd.push_back({false, true, T, Dh, D, 1.f, X, true, D, c->w[i1], true, D, z1, Dh});
+    fwd.push_back({false, true, T, Dh, Dh, 1.f, h1, false, Dh, c->w[i1 + 2], true, Dh, h2, Dh});
+    fwd.push_back({false, true, T, dp, Dh, 1.f, h2, false, Dh, c->w[ip], true, Dh, pre, dp});
+  };
+  branch_fwd(vis_feats, Tv, 5, z1v, h1v, h2v, 9, kp);
+  branch_fwd(text_feats, Tt, 0, z1t, h1t, h2t, 4, qp);
+  for (int b = 0; b < B; ++b)     // Eq. 3 logits per image, then (after the loss) dq and dk
+    mid.push_back({false, true, lens[b], N, dp, rs, qq + offs[b] * dp, false, dp, kk + b * N * dp, false, dp,
+                   S + offs[b] * Np, Np});
+  for (int b = 0; b < B; ++b) {
+    mid.push_back({false, false, lens[b], dp, N, rs, S + offs[b] * Np, false, Np, kk + b * N * dp, false, dp,
+                   dq + offs[b] * dp, dp});
+    mid.push_back({true, false, N, dp, lens[b], rs, S + offs[b] * Np, false, Np, qq + offs[b] * dp, false, dp,
+                   dk + b * N * dp, dp});
+  }
+  auto branch_bwd = [&](long long T, float* dpre, const void* X, int i1, const float* h1, const float* h2, float* dh2,
+                        float* dh1, int ip) {
+    bwd.push_back({true, false, dp, Dh, T, 1.f, dpre, false, dp, h2, false, Dh, gout[ip], Dh});
+    bwd.push_back({false, false, T, Dh, dp, 1.f, dpre, false, dp, c->w[ip], true, Dh, dh2, Dh});
+    bwd.push_back({true, false, Dh, Dh, T, 1.f, dh2, false, Dh, h1, false, Dh, gout[i1 + 2], Dh});
+    bwd.push_back({false, false, T, Dh, Dh, 1.f, dh2, false, Dh, c->w[i1 + 2], true, Dh, dh1, Dh});
+    bwd.push_back({true, false, Dh, D, T, 1.f, dh1, false, Dh, X, true, D, gout[i1], D});
+  };
+  branch_bwd(Tv, dkp, vis_feats, 5, h1v, h2v, dh2v, dh1v, 9);
+  branch_bwd(Tt, dqp, text_feats, 0, h1t, h2t, dh2t, dh1t, 4);
+  // staging buffers for the split-bf16 operands: the largest any contraction needs
+  size_t wa = 0, wb = 0;
+  for (const auto* list : {&fwd, &mid, &bwd})
+    for (const Mm& m : *list) {
+      size_t a = 0, bb = 0;
+      mapk::tc_matmul_ws(static_cast<int>(m.M), static_cast<int>(m.N), static_cast<int>(m.K), m.alpha, m.abf, m.bbf,
+                         &a, &bb);
+      wa = std::max(wa, a);
+      wb = std::max(wb, bb);
+    }
+  MAP_TRY(ensure(c->dsa, wa * 2));
+  MAP_TRY(ensure(c->dsb, wb * 2));
+  long long n_mm = 0;
+  auto run_mm = [&](const Mm& m) -> int {
+    ++n_mm;
+    cudaError_t e = mapk::launch_tc_matmul(m.ta, m.tb, static_cast<int>(m.M), static_cast<int>(m.N),
+                                           static_cast<int>(m.K), m.alpha, m.A, m.abf, m.lda, m.Bm, m.bbf, m.ldb,
+                                           m.C, m.ldc, c->dsa.p, c->dsb.p, c->num_sms, c->status, c->wait_ns, st);
+    if (e == cudaErrorInvalidValue) return MAP_EUNSUPPORTED;
+    return cuda_err(e);
+  };
+  CU_TRY(mapk::launch_put_ints(row_img.data(), static_cast<int>(total_m), d_row_img, st));
+  for (int i : bias_idx) CU_TRY(mapk::launch_bf16_to_f32(c->w[i], Dh, Wb[i], st));
+  const float2* tab = static_cast<const float2*>(c->rope.p);
   // forward: z1 = X W1^T + b1, h1 = GELU(z1), h2 = h1 W2^T + b2, projection, RoPE
-  auto branch_fwd = [&](const float* X, long long T, int i1, float* z1, float* h1, float* h2, int ip, float* pre,
-                        float* post_rope, const int32_t* pos, int pos_mod) -> int {
-    CU_TRY(mapk::launch_sgemm(false, true, T, Dh, D, 1.f, X, D, Wf[i1], D, false, z1, Dh, st));
-    CU_TRY(mapk::launch_bias_gelu(z1, Wf[i1 + 1], T, Dh, h1, st));
-    CU_TRY(mapk::launch_sgemm(false, true, T, Dh, Dh, 1.f, h1, Dh, Wf[i1 + 2], Dh, false, h2, Dh, st));
-    CU_TRY(mapk::launch_bias_add(h2, Wf[i1 + 3], T, Dh, st));
-    CU_TRY(mapk::launch_sgemm(false, true, T, dp, Dh, 1.f, h2, Dh, Wf[ip], Dh, false, pre, dp, st));
+  auto fwd_tail = [&](int j, long long T, int i1, float* z1, float* h1, float* h2, float* pre, float* post_rope,
+                      const int32_t* pos, int pos_mod) -> int {
+    MAP_TRY(run_mm(fwd[j]));
+    CU_TRY(mapk::launch_bias_gelu(z1, Wb[i1 + 1], T, Dh, h1, st));
+    MAP_TRY(run_mm(fwd[j + 1]));
+    CU_TRY(mapk::launch_bias_add(h2, Wb[i1 + 3], T, Dh, st));
+    MAP_TRY(run_mm(fwd[j + 2]));
     CU_TRY(mapk::launch_rope_f32(false, pre, T, dp, tab, c->rope_rows, pos, pos_mod, post_rope, st));
     return MAP_OK;
   };
-  MAP_TRY(branch_fwd(Vf, Tv, 5, z1v, h1v, h2v, 9, kp, kk, nullptr, g.rope_on ? N : 1));
-  MAP_TRY(branch_fwd(Tf, Tt, 0, z1t, h1t, h2t, 4, qp, qq, g.rope_on ? post : nullptr, 1));
+  MAP_TRY(fwd_tail(0, Tv, 5, z1v, h1v, h2v, kp, kk, nullptr, g.rope_on ? N : 1));
+  MAP_TRY(fwd_tail(3, Tt, 0, z1t, h1t, h2t, qp, qq, g.rope_on ? post : nullptr, 1));
   // Eq. 3 logits per image, softmax, KL, and dL/dlogits
-  for (int b = 0; b < B; ++b)
-    CU_TRY(mapk::launch_sgemm(false, true, lens[b], N, dp, rs, qq + offs[b] * dp, dp, kk + b * N * dp, dp, false,
-                              S + offs[b] * N, N, st));
-  CU_TRY(mapk::launch_distill_loss_grad(S, total_m, qo, d_row_img, teacher, B, N, p_hat, gb, part, loss, st));
-  for (int b = 0; b < B; ++b) {
-    CU_TRY(mapk::launch_sgemm(false, false, lens[b], dp, N, rs, S + offs[b] * N, N, kk + b * N * dp, dp, false,
-                              dq + offs[b] * dp, dp, st));
-    CU_TRY(mapk::launch_sgemm(true, false, N, dp, lens[b], rs, S + offs[b] * N, N, qq + offs[b] * dp, dp, false,
-                              dk + b * N * dp, dp, st));
-  }
+  for (int b = 0; b < B; ++b) MAP_TRY(run_mm(mid[b]));
+  CU_TRY(mapk::launch_distill_loss_grad(S, Np, total_m, qo, d_row_img, teacher, B, N, p_hat, gb, part, loss, st));
+  for (size_t j = B; j < mid.size(); ++j) MAP_TRY(run_mm(mid[j]));
   // backward through RoPE, the projection and the MLP of each branch
-  auto branch_bwd = [&](float* dpost, long long T, const int32_t* pos, int pos_mod, float* dpre, const float* X,
-                        int i1, const float* z1, const float* h1, const float* h2, float* dh2, float* dh1,
-                        int ip) -> int {
+  auto bwd_tail = [&](int j, float* dpost, long long T, const int32_t* pos, int pos_mod, float* dpre, const float* z1,
+                      float* dh2, float* dh1, int i1) -> int {
     CU_TRY(mapk::launch_rope_f32(true, dpost, T, dp, tab, c->rope_rows, pos, pos_mod, dpre, st));
-    CU_TRY(mapk::launch_sgemm(true, false, dp, Dh, T, 1.f, dpre, dp, h2, Dh, false, gout[ip], Dh, st));
-    CU_TRY(mapk::launch_sgemm(false, false, T, Dh, dp, 1.f, dpre, dp, Wf[ip], Dh, false, dh2, Dh, st));
-    CU_TRY(mapk::launch_sgemm(true, false, Dh, Dh, T, 1.f, dh2, Dh, h1, Dh, false, gout[i1 + 2], Dh, st));
+    MAP_TRY(run_mm(bwd[j]));                         // dW_p
+    MAP_TRY(run_mm(bwd[j + 1]));                     // dh2
+    MAP_TRY(run_mm(bwd[j + 2]));                     // dW2
     CU_TRY(mapk::launch_colsum(dh2, T, Dh, gout[i1 + 3], st));
-    CU_TRY(mapk::launch_sgemm(false, false, T, Dh, Dh, 1.f, dh2, Dh, Wf[i1 + 2], Dh, false, dh1, Dh, st));
+    MAP_TRY(run_mm(bwd[j + 3]));                     // dh1
     CU_TRY(mapk::launch_gelu_back(dh1, z1, T * Dh, st));
-    CU_TRY(mapk::launch_sgemm(true, false, Dh, D, T, 1.f, dh1, Dh, X, D, false, gout[i1], D, st));
+    MAP_TRY(run_mm(bwd[j + 4]));                     // dW1
     CU_TRY(mapk::launch_colsum(dh1, T, Dh, gout[i1 + 1], st));
     return MAP_OK;
   };
-  MAP_TRY(branch_bwd(dk, Tv, nullptr, g.rope_on ? N : 1, dkp, Vf, 5, z1v, h1v, h2v, dh2v, dh1v, 9));
-  MAP_TRY(branch_bwd(dq, Tt, g.rope_on ? post : nullptr, 1, dqp, Tf, 0, z1t, h1t, h2t, dh2t, dh1t, 4));
-  // query metadata, question-row images, 12 conversions, 2 x 6 forward, B logits, 4 loss /
-  // softmax-backward kernels, 2B logits backward, 2 x 9 branch backward
-  c->counters.launches += (B + 1023) / 1024 + (total_m + 2047) / 2048 + 12 + 12 + 3LL * B + 4 + 18;
+  MAP_TRY(bwd_tail(0, dk, Tv, nullptr, g.rope_on ? N : 1, dkp, z1v, dh2v, dh1v, 5));
+  MAP_TRY(bwd_tail(5, dq, Tt, g.rope_on ? post : nullptr, 1, dqp, z1t, dh2t, dh1t, 0));
+  // query metadata, question-row images, 4 bias conversions, 3 launches per contraction (two
+  // operand stagings, the GEMM), 2 x 3 forward elementwise, 4 loss / softmax-backward kernels,
+  // 2 x 5 backward elementwise
+  c->counters.launches += (B + 1023) / 1024 + (total_m + 2047) / 2048 + 4 + 3 * n_mm + 6 + 4 + 10;
   return MAP_OK;
 }
 
@@ -973,16 +1016,21 @@ void map_destroy(map_ctx* ctx) {
   for (void* p : {ctx->wqt, ctx->wkv, static_cast<void*>(ctx->bqt), static_cast<void*>(ctx->bkv)})
     if (p) cudaFree(p);
   DevBuf* bufs[] = {&ctx->rope, &ctx->h1, &ctx->kb, &ctx->th1, &ctx->qb, &ctx->stats,
-                    &ctx->qoff, &ctx->post, &ctx->sqn, &ctx->pmean, &ctx->snv, &ctx->dist, &ctx->sU, &ctx->sr2, &ctx->scstep, &ctx->sstate,
+                    &ctx->qoff, &ctx->post, &ctx->sqn, &ctx->pmean, &ctx->snv, &ctx->dist, &ctx->dsa, &ctx->dsb, &ctx->sU, &ctx->sr2, &ctx->scstep, &ctx->sstate,
                     &ctx->sEc, &ctx->spicks, &ctx->sr0, &ctx->sbt, &ctx->srn, &ctx->ssmall, &ctx->stheta,
                     &ctx->saslot, &ctx->sVg, &ctx->sG, &ctx->pvis, &ctx->ptext, &ctx->pout, &ctx->pkeep,
                     &ctx->pscores};
   for (DevBuf* b : bufs) release(*b);
   if (ctx->status) cudaFree(ctx->status);
+  if (ctx->loop_iters_total) cudaFree(ctx->loop_iters_total);
+  mapk::sel_loop_cache_destroy(ctx->loops);
   if (ctx->h_status) cudaFreeHost(ctx->h_status);
   if (ctx->h_done) cudaFreeHost(ctx->h_done);
   if (ctx->s_in) cudaStreamDestroy(ctx->s_in);
   if (ctx->s_out) cudaStreamDestroy(ctx->s_out);
+  if (ctx->s_aux) cudaStreamDestroy(ctx->s_aux);
+  if (ctx->ev_fork) cudaEventDestroy(ctx->ev_fork);
+  if (ctx->ev_join) cudaEventDestroy(ctx->ev_join);
   for (auto& pr : ctx->pairs) { cudaEventDestroy(pr.a); cudaEventDestroy(pr.b); }
   for (auto e : ctx->free_events) cudaEventDestroy(e);
   delete ctx;
@@ -1004,6 +1052,18 @@ const char* map_strerror(int code) {
 int map_get_counters(map_ctx* ctx, map_counters* out) {
   if (!ctx || !out) return MAP_EINVAL;
   *out = ctx->counters;
+  long long iters = 0;   // iterations of the device-side selection loop (completed work)
+  if (cudaSetDevice(ctx->device) != cudaSuccess ||
+      cudaMemcpy(&iters, ctx->loop_iters_total, sizeof(iters), cudaMemcpyDeviceToHost) != cudaSuccess)
+    return MAP_ECUDA;
+  out->launches += mapk::kSelLoopKernelsPerIter * iters;
+  out->select_rounds += 2 * iters;
+  return MAP_OK;
+}
+
+int map_set_wait_limit(map_ctx* ctx, long long ns) {
+  if (!ctx) return MAP_EINVAL;
+  ctx->wait_ns = ns > 0 ? ns : 0;
   return MAP_OK;
 }
 

@@ -3,14 +3,20 @@
 // QCTS selected, and its gradient with respect to every predictor weight (the backward pass
 // through Eq. 3's softmax-mean, RoPE, the projections and both MLPs).
 //
-// Everything is fp32 (the bf16 features and weights are decoded exactly): the gradient is
-// checked against a float64 oracle, and the training step is off the inference path.  The
-// contractions run on one tiled SIMT GEMM with either operand transposed (64 x 64 tiles,
-// 4 x 4 outputs per thread, fixed summation order); the softmax, KL, RoPE and GELU steps
-// and their derivatives are elementwise or row/column reductions in their own kernels, with
-// fixed-order (deterministic) reductions.
+// Activations and gradients are fp32 (the bf16 features and weights are decoded exactly): the
+// gradient is checked against a float64 oracle.  The contractions run on the tcgen05 GEMM of
+// gemm_tc.cu with split-bf16 operands: an fp32 operand x is staged as hi = bf16(x) and
+// lo = bf16(x - hi) (about 16 significant bits), a bf16 feature or weight as itself, and the
+// product is formed from the terms that carry fp32-level weight (hi.hi + hi.lo + lo.hi for two
+// fp32 operands, hi.b + lo.b against an exact bf16 one), accumulated in fp32 in TMEM.  The
+// staging kernels also transpose, so that both operands are K-major whichever index the
+// contraction runs over (tokens for the weight gradients).  The softmax, KL, RoPE and GELU
+// steps and their derivatives are elementwise or row/column reductions in their own kernels,
+// with fixed-order (deterministic) reductions.
 #include <cmath>
 #include <cstdint>
+
+#include <cuda_bf16.h>
 
 #include "kernels.h"
 #include "ptx.cuh"
@@ -18,66 +24,48 @@
 namespace mapk {
 namespace {
 
-constexpr int kGT = 64, kGK = 16;
-
-// C[i, j] = alpha sum_k A(i, k) B(k, j) (+ C[i, j] when accumulate), row-major storage:
-// A(i, k) = TA ? A[k lda + i] : A[i lda + k];  B(k, j) = TB ? B[j ldb + k] : B[k ldb + j].
-template <bool TA, bool TB>
-__global__ void __launch_bounds__(256) sgemm_kernel(int M, int N, int K, float alpha, const float* __restrict__ A,
-                                                    long long lda, const float* __restrict__ B, long long ldb,
-                                                    int accumulate, float* __restrict__ C, long long ldc) {
-  __shared__ __align__(16) float As[kGK][kGT + 4];
-  __shared__ __align__(16) float Bs[kGK][kGT + 4];
+// Operand staging for the tensor-core GEMM.  Element (r, c) of the logical matrix X (r < rows,
+// c < cols; X(r, c) = src[c * ld + r] when TRANS, else src[r * ld + c]; times alpha) is written to
+// row r of dst (row stride ldd elements) as hi = bf16(x) at columns hi0 + c and, if hi1 >= 0,
+// hi1 + c, and as lo = bf16(x - hi) at column lo0 + c if lo0 >= 0; columns cols .. kpad - 1 of
+// each segment are written as zeros.  32 x 32 tiles through shared memory, so that the reads
+// (along the source's contiguous index) and the writes (along c) are both coalesced.  BF16:
+// the source holds bf16 bit patterns (then lo = 0 when alpha = 1).
+template <bool TRANS, bool BF16>
+__global__ void __launch_bounds__(256) split_operand_kernel(const void* __restrict__ src, long long ld, int rows,
+                                                            int cols, int kpad, float alpha,
+                                                            uint16_t* __restrict__ dst, long long ldd, int hi0,
+                                                            int hi1, int lo0) {
+  __shared__ float t[32][33];                        // t[c - c0][r - r0]
   pdl_enter();
-  const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
-  const int i0 = blockIdx.x * kGT, j0 = blockIdx.y * kGT;   // rows along x: up to 2^31 - 1 tiles
-  float acc[4][4];
+  const int c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
+  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+  auto load = [&](long long i) -> float {
+    if constexpr (BF16) return __uint_as_float(static_cast<uint32_t>(static_cast<const uint16_t*>(src)[i]) << 16);
+    else return static_cast<const float*>(src)[i];
+  };
 #pragma unroll
-  for (int r = 0; r < 4; ++r)
-#pragma unroll
-    for (int c = 0; c < 4; ++c) acc[r][c] = 0.f;
-  for (int k0 = 0; k0 < K; k0 += kGK) {
-#pragma unroll
-    for (int e = threadIdx.x; e < kGT * kGK; e += 256) {
-      // consecutive threads walk the operand's contiguous dimension
-      const int ii = TA ? e % kGT : e / kGK, kk = TA ? e / kGT : e % kGK;
-      const int gi = i0 + ii, gk = k0 + kk;
-      float v = 0.f;
-      if (gi < M && gk < K) v = TA ? A[static_cast<long long>(gk) * lda + gi] : A[static_cast<long long>(gi) * lda + gk];
-      As[kk][ii] = v;
+  for (int i = ty; i < 32; i += 8) {
+    if (TRANS) {                                     // consecutive threads: consecutive r
+      const int r = r0 + tx, c = c0 + i;
+      t[i][tx] = (r < rows && c < cols) ? load(static_cast<long long>(c) * ld + r) : 0.f;
+    } else {                                         // consecutive threads: consecutive c
+      const int r = r0 + i, c = c0 + tx;
+      t[tx][i] = (r < rows && c < cols) ? load(static_cast<long long>(r) * ld + c) : 0.f;
     }
-#pragma unroll
-    for (int e = threadIdx.x; e < kGT * kGK; e += 256) {
-      const int jj = TB ? e / kGK : e % kGT, kk = TB ? e % kGK : e / kGT;
-      const int gj = j0 + jj, gk = k0 + kk;
-      float v = 0.f;
-      if (gj < N && gk < K) v = TB ? B[static_cast<long long>(gj) * ldb + gk] : B[static_cast<long long>(gk) * ldb + gj];
-      Bs[kk][jj] = v;
-    }
-    __syncthreads();
-#pragma unroll
-    for (int kk = 0; kk < kGK; ++kk) {
-      const float4 a = *reinterpret_cast<const float4*>(&As[kk][ty * 4]);
-      const float4 b = *reinterpret_cast<const float4*>(&Bs[kk][tx * 4]);
-      const float av[4] = {a.x, a.y, a.z, a.w}, bv[4] = {b.x, b.y, b.z, b.w};
-#pragma unroll
-      for (int r = 0; r < 4; ++r)
-#pragma unroll
-        for (int c = 0; c < 4; ++c) acc[r][c] = fmaf(av[r], bv[c], acc[r][c]);
-    }
-    __syncthreads();
   }
+  __syncthreads();
 #pragma unroll
-  for (int r = 0; r < 4; ++r) {
-    const int i = i0 + ty * 4 + r;
-    if (i >= M) continue;
-#pragma unroll
-    for (int c = 0; c < 4; ++c) {
-      const int j = j0 + tx * 4 + c;
-      if (j >= N) continue;
-      float* o = C + static_cast<long long>(i) * ldc + j;
-      *o = accumulate ? *o + alpha * acc[r][c] : alpha * acc[r][c];
-    }
+  for (int i = ty; i < 32; i += 8) {
+    const int r = r0 + i, c = c0 + tx;
+    if (r >= rows || c >= kpad) continue;
+    const float x = t[tx][i] * alpha;
+    const __nv_bfloat16 h = __float2bfloat16_rn(x);
+    uint16_t* row = dst + static_cast<long long>(r) * ldd;
+    const uint16_t hb = __bfloat16_as_ushort(h);
+    row[hi0 + c] = hb;
+    if (hi1 >= 0) row[hi1 + c] = hb;
+    if (lo0 >= 0) row[lo0 + c] = __bfloat16_as_ushort(__float2bfloat16_rn(x - __bfloat162float(h)));
   }
 }
 
@@ -177,10 +165,10 @@ __device__ __forceinline__ float block_max(float v, float* red) {
 }
 
 // One CTA per question row: logits row -> softmax over the N visual tokens, in place.
-__global__ void __launch_bounds__(kRowThreads) row_softmax_kernel(float* __restrict__ L, int N) {
+__global__ void __launch_bounds__(kRowThreads) row_softmax_kernel(float* __restrict__ L, long long ld, int N) {
   __shared__ float red[kRowThreads / 32 + 1];
   pdl_enter();
-  float* row = L + static_cast<long long>(blockIdx.x) * N;
+  float* row = L + static_cast<long long>(blockIdx.x) * ld;
   float m = -INFINITY;
   for (int n = threadIdx.x; n < N; n += kRowThreads) m = fmaxf(m, row[n]);
   m = block_max(m, red);
@@ -193,7 +181,8 @@ __global__ void __launch_bounds__(kRowThreads) row_softmax_kernel(float* __restr
 
 // Per image b (grid.y) and column block: p_hat[n] = mean_m s[m, n]; g[n] = -p*[n] / (B p_hat[n]);
 // the block's share of D_KL(p* || p_hat) goes to part[b * nblk + blockIdx.x].
-__global__ void __launch_bounds__(kRowThreads) phat_kl_kernel(const float* __restrict__ S, const int32_t* __restrict__ qoff,
+__global__ void __launch_bounds__(kRowThreads) phat_kl_kernel(const float* __restrict__ S, long long ld,
+                                                              const int32_t* __restrict__ qoff,
                                                               const float* __restrict__ teacher, int N, int B,
                                                               float* __restrict__ p_hat, float* __restrict__ g,
                                                               float* __restrict__ part) {
@@ -204,9 +193,9 @@ __global__ void __launch_bounds__(kRowThreads) phat_kl_kernel(const float* __res
   const int o = qoff[b], M = qoff[b + 1] - o;
   float kl = 0.f;
   if (n < N) {
-    const float* col = S + static_cast<long long>(o) * N + n;
+    const float* col = S + static_cast<long long>(o) * ld + n;
     float acc = 0.f;
-    for (int m = 0; m < M; ++m) acc += col[static_cast<long long>(m) * N];
+    for (int m = 0; m < M; ++m) acc += col[static_cast<long long>(m) * ld];
     const float ph = acc / static_cast<float>(M);
     const float ps = teacher[static_cast<long long>(b) * N + n];
     p_hat[static_cast<long long>(b) * N + n] = ph;
@@ -229,7 +218,8 @@ __global__ void loss_reduce_kernel(const float* __restrict__ part, int n, int B,
 
 // One CTA per question row m of image b (row_img[m]): softmax backward of the mean,
 //   dl[m, n] = s[m, n] (g[n] - sum_n' s[m, n'] g[n']) / M_b, written over s.
-__global__ void __launch_bounds__(kRowThreads) softmax_back_kernel(float* __restrict__ S, const int32_t* __restrict__ qoff,
+__global__ void __launch_bounds__(kRowThreads) softmax_back_kernel(float* __restrict__ S, long long ld,
+                                                                   const int32_t* __restrict__ qoff,
                                                                    const int32_t* __restrict__ row_img,
                                                                    const float* __restrict__ g, int N) {
   __shared__ float red[kRowThreads / 32 + 1];
@@ -237,7 +227,7 @@ __global__ void __launch_bounds__(kRowThreads) softmax_back_kernel(float* __rest
   const long long m = blockIdx.x;
   const int b = row_img[m];
   const float inv_m = 1.0f / static_cast<float>(qoff[b + 1] - qoff[b]);
-  float* row = S + m * N;
+  float* row = S + m * ld;
   const float* gb = g + static_cast<long long>(b) * N;
   float c = 0.f;
   for (int n = threadIdx.x; n < N; n += kRowThreads) c += row[n] * gb[n];
@@ -277,16 +267,69 @@ unsigned grid_for(long long n) {
 
 }  // namespace
 
-cudaError_t launch_sgemm(bool ta, bool tb, int M, int N, int K, float alpha, const float* A, long long lda,
-                         const float* B, long long ldb, bool accumulate, float* C, long long ldc, cudaStream_t st) {
-  if (M <= 0 || N <= 0) return cudaSuccess;
-  const dim3 grid((M + kGT - 1) / kGT, (N + kGT - 1) / kGT);
-  if (grid.y > 65535) return cudaErrorInvalidValue;
-  const int acc = accumulate ? 1 : 0;
-  if (!ta && !tb) return launch_k(sgemm_kernel<false, false>, grid, dim3(256), 0, st, M, N, K, alpha, A, lda, B, ldb, acc, C, ldc);
-  if (!ta && tb) return launch_k(sgemm_kernel<false, true>, grid, dim3(256), 0, st, M, N, K, alpha, A, lda, B, ldb, acc, C, ldc);
-  if (ta && !tb) return launch_k(sgemm_kernel<true, false>, grid, dim3(256), 0, st, M, N, K, alpha, A, lda, B, ldb, acc, C, ldc);
-  return launch_k(sgemm_kernel<true, true>, grid, dim3(256), 0, st, M, N, K, alpha, A, lda, B, ldb, acc, C, ldc);
+namespace {
+
+struct TcPlan {
+  int Kp, ka, kb, kprime;   // padded K, staged widths of A and B, GEMM K
+  bool a_split, b_split;
+};
+
+TcPlan tc_plan(int K, float alpha, bool a_bf16, bool b_bf16) {
+  TcPlan p;
+  p.Kp = ((K + 63) / 64) * 64;
+  p.a_split = !(a_bf16 && alpha == 1.0f);
+  p.b_split = !b_bf16;
+  if (!p.a_split && !p.b_split) { p.ka = p.kb = p.kprime = p.Kp; }          // a.b
+  else if (p.a_split && p.b_split) { p.ka = 2 * p.Kp; p.kb = p.kprime = 3 * p.Kp; }   // ah.bh + ah.bl + al.bh
+  else { p.ka = p.kb = p.kprime = 2 * p.Kp; }                                  // ah.b + al.b (or a.bh + a.bl)
+  return p;
+}
+
+cudaError_t stage(const void* src, bool bf16, bool trans, long long ld, int rows, int cols, int kpad, float alpha,
+                  uint16_t* dst, long long ldd, int hi0, int hi1, int lo0, cudaStream_t st) {
+  const dim3 grid((kpad + 31) / 32, (rows + 31) / 32);
+  if (grid.y > 65535u) return cudaErrorInvalidValue;
+  if (trans) {
+    if (bf16) return launch_k(split_operand_kernel<true, true>, grid, dim3(256), 0, st, src, ld, rows, cols, kpad, alpha, dst, ldd, hi0, hi1, lo0);
+    return launch_k(split_operand_kernel<true, false>, grid, dim3(256), 0, st, src, ld, rows, cols, kpad, alpha, dst, ldd, hi0, hi1, lo0);
+  }
+  if (bf16) return launch_k(split_operand_kernel<false, true>, grid, dim3(256), 0, st, src, ld, rows, cols, kpad, alpha, dst, ldd, hi0, hi1, lo0);
+  return launch_k(split_operand_kernel<false, false>, grid, dim3(256), 0, st, src, ld, rows, cols, kpad, alpha, dst, ldd, hi0, hi1, lo0);
+}
+
+}  // namespace
+
+void tc_matmul_ws(int M, int N, int K, float alpha, bool a_bf16, bool b_bf16, size_t* a_elems, size_t* b_elems) {
+  const TcPlan p = tc_plan(K, alpha, a_bf16, b_bf16);
+  *a_elems = static_cast<size_t>(M) * p.ka;
+  *b_elems = static_cast<size_t>(N) * p.kb;
+}
+
+cudaError_t launch_tc_matmul(bool ta, bool tb, int M, int N, int K, float alpha, const void* A, bool a_bf16,
+                             long long lda, const void* B, bool b_bf16, long long ldb, float* C, long long ldc,
+                             void* wsA, void* wsB, int num_sms, int* status, long long wait_ns, cudaStream_t st) {
+  if (M <= 0 || N <= 0 || K <= 0) return cudaSuccess;
+  const TcPlan p = tc_plan(K, alpha, a_bf16, b_bf16);
+  uint16_t* As = static_cast<uint16_t*>(wsA);
+  uint16_t* Bs = static_cast<uint16_t*>(wsB);
+  // A_s(i, k) = A(i, k): a transposed read when ta.  B_s(j, k) = B(k, j): transposed unless tb.
+  const int a_hi1 = (!p.a_split && p.b_split) ? p.Kp : -1, a_lo = p.a_split ? p.Kp : -1;
+  cudaError_t e = stage(A, a_bf16, ta, lda, M, K, p.Kp, alpha, As, p.ka, 0, a_hi1, a_lo, st);
+  if (e != cudaSuccess) return e;
+  int b_hi1 = -1, b_lo = -1;
+  if (p.a_split && p.b_split) { b_hi1 = p.Kp; b_lo = 2 * p.Kp; }
+  else if (p.a_split) { b_hi1 = p.Kp; }
+  else if (p.b_split) { b_lo = p.Kp; }
+  e = stage(B, b_bf16, !tb, ldb, N, K, p.Kp, 1.0f, Bs, p.kb, 0, b_hi1, b_lo, st);
+  if (e != cudaSuccess) return e;
+  GemmDesc d{};
+  d.A = As; d.a_rows_total = M; d.a_row_stride = 0;
+  d.B = Bs; d.b_rows_total = N; d.b_row_stride = 0;
+  d.M = M; d.N = N; d.K = p.kprime; d.batch = 1;
+  d.C = C; d.ldc = ldc; d.c_batch_stride = 0;
+  d.epi = EPI_F32; d.status = status; d.wait_ns = wait_ns;
+  if (p.a_split && p.b_split) { d.split3 = 1; d.a_kwrap = 2 * p.Kp; }
+  return launch_gemm(d, num_sms, st);
 }
 
 cudaError_t launch_bf16_to_f32(const void* x, long long n, float* y, cudaStream_t st) {
@@ -311,18 +354,18 @@ cudaError_t launch_rope_f32(bool backward, const float* x, long long rows, int d
                   pos_mod, y);
 }
 
-cudaError_t launch_distill_loss_grad(float* S, long long total_m, const int32_t* qoff, const int32_t* row_img,
-                                     const float* teacher, int B, int N, float* p_hat, float* g, float* part,
-                                     float* loss, cudaStream_t st) {
-  cudaError_t e = launch_k(row_softmax_kernel, dim3(static_cast<unsigned>(total_m)), dim3(kRowThreads), 0, st, S, N);
+cudaError_t launch_distill_loss_grad(float* S, long long ld, long long total_m, const int32_t* qoff,
+                                     const int32_t* row_img, const float* teacher, int B, int N, float* p_hat,
+                                     float* g, float* part, float* loss, cudaStream_t st) {
+  cudaError_t e = launch_k(row_softmax_kernel, dim3(static_cast<unsigned>(total_m)), dim3(kRowThreads), 0, st, S, ld, N);
   if (e != cudaSuccess) return e;
   const int nblk = (N + kRowThreads - 1) / kRowThreads;
-  e = launch_k(phat_kl_kernel, dim3(nblk, B), dim3(kRowThreads), 0, st, static_cast<const float*>(S), qoff, teacher,
-               N, B, p_hat, g, part);
+  e = launch_k(phat_kl_kernel, dim3(nblk, B), dim3(kRowThreads), 0, st, static_cast<const float*>(S), ld, qoff,
+               teacher, N, B, p_hat, g, part);
   if (e != cudaSuccess) return e;
   e = launch_k(loss_reduce_kernel, dim3(1), dim3(32), 0, st, static_cast<const float*>(part), nblk * B, B, loss);
   if (e != cudaSuccess) return e;
-  return launch_k(softmax_back_kernel, dim3(static_cast<unsigned>(total_m)), dim3(kRowThreads), 0, st, S, qoff,
+  return launch_k(softmax_back_kernel, dim3(static_cast<unsigned>(total_m)), dim3(kRowThreads), 0, st, S, ld, qoff,
                   row_img, static_cast<const float*>(g), N);
 }
 

@@ -18,8 +18,9 @@
 //               thread), apply bias / GELU / RoPE, store (bf16, bf16 hi/lo pair, or fp32);
 //               release the accumulator so the
 //               MMA warp can start the tile after next while this one drains.
-//   EPI_PROJECT: the MMA thread also accumulates A A^T (N = 128) of every stage into a second
-//               TMEM accumulator, whose diagonal is ||row||^2.
+//   EPI_PROJECT: two more warps (6-7) read every staged A tile and sum each row's squares
+//               (||v||^2) on the CUDA cores; they release the stage together with the MMA
+//               commit and hand the tile's norms to the epilogue with the accumulator.
 // All waits are bounded (ptx.cuh); a timeout sets ST_TIMEOUT and every role drains and exits.
 #include <algorithm>
 #include <cstdio>
@@ -54,6 +55,7 @@ struct KArgs {
   const float* biasf;
   const int* blist; const int* bcount;
   const int* m_limit;
+  unsigned long long wait_ns;   // limit of the role waits (the drain waits keep kWaitLimitNs)
 };
 
 __device__ __forceinline__ float gelu_erf(float x) {
@@ -83,9 +85,10 @@ struct Smem {
   static constexpr uint32_t STG = TSTORE ? 4 * 4 * 32 * 32 * 2 : 0;
   static constexpr uint32_t LSM = PROJ ? BN * BN * 4 : 0;       // L rows of the basis (pitch BN)
   static constexpr uint32_t PEXTRA = PROJ ? BN * 4 : 0;          // 1/r of the basis
-  static constexpr uint32_t TOTAL = 1024 + TILES + STG + BARS + 16 + XPOSE + LSM + PEXTRA;
-  static constexpr uint32_t TMEM_COLS = PROJ ? (2 * BN + 2 * kBM <= 256 ? 256u : 512u) : 2 * BN;   // + A A^T
-  static constexpr int THREADS = 192;
+  static constexpr uint32_t NSQ = PROJ ? 2 * kBM * 4 : 0;        // ||row||^2 of a tile, per accumulator
+  static constexpr uint32_t TOTAL = 1024 + TILES + STG + BARS + 16 + XPOSE + LSM + PEXTRA + NSQ;
+  static constexpr uint32_t TMEM_COLS = PROJ ? (2 * BN <= 256 ? 256u : 512u) : 2 * BN;
+  static constexpr int THREADS = PROJ ? 256 : 192;               // + 2 row-norm warps
 };
 
 // Selection value, squared: p^2 * rho^(2 lambda) orders candidates like p * rho^lambda (both are
@@ -144,12 +147,16 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   float* xpose = reinterpret_cast<float*>(smem + S::TILES + S::STG + S::BARS + 16);
   float* Lsm = xpose + S::XPOSE / 4;
   float* rinv_sm = Lsm + S::LSM / 4;
+  float* sqn_sm = rinv_sm + S::PEXTRA / 4;         // EPI_PROJECT: [2][kBM] row norms per accumulator
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
-    for (int s = 0; s < STAGES; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
+    // EPI_PROJECT: a stage is free once the MMA commit and both row-norm warps have arrived, and
+    // an accumulator is full once the MMA commit and both row-norm warps (its norms) have
+    constexpr uint32_t kArrive = S::PROJ ? 3 : 1;
+    for (int s = 0; s < STAGES; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], kArrive); }
     // tempty: one arrive per epilogue warp (of both CTAs with CG2, on the leader's barrier)
-    for (int i = 0; i < 2; ++i) { mbar_init(&tfull[i], 1); mbar_init(&tempty[i], CG2 ? 8 : 4); }
+    for (int i = 0; i < 2; ++i) { mbar_init(&tfull[i], kArrive); mbar_init(&tempty[i], CG2 ? 8 : 4); }
     mbar_init(drain, 1);
     if constexpr (S::PROJ) {
       mbar_init(egsync, 128);
@@ -190,13 +197,14 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     }
   };
 
+  // Producer: parity of the last load issued into each stage (-1: none), for the drain below.
+  int last_par[STAGES];
+#pragma unroll
+  for (int s = 0; s < STAGES; ++s) last_par[s] = -1;
   if (warp == 0) {
     if (lane == 0) {
       // ---------------------------------------------------------------- TMA producer
       uint32_t stage = 0, phase = 0;
-      int last_par[STAGES];
-#pragma unroll
-      for (int s = 0; s < STAGES; ++s) last_par[s] = -1;
       bool ok = true;
       for (int t = unit0; t < total && ok; t += units_step) {
         TileCoord c = tile_coord<PAIR>(a, t, m_units, n_tiles, BN, crank);
@@ -204,7 +212,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         const int arow = c.b * a.a_row_stride + c.m_blk * kBM;
         const int brow = (a.b_off ? __ldg(a.b_off + c.b) : c.b * a.b_row_stride + a.b_base) + c.n_blk * BN;
         for (int kb = 0; kb < KB; ++kb) {
-          if (!mbar_wait(&empty[stage], phase ^ 1, a.status, abort_flag)) { ok = false; break; }
+          if (!mbar_wait(&empty[stage], phase ^ 1, a.status, abort_flag, a.wait_ns)) { ok = false; break; }
           int ac, bc;
           kcols(kb, ac, bc);
           if constexpr (CG2) {
@@ -222,10 +230,6 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           if (++stage == STAGES) { stage = 0; phase ^= 1; }
         }
       }
-      if (!ok && crank == 0) {   // let every copy already in flight land before the CTA exits
-        for (int s = 0; s < STAGES; ++s)
-          if (last_par[s] >= 0) mbar_wait(&full[s], static_cast<uint32_t>(last_par[s]), a.status, nullptr);
-      }
     }
     __syncwarp();
   } else if (warp == 1) {
@@ -236,11 +240,11 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       for (int t = unit0; t < total && ok; t += units_step) {
         TileCoord c = tile_coord<PAIR>(a, t, m_units, n_tiles, BN, crank);
         if (c.skip) continue;
-        if (!mbar_wait(&tempty[acc], acc_phase ^ 1, a.status, abort_flag)) break;
+        if (!mbar_wait(&tempty[acc], acc_phase ^ 1, a.status, abort_flag, a.wait_ns)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + acc * BN;
         for (int kb = 0; kb < KB; ++kb) {
-          if (!mbar_wait(&full[stage], phase, a.status, abort_flag)) { ok = false; break; }
+          if (!mbar_wait(&full[stage], phase, a.status, abort_flag, a.wait_ns)) { ok = false; break; }
           tc_fence_after();
           const uint32_t a0 = smem_u32(sA + stage * S::A_BYTES);
           const uint32_t b0 = smem_u32(sB + stage * S::B_BYTES);
@@ -253,13 +257,6 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
 #pragma unroll
             for (int k = 0; k < kBK / 16; ++k)
               umma_bf16(d_tmem, desc_sw128(a0 + k * 32), desc_sw128(b0 + k * 32), IDESC, (kb | k) != 0);
-            if constexpr (S::PROJ) {   // A A^T: its diagonal is ||row||^2
-              const uint32_t n_tmem = tmem_base + 2 * BN + acc * kBM;
-#pragma unroll
-              for (int k = 0; k < kBK / 16; ++k)
-                umma_bf16(n_tmem, desc_sw128(a0 + k * 32), desc_sw128(a0 + k * 32), idesc_bf16(kBM, kBM),
-                          (kb | k) != 0);
-            }
             umma_commit(&empty[stage]);
           }
           issued = true;
@@ -278,6 +275,50 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       }
     }
     __syncwarp();
+  } else if (S::PROJ && warp >= 6) {
+    // ------------------------------------------------------------------ row norms (EPI_PROJECT)
+    // Warp 6 sums rows 0-63 of every staged A tile, warp 7 rows 64-127, two rows per lane.  A
+    // row's 64 values are its own 128-byte line in the 128-byte swizzle (only the 16-byte
+    // chunks are permuted), so lane l reads physical chunk c ^ (row & 7) at step c: the eight
+    // rows of a quarter warp hit distinct banks, and the order of a sum is not an issue.
+    const int r0 = (warp - 6) * 64 + lane, r1 = r0 + 32;
+    uint32_t stage = 0, phase = 0, acc = 0, acc_phase = 0;
+    for (int t = unit0; t < total; t += units_step) {
+      TileCoord c = tile_coord<PAIR>(a, t, m_units, n_tiles, BN, crank);
+      if (c.skip) continue;
+      if (!mbar_wait(&tempty[acc], acc_phase ^ 1, a.status, abort_flag, a.wait_ns)) break;   // norms slot free
+      float s0 = 0.f, s1 = 0.f;
+      bool ok = true;
+      for (int kb = 0; kb < KB; ++kb) {
+        if (!mbar_wait(&full[stage], phase, a.status, abort_flag, a.wait_ns)) { ok = false; break; }
+        const uint8_t* At = sA + stage * S::A_BYTES;
+#pragma unroll
+        for (int ch = 0; ch < 8; ++ch) {
+          const uint4 x0 = *reinterpret_cast<const uint4*>(At + r0 * 128 + ((ch ^ (r0 & 7)) << 4));
+          const uint4 x1 = *reinterpret_cast<const uint4*>(At + r1 * 128 + ((ch ^ (r1 & 7)) << 4));
+          const uint32_t w0[4] = {x0.x, x0.y, x0.z, x0.w}, w1[4] = {x1.x, x1.y, x1.z, x1.w};
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const float2 f0 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w0[u]));
+            const float2 f1 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w1[u]));
+            s0 = fmaf(f0.x, f0.x, s0);
+            s0 = fmaf(f0.y, f0.y, s0);
+            s1 = fmaf(f1.x, f1.x, s1);
+            s1 = fmaf(f1.y, f1.y, s1);
+          }
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&empty[stage]);
+        if (++stage == STAGES) { stage = 0; phase ^= 1; }
+      }
+      if (!ok) break;
+      sqn_sm[acc * kBM + r0] = s0;
+      sqn_sm[acc * kBM + r1] = s1;
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tfull[acc]);        // release: the norms are visible to the epilogue
+      acc ^= 1;
+      if (acc == 0) acc_phase ^= 1;
+    }
   } else if (warp < 6) {
     // ------------------------------------------------------------------ epilogue
     const int lane_grp = warp & 3;                 // TMEM lanes this warp may access
@@ -293,7 +334,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         if (c.b != staged_b) {                     // stage L and 1/r of this image's R0 basis
           // group barrier of the 128 epilogue threads (bounded, unlike a named barrier)
           mbar_arrive(egsync);
-          if (!mbar_wait(egsync, eg_phase, a.status, abort_flag)) { eg_ok = false; break; }
+          if (!mbar_wait(egsync, eg_phase, a.status, abort_flag, a.wait_ns)) { eg_ok = false; break; }
           eg_phase ^= 1;
           const ProjArgs& pj = a.proj;
           const int nb0 = min(BN, __ldg(pj.nbasis + c.b));
@@ -315,12 +356,12 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           for (int i = threadIdx.x - 64; i < nb0; i += 128)
             rinv_sm[i] = 1.0f / __ldg(pj.rnorm + static_cast<long long>(c.b) * pj.Kcap + i);
           mbar_arrive(egsync);
-          if (!mbar_wait(egsync, eg_phase, a.status, abort_flag)) { eg_ok = false; break; }
+          if (!mbar_wait(egsync, eg_phase, a.status, abort_flag, a.wait_ns)) { eg_ok = false; break; }
           eg_phase ^= 1;
           staged_b = c.b;
         }
       }
-      if (!mbar_wait(&tfull[acc], acc_phase, a.status, abort_flag)) break;
+      if (!mbar_wait(&tfull[acc], acc_phase, a.status, abort_flag, a.wait_ns)) break;
       tc_fence_after();
       const int row = c.m_blk * kBM + r_in_tile;
       const bool row_ok = row < (a.m_limit ? min(a.M, __ldg(a.m_limit + c.b)) : a.M);
@@ -548,13 +589,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         const long long tok = static_cast<long long>(c.b) * a.M + row;
         const bool alive = row_ok && __ldg(pj.state + tok) == 0;
         float* erow = pj.Ec + tok * pj.KP;
-        float sq = 0.f;
-        {
-          uint32_t dg[32];
-          tmem_ld32(tmem_base + (static_cast<uint32_t>(lane_grp * 32) << 16) + 2 * BN + acc * kBM + lane_grp * 32, dg);
-#pragma unroll
-          for (int j = 0; j < 32; ++j) sq = j == lane ? __uint_as_float(dg[j]) : sq;
-        }
+        const float sq = sqn_sm[acc * kBM + r_in_tile];
         float r2 = sq;
 #pragma unroll 1
         for (int b0 = 0; b0 < nb0; b0 += 32) {
@@ -743,6 +778,14 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       __syncwarp();
     }
   }
+  // Every role of this CTA has left its loop.  If one gave up (a bounded wait ran out), loads
+  // may still be in flight that no MMA waited for: let them land before the CTA exits.  With
+  // 2-SM pairs both CTAs' loads complete on the leader's barriers, which the leader drains.
+  __syncthreads();
+  if (*abort_flag && warp == 0 && lane == 0 && crank == 0) {
+    for (int s = 0; s < STAGES; ++s)
+      if (last_par[s] >= 0) mbar_wait(&full[s], static_cast<uint32_t>(last_par[s]), a.status, nullptr);
+  }
   if constexpr (PAIR) cluster_sync();             // no commit or remote arrive still in flight
   else __syncthreads();
   if (warp == 1) {
@@ -823,7 +866,7 @@ cudaError_t run(const GemmDesc& d, const KArgs& ka, int num_sms, cudaStream_t st
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
     attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    attr[1].val.programmaticStreamSerializationAllowed = pdl_disabled() ? 0 : 1;
     cfg.attrs = attr;
     cfg.numAttrs = 2;
     return cudaLaunchKernelEx(&cfg, kern, ta, tb, tc, ka);
@@ -868,6 +911,7 @@ cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t st) {
   ka.a_kwrap = d.a_kwrap; ka.biasf = d.biasf; ka.split3 = d.split3;
   ka.blist = d.blist; ka.bcount = d.blist ? d.bcount : nullptr;
   ka.m_limit = d.m_limit;
+  ka.wait_ns = d.wait_ns > 0 ? static_cast<unsigned long long>(d.wait_ns) : kWaitLimitNs;
   if (d.blist && !d.bcount) return cudaErrorInvalidValue;
   switch (d.epi) {
     case EPI_GELU_BF16:

@@ -76,6 +76,9 @@ struct GemmDesc {
   // Per-batch number of valid A rows (device) or nullptr: rows at or past it are treated as
   // absent (EPI_SM_STATS: excluded from the column statistics; EPI_SM_MEAN: output 0)
   const int* m_limit = nullptr;
+  // Limit (ns) of the producer / MMA / epilogue waits; 0 = the default 2 s.  The waits that
+  // let in-flight copies and MMAs land before an aborting CTA exits keep the default.
+  long long wait_ns = 0;
 };
 
 // Returns cudaSuccess, or an error for an unsupported shape (cudaErrorInvalidValue).
@@ -125,10 +128,15 @@ cudaError_t launch_assemble(const void* V, const int32_t* idx, const void* T, co
                             cudaStream_t st);
 
 // ------------------------------------------------------------------ distillation step (fp32)
-// C[i, j] = alpha sum_k A(i, k) B(k, j) (+ C when accumulate); row-major, A(i, k) = ta ? A[k lda + i]
-// : A[i lda + k], B(k, j) = tb ? B[j ldb + k] : B[k ldb + j].  Tiled SIMT, fixed summation order.
-cudaError_t launch_sgemm(bool ta, bool tb, int M, int N, int K, float alpha, const float* A, long long lda,
-                         const float* B, long long ldb, bool accumulate, float* C, long long ldc, cudaStream_t st);
+// C[i, j] = alpha sum_k A(i, k) B(k, j) on the tcgen05 GEMM, fp32 in (or bf16: a_bf16 / b_bf16)
+// and fp32 out; row-major, A(i, k) = ta ? A[k lda + i] : A[i lda + k], B(k, j) = tb ? B[j ldb + k]
+// : B[k ldb + j].  fp32 operands are staged as bf16 (hi, lo) pairs (split-bf16 products, see
+// distill.cu) in wsA / wsB, of at least the element counts tc_matmul_ws returns; C must be
+// 16-byte aligned with ldc % 4 == 0.  Deterministic (fixed summation order).
+void tc_matmul_ws(int M, int N, int K, float alpha, bool a_bf16, bool b_bf16, size_t* a_elems, size_t* b_elems);
+cudaError_t launch_tc_matmul(bool ta, bool tb, int M, int N, int K, float alpha, const void* A, bool a_bf16,
+                             long long lda, const void* B, bool b_bf16, long long ldb, float* C, long long ldc,
+                             void* wsA, void* wsB, int num_sms, int* status, long long wait_ns, cudaStream_t st);
 cudaError_t launch_bf16_to_f32(const void* x, long long n, float* y, cudaStream_t st);
 // z += b (per column); h = GELU(z)
 cudaError_t launch_bias_gelu(float* z, const float* b, long long rows, int cols, float* h, cudaStream_t st);
@@ -136,12 +144,13 @@ cudaError_t launch_bias_add(float* x, const float* b, long long rows, int cols, 
 // RoPE (or its transpose when backward) on [rows, d] fp32 rows; positions pos[r] or r % pos_mod.
 cudaError_t launch_rope_f32(bool backward, const float* x, long long rows, int d, const float2* tab, int ld,
                             const int32_t* pos, int pos_mod, float* y, cudaStream_t st);
-// S [total_m, N] logits of all images' question rows (image b: rows qoff[b] .. qoff[b+1]) ->
-// softmax, p_hat [B, N], g = dL/dp_hat, *loss = mean_b D_KL(teacher_b || p_hat_b), then S is
-// overwritten with dL/dlogits.  row_img [total_m]: image of each row; part: B * ceil(N/256) floats.
-cudaError_t launch_distill_loss_grad(float* S, long long total_m, const int32_t* qoff, const int32_t* row_img,
-                                     const float* teacher, int B, int N, float* p_hat, float* g, float* part,
-                                     float* loss, cudaStream_t st);
+// S [total_m, N] logits of all images' question rows (row stride ld; image b: rows qoff[b] ..
+// qoff[b+1]) -> softmax, p_hat [B, N], g = dL/dp_hat, *loss = mean_b D_KL(teacher_b || p_hat_b),
+// then S is overwritten with dL/dlogits.  row_img [total_m]: image of each row; part: B * ceil(N/256)
+// floats.
+cudaError_t launch_distill_loss_grad(float* S, long long ld, long long total_m, const int32_t* qoff,
+                                     const int32_t* row_img, const float* teacher, int B, int N, float* p_hat,
+                                     float* g, float* part, float* loss, cudaStream_t st);
 // dh *= GELU'(z)
 cudaError_t launch_gelu_back(float* dh, const float* z, long long n, cudaStream_t st);
 // out[c] = sum_r X[r, c]

@@ -59,16 +59,16 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 // Wait until the phase with the given parity has completed.  Bounded: returns false
-// (and sets ST_TIMEOUT in *status) after kWaitLimitNs, or at once if *abort is set.
+// (and sets ST_TIMEOUT in *status) after limit_ns, or at once if *abort is set.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* status,
-                                          volatile int* abort) {
+                                          volatile int* abort, unsigned long long limit_ns = kWaitLimitNs) {
   if (mbar_try_wait(bar, parity)) return true;
   unsigned long long t0 = global_ns();
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
-    if ((it & 255u) == 0) {
+    if ((it & 15u) == 0) {
       if (abort != nullptr && *abort) return false;
-      if (global_ns() - t0 > kWaitLimitNs) {
+      if (global_ns() - t0 > limit_ns) {
         if (status) atomicOr(status, ST_TIMEOUT);
         if (abort != nullptr) *abort = 1;
         return false;
@@ -289,6 +289,14 @@ __device__ __forceinline__ void pdl_enter() {
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
+// Programmatic dependent launch is turned off (per host thread) while kernels are captured
+// into the body of a conditional graph node; the kernels' griddepcontrol instructions are then
+// no-ops and the graph's ordinary edges order them.
+inline bool& pdl_disabled() {
+  static thread_local bool off = false;
+  return off;
+}
+
 // Launch with the programmatic-serialisation attribute (the next kernel may be scheduled
 // early; its pdl_enter() orders it after this one); extra attributes are appended.
 template <typename... KParams, typename... Args>
@@ -301,7 +309,7 @@ cudaError_t launch_k(void (*kern)(KParams...), dim3 grid, dim3 block, size_t sme
   cfg.stream = st;
   cudaLaunchAttribute at[1];
   at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  at[0].val.programmaticStreamSerializationAllowed = 1;
+  at[0].val.programmaticStreamSerializationAllowed = pdl_disabled() ? 0 : 1;
   cfg.attrs = at;
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);

@@ -30,7 +30,10 @@
 // The result equals the eager fp32 greedy whatever s is; s only changes how much work is
 // batched.
 #include <algorithm>
+#include <cstring>
+#include <vector>
 
+#include "kernels.h"
 #include "ptx.cuh"
 #include "select.h"
 
@@ -45,6 +48,13 @@ __device__ __forceinline__ uint64_t make_key(float v, int idx) {
 __device__ __forceinline__ int key_index(uint64_t key) {
   return static_cast<int>(0xFFFFFFFFu - static_cast<uint32_t>(key & 0xFFFFFFFFull));
 }
+
+// The caller's buffers: through s.uptr when set (the cached loop graph was built for another
+// call's pointers), else the fields themselves.
+__device__ __forceinline__ const float* sel_scores(const SelState& s) {
+  return s.uptr ? static_cast<const float*>(s.uptr[0]) : s.scores;
+}
+__device__ __forceinline__ const void* sel_features(const SelState& s) { return s.uptr ? s.uptr[1] : s.V; }
 
 // Selection value, squared: p^2 * rho^(2 lambda) orders candidates like p * rho^lambda (both are
 // >= 0) and needs no square root for lambda = 1.  rho^2 = r2 unless r2 <= tau ||v||^2 (then 0).
@@ -188,6 +198,7 @@ __global__ void __launch_bounds__(1024) sel_init_kernel(SelState s) {
   if (b == 0 && threadIdx.x == 0) {   // counters of this selection (earlier readers have completed)
     if (s.bcount) { s.bcount[0] = 0; s.bcount[1] = 0; }
     if (s.done_count) *s.done_count = 0;
+    if (s.uptr) { s.uptr[0] = s.scores; s.uptr[1] = s.V; }
   }
   if (threadIdx.x == 0) {
     s.npicks[b] = 0; s.nbasis[b] = 0; s.nb_gathered[b] = 0; s.done[b] = 0; s.nlimit[b] = 0;
@@ -286,7 +297,7 @@ __global__ void __launch_bounds__(kGatherThreads) sel_gather_kernel(SelState s) 
       if (beta >= lo && beta < hi) src = s.basis_tok[static_cast<long long>(b) * s.K + beta];
     }
     if (src < 0) continue;                               // uniform in the CTA
-    const uint4* __restrict__ V = reinterpret_cast<const uint4*>(s.V) + (static_cast<long long>(b) * s.N + src) * vec;
+    const uint4* __restrict__ V = reinterpret_cast<const uint4*>(sel_features(s)) + (static_cast<long long>(b) * s.N + src) * vec;
     uint4* __restrict__ dst = reinterpret_cast<uint4*>(s.Vg) + (static_cast<long long>(b) * s.R + r) * vec;
     // four 16-byte loads in flight per thread before their stores (V and Vg never overlap)
     int c = threadIdx.x;
@@ -584,7 +595,7 @@ __global__ void __launch_bounds__(256, 1) sel_greedy_kernel(SelState s) {
   int mine = nb;                                     // valid coordinates at the end
   bool alive = false;
   if (tok >= 0) {
-    p = s.scores[base + tok];
+    p = sel_scores(s)[base + tok];
     alive = s.state[base + tok] == 0;
     if (s.cstep[base + tok] < nb) {                  // sel_update_kernel did not run
       atomicOr(s.status, ST_INTERNAL);
@@ -814,6 +825,30 @@ __global__ void sel_identity_kernel(int N, int32_t* keep, int32_t* order) {
   }
 }
 
+
+// ------------------------------------------------------------------ device-side round loop
+// First node of the loop graph: the WHILE body runs only if an image still selects.
+__global__ void sel_loop_init_kernel(SelState s, cudaGraphConditionalHandle h, int32_t* iters) {
+  if (threadIdx.x == 0) {
+    *iters = 0;
+    cudaGraphSetConditional(h, (*s.done_count < s.B && *s.status == 0) ? 1u : 0u);
+  }
+}
+
+// Last node of the WHILE body: run another two rounds while an image still selects, no kernel
+// has reported an error and the iteration cap has not been reached (then ST_INTERNAL).
+__global__ void sel_loop_cond_kernel(SelState s, cudaGraphConditionalHandle h, int32_t* iters, int cap_iters,
+                                     long long* iters_total) {
+  if (threadIdx.x == 0) {
+    const int it = *iters + 1;
+    *iters = it;
+    *iters_total += 1;
+    const bool pending = *s.done_count < s.B, err = *s.status != 0;
+    if (pending && !err && it >= cap_iters) atomicOr(s.status, ST_INTERNAL);
+    cudaGraphSetConditional(h, (pending && !err && it < cap_iters) ? 1u : 0u);
+  }
+}
+
 }  // namespace
 
 size_t sel_init_smem(int N, int K0) { return (static_cast<size_t>(N) + pow2_at_least(std::max(K0, 1))) * 8; }
@@ -896,6 +931,141 @@ cudaError_t launch_sel_proj_done(const SelState& s, cudaStream_t st) {
 
 cudaError_t launch_sel_identity(int B, int N, int32_t* keep, int32_t* order, cudaStream_t st) {
   return launch_k(sel_identity_kernel, dim3(B), dim3(256), 0, st, N, keep, order);
+}
+
+// ------------------------------------------------------------------ loop graph cache
+struct SelLoopEntry {
+  std::vector<long long> key;
+  cudaGraph_t graph = nullptr;
+  cudaGraphExec_t exec = nullptr;
+};
+
+struct SelLoopCache {
+  std::vector<SelLoopEntry> entries;   // most recently used last
+  cudaStream_t cap = nullptr;          // stream the loop body is captured on
+};
+
+namespace {
+constexpr size_t kSelLoopCacheMax = 8;
+
+void release_entry(SelLoopEntry& e) {
+  if (e.exec) cudaGraphExecDestroy(e.exec);
+  if (e.graph) cudaGraphDestroy(e.graph);
+  e.exec = nullptr;
+  e.graph = nullptr;
+}
+
+long long fbits(float f) {
+  uint32_t u;
+  std::memcpy(&u, &f, 4);
+  return static_cast<long long>(u);
+}
+long long pbits(const void* p) { return static_cast<long long>(reinterpret_cast<uintptr_t>(p)); }
+
+// Everything the captured kernels depend on, except the caller's scores and features (read
+// through s.uptr).
+std::vector<long long> loop_key(const SelState& s, const GemmDesc& g, int num_sms, int cap_iters, const int32_t* iters,
+                                const long long* iters_total) {
+  return {s.B, s.N, s.D, s.K, s.K0, s.S, s.R, s.KP, fbits(s.lambda), fbits(s.tau), pbits(s.sqn), pbits(s.U),
+          pbits(s.r2), pbits(s.cstep), pbits(s.state), pbits(s.Ec), pbits(s.picks), pbits(s.r0), pbits(s.basis_tok),
+          pbits(s.rnorm), pbits(s.npicks), pbits(s.nbasis), pbits(s.nb_gathered), pbits(s.done), pbits(s.mode),
+          pbits(s.nlimit), pbits(s.gb_lo), pbits(s.gb_hi), pbits(s.gbase), pbits(s.theta), pbits(s.aslot),
+          pbits(s.Vg), pbits(s.G), pbits(s.done_count), pbits(s.proj_lim), pbits(s.blist), pbits(s.bcount),
+          s.bc_par, pbits(s.status), pbits(s.nvalid), pbits(s.uptr),
+          pbits(g.A), g.a_rows_total, g.a_row_stride, pbits(g.B), g.b_rows_total, g.b_row_stride, g.M, g.N, g.K,
+          g.batch, pbits(g.n_limit), pbits(g.C), g.ldc, g.c_batch_stride, g.epi, pbits(g.status), pbits(g.blist),
+          g.wait_ns, num_sms, cap_iters, pbits(iters), pbits(iters_total)};
+}
+
+// Builds the graph: [test kernel] -> WHILE { 2 x (choose + gather, Gram, update + greedy); test }.
+cudaError_t build_loop(SelLoopCache* c, const SelState& s, const GemmDesc& gram, int num_sms, int cap_iters,
+                       int32_t* iters, long long* iters_total, SelLoopEntry& out) {
+  cudaError_t e = cudaSuccess;
+  if (!c->cap && (e = cudaStreamCreateWithFlags(&c->cap, cudaStreamNonBlocking)) != cudaSuccess) return e;
+  cudaGraph_t g = nullptr;
+  if ((e = cudaGraphCreate(&g, 0)) != cudaSuccess) return e;
+  auto fail = [&](cudaError_t err) {
+    cudaGraphDestroy(g);
+    return err;
+  };
+  cudaGraphConditionalHandle h;
+  if ((e = cudaGraphConditionalHandleCreate(&h, g, 0, 0)) != cudaSuccess) return fail(e);
+  SelState sc = s;
+  void* init_args[] = {&sc, &h, &iters};
+  cudaKernelNodeParams kp = {};
+  kp.func = reinterpret_cast<void*>(sel_loop_init_kernel);
+  kp.gridDim = dim3(1);
+  kp.blockDim = dim3(32);
+  kp.kernelParams = init_args;
+  cudaGraphNode_t init_node;
+  if ((e = cudaGraphAddKernelNode(&init_node, g, nullptr, 0, &kp)) != cudaSuccess) return fail(e);
+  cudaGraphNodeParams cp = {};
+  cp.type = cudaGraphNodeTypeConditional;
+  cp.conditional.handle = h;
+  cp.conditional.type = cudaGraphCondTypeWhile;
+  cp.conditional.size = 1;
+  cudaGraphNode_t loop_node;
+  if ((e = cudaGraphAddNode(&loop_node, g, &init_node, nullptr, 1, &cp)) != cudaSuccess) return fail(e);
+  cudaGraph_t body = cp.conditional.phGraph_out[0];
+  if ((e = cudaStreamBeginCaptureToGraph(c->cap, body, nullptr, nullptr, 0, cudaStreamCaptureModeRelaxed)) !=
+      cudaSuccess)
+    return fail(e);
+  pdl_disabled() = true;
+  SelState r = s;
+  for (int round = 0; round < 2 && e == cudaSuccess; ++round) {
+    GemmDesc d = gram;
+    d.bcount = r.bcount + r.bc_par;              // the count this round's choose appends to
+    if ((e = launch_sel_choose(r, c->cap)) != cudaSuccess) break;
+    if ((e = launch_gemm(d, num_sms, c->cap)) != cudaSuccess) break;
+    r.bc_par ^= 1;
+    e = launch_sel_greedy(r, c->cap);
+  }
+  if (e == cudaSuccess) e = launch_k(sel_loop_cond_kernel, dim3(1), dim3(32), 0, c->cap, r, h, iters, cap_iters, iters_total);
+  pdl_disabled() = false;
+  cudaGraph_t captured = nullptr;
+  const cudaError_t e2 = cudaStreamEndCapture(c->cap, &captured);
+  if (e == cudaSuccess) e = e2;
+  if (e != cudaSuccess) return fail(e);
+  cudaGraphExec_t x = nullptr;
+  if ((e = cudaGraphInstantiate(&x, g, 0)) != cudaSuccess) return fail(e);
+  out.graph = g;
+  out.exec = x;
+  return cudaSuccess;
+}
+}  // namespace
+
+SelLoopCache* sel_loop_cache_create() { return new SelLoopCache(); }
+
+void sel_loop_cache_destroy(SelLoopCache* c) {
+  if (!c) return;
+  for (auto& e : c->entries) release_entry(e);
+  if (c->cap) cudaStreamDestroy(c->cap);
+  delete c;
+}
+
+cudaError_t launch_sel_loop(SelLoopCache* c, const SelState& s, const GemmDesc& gram, int num_sms, int cap_iters,
+                            int32_t* iters, long long* iters_total, cudaStream_t st) {
+  if (!c || !s.uptr || !s.done_count || !iters || !iters_total || (s.bc_par & ~1)) return cudaErrorInvalidValue;
+  std::vector<long long> key = loop_key(s, gram, num_sms, cap_iters, iters, iters_total);
+  size_t hit = c->entries.size();
+  for (size_t i = 0; i < c->entries.size(); ++i)
+    if (c->entries[i].key == key) { hit = i; break; }
+  if (hit == c->entries.size()) {
+    SelLoopEntry ent;
+    ent.key = std::move(key);
+    const cudaError_t e = build_loop(c, s, gram, num_sms, cap_iters, iters, iters_total, ent);
+    if (e != cudaSuccess) return e;
+    if (c->entries.size() >= kSelLoopCacheMax) {
+      release_entry(c->entries.front());
+      c->entries.erase(c->entries.begin());
+    }
+    c->entries.push_back(std::move(ent));
+  } else if (hit + 1 != c->entries.size()) {
+    SelLoopEntry ent = std::move(c->entries[hit]);
+    c->entries.erase(c->entries.begin() + static_cast<long>(hit));
+    c->entries.push_back(std::move(ent));
+  }
+  return cudaGraphLaunch(c->entries.back().exec, st);
 }
 
 }  // namespace mapk

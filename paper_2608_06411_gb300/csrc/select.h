@@ -44,6 +44,10 @@ struct SelState {
   int32_t* blist; int32_t* bcount; int bc_par;
   int* status;
   const int32_t* nvalid;          // [B] valid tokens per image (nullptr: all N); the rest are padding
+  // Optional device array {scores, V}, written by sel_init from the two fields above: the
+  // kernels of the cached selection-loop graph read the caller's buffers through it, so one
+  // graph serves every call of the same shape.
+  const void** uptr;
 };
 
 size_t sel_init_smem(int N, int K0);
@@ -67,5 +71,21 @@ cudaError_t launch_sel_proj_prep(const SelState& s, bool first, cudaStream_t st)
 cudaError_t launch_sel_gather(const SelState& s, cudaStream_t st);
 // After a projection: the projected images' later Gram blocks start past their basis.
 cudaError_t launch_sel_proj_done(const SelState& s, cudaStream_t st);
+
+// ------------------------------------------------------------------ device-side round loop
+// The selection rounds after the first ones run as a CUDA graph: a kernel node that tests
+// whether any image still selects, then a WHILE conditional node whose body is two rounds
+// (choose + gather, Gram block, coordinate update + greedy picks) followed by the same test.
+// The host never waits for the rounds.  Graphs are cached per shape and workspace.
+struct GemmDesc;
+struct SelLoopCache;
+SelLoopCache* sel_loop_cache_create();
+void sel_loop_cache_destroy(SelLoopCache* c);
+// iters: device int (this call's loop iterations); iters_total: device counter of every loop
+// iteration run so far (for launch counts).  After cap_iters iterations with images still
+// selecting the loop stops and sets ST_INTERNAL.
+cudaError_t launch_sel_loop(SelLoopCache* cache, const SelState& s, const GemmDesc& gram, int num_sms, int cap_iters,
+                            int32_t* iters, long long* iters_total, cudaStream_t st);
+constexpr int kSelLoopKernelsPerIter = 11;
 
 }  // namespace mapk
