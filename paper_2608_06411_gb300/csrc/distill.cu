@@ -5,11 +5,11 @@
 //
 // Activations and gradients are fp32 (the bf16 features and weights are decoded exactly): the
 // gradient is checked against a float64 oracle.  The contractions run on the tcgen05 GEMM of
-// gemm_tc.cu with split-bf16 operands: an fp32 operand x is staged as hi = bf16(x) and
-// lo = bf16(x - hi) (about 16 significant bits), a bf16 feature or weight as itself, and the
-// product is formed from the terms that carry fp32-level weight (hi.hi + hi.lo + lo.hi for two
-// fp32 operands, hi.b + lo.b against an exact bf16 one), accumulated in fp32 in TMEM.  The
-// staging kernels also transpose, so that both operands are K-major whichever index the
+// gemm_tc.cu with split-bf16 operands: an fp32 operand x is staged as three bf16 terms hi, mid,
+// lo (x to about 24 significant bits), a bf16 feature or weight as itself, and the product is
+// formed from every term pair above 2^-24 (six for two fp32 operands, three against an exact
+// bf16 one, one for two bf16 ones), accumulated in fp32 in TMEM.  The staging kernels also
+// transpose, so that both operands are K-major whichever index the
 // contraction runs over (tokens for the weight gradients).  The softmax, KL, RoPE and GELU
 // steps and their derivatives are elementwise or row/column reductions in their own kernels,
 // with fixed-order (deterministic) reductions.
@@ -25,17 +25,22 @@ namespace mapk {
 namespace {
 
 // Operand staging for the tensor-core GEMM.  Element (r, c) of the logical matrix X (r < rows,
-// c < cols; X(r, c) = src[c * ld + r] when TRANS, else src[r * ld + c]; times alpha) is written to
-// row r of dst (row stride ldd elements) as hi = bf16(x) at columns hi0 + c and, if hi1 >= 0,
-// hi1 + c, and as lo = bf16(x - hi) at column lo0 + c if lo0 >= 0; columns cols .. kpad - 1 of
-// each segment are written as zeros.  32 x 32 tiles through shared memory, so that the reads
-// (along the source's contiguous index) and the writes (along c) are both coalesced.  BF16:
-// the source holds bf16 bit patterns (then lo = 0 when alpha = 1).
+// c < cols; X(r, c) = src[c * ld + r] when TRANS, else src[r * ld + c]; times alpha) is split into
+// three bf16 terms, hi = bf16(x), mid = bf16(x - hi), lo = bf16(x - hi - mid) (x = hi + mid + lo
+// to about 24 significant bits; both differences are exact in fp32), and each term is written to
+// row r of dst (row stride ldd elements) at column off + c for every offset of its list (up to
+// three, -1 = unused).  Columns cols .. kpad - 1 of each segment are written as zeros.  32 x 32
+// tiles through shared memory, so that the reads (along the source's contiguous index) and the
+// writes (along c) are both coalesced.  BF16: the source holds bf16 bit patterns.
+struct SplitOffsets {
+  int hi[3], mid[3], lo[3];
+};
+
 template <bool TRANS, bool BF16>
 __global__ void __launch_bounds__(256) split_operand_kernel(const void* __restrict__ src, long long ld, int rows,
                                                             int cols, int kpad, float alpha,
-                                                            uint16_t* __restrict__ dst, long long ldd, int hi0,
-                                                            int hi1, int lo0) {
+                                                            uint16_t* __restrict__ dst, long long ldd,
+                                                            SplitOffsets o) {
   __shared__ float t[32][33];                        // t[c - c0][r - r0]
   pdl_enter();
   const int c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
@@ -61,11 +66,16 @@ __global__ void __launch_bounds__(256) split_operand_kernel(const void* __restri
     if (r >= rows || c >= kpad) continue;
     const float x = t[tx][i] * alpha;
     const __nv_bfloat16 h = __float2bfloat16_rn(x);
-    uint16_t* row = dst + static_cast<long long>(r) * ldd;
-    const uint16_t hb = __bfloat16_as_ushort(h);
-    row[hi0 + c] = hb;
-    if (hi1 >= 0) row[hi1 + c] = hb;
-    if (lo0 >= 0) row[lo0 + c] = __bfloat16_as_ushort(__float2bfloat16_rn(x - __bfloat162float(h)));
+    const float r1 = x - __bfloat162float(h);
+    const __nv_bfloat16 m = __float2bfloat16_rn(r1);
+    const __nv_bfloat16 l = __float2bfloat16_rn(r1 - __bfloat162float(m));
+    uint16_t* row = dst + static_cast<long long>(r) * ldd + c;
+#pragma unroll
+    for (int j = 0; j < 3; ++j) {
+      if (o.hi[j] >= 0) row[o.hi[j]] = __bfloat16_as_ushort(h);
+      if (o.mid[j] >= 0) row[o.mid[j]] = __bfloat16_as_ushort(m);
+      if (o.lo[j] >= 0) row[o.lo[j]] = __bfloat16_as_ushort(l);
+    }
   }
 }
 
@@ -269,40 +279,73 @@ unsigned grid_for(long long n) {
 
 namespace {
 
+// Terms of the product a.b kept for each kind of operand pair (x = hi + mid + lo for an fp32
+// operand, exact for a bf16 one): everything down to about 2^-24 relative, so the result is as
+// good as an fp32 product accumulated in fp32.
+//   bf16 . bf16 : a.b                                           1 product
+//   fp32 . bf16 : lo.b + mid.b + hi.b                           3 products
+//   fp32 . fp32 : mm + hl + lh + hm + mh + hh                   6 products (ml, lm, ll are below 2^-24)
+// The staged operands are the matching segments side by side along K, so one GEMM with
+// K' = (number of products) * Kp forms the sum.
 struct TcPlan {
-  int Kp, ka, kb, kprime;   // padded K, staged widths of A and B, GEMM K
-  bool a_split, b_split;
+  int Kp, n;                // padded K, number of products (K' = n Kp)
+  SplitOffsets a, b;
 };
+
+SplitOffsets no_offsets() {
+  SplitOffsets o;
+  for (int j = 0; j < 3; ++j) o.hi[j] = o.mid[j] = o.lo[j] = -1;
+  return o;
+}
 
 TcPlan tc_plan(int K, float alpha, bool a_bf16, bool b_bf16) {
   TcPlan p;
   p.Kp = ((K + 63) / 64) * 64;
-  p.a_split = !(a_bf16 && alpha == 1.0f);
-  p.b_split = !b_bf16;
-  if (!p.a_split && !p.b_split) { p.ka = p.kb = p.kprime = p.Kp; }          // a.b
-  else if (p.a_split && p.b_split) { p.ka = 2 * p.Kp; p.kb = p.kprime = 3 * p.Kp; }   // ah.bh + ah.bl + al.bh
-  else { p.ka = p.kb = p.kprime = 2 * p.Kp; }                                  // ah.b + al.b (or a.bh + a.bl)
+  const int Kp = p.Kp;
+  const bool a_split = !(a_bf16 && alpha == 1.0f), b_split = !b_bf16;
+  p.a = no_offsets();
+  p.b = no_offsets();
+  // Segments are ordered smallest term first, so that the tensor cores' fp32 accumulator adds
+  // the small terms while it is still small and runs only the last Kp / 16 steps at full
+  // magnitude (their additions are where the accumulation error comes from).
+  if (!a_split && !b_split) {
+    p.n = 1;
+    p.a.hi[0] = 0;
+    p.b.hi[0] = 0;
+  } else if (a_split && !b_split) {                 // [lo | mid | hi] . [b | b | b]
+    p.n = 3;
+    p.a.lo[0] = 0; p.a.mid[0] = Kp; p.a.hi[0] = 2 * Kp;
+    p.b.hi[0] = 0; p.b.hi[1] = Kp; p.b.hi[2] = 2 * Kp;
+  } else if (!a_split && b_split) {                 // [a | a | a] . [lo | mid | hi]
+    p.n = 3;
+    p.a.hi[0] = 0; p.a.hi[1] = Kp; p.a.hi[2] = 2 * Kp;
+    p.b.lo[0] = 0; p.b.mid[0] = Kp; p.b.hi[0] = 2 * Kp;
+  } else {                                          // [m h l h m h] . [m l h m h h]
+    p.n = 6;
+    p.a.mid[0] = 0; p.a.hi[0] = Kp; p.a.lo[0] = 2 * Kp; p.a.hi[1] = 3 * Kp; p.a.mid[1] = 4 * Kp; p.a.hi[2] = 5 * Kp;
+    p.b.mid[0] = 0; p.b.lo[0] = Kp; p.b.hi[0] = 2 * Kp; p.b.mid[1] = 3 * Kp; p.b.hi[1] = 4 * Kp; p.b.hi[2] = 5 * Kp;
+  }
   return p;
 }
 
 cudaError_t stage(const void* src, bool bf16, bool trans, long long ld, int rows, int cols, int kpad, float alpha,
-                  uint16_t* dst, long long ldd, int hi0, int hi1, int lo0, cudaStream_t st) {
+                  uint16_t* dst, long long ldd, const SplitOffsets& o, cudaStream_t st) {
   const dim3 grid((kpad + 31) / 32, (rows + 31) / 32);
   if (grid.y > 65535u) return cudaErrorInvalidValue;
   if (trans) {
-    if (bf16) return launch_k(split_operand_kernel<true, true>, grid, dim3(256), 0, st, src, ld, rows, cols, kpad, alpha, dst, ldd, hi0, hi1, lo0);
-    return launch_k(split_operand_kernel<true, false>, grid, dim3(256), 0, st, src, ld, rows, cols, kpad, alpha, dst, ldd, hi0, hi1, lo0);
+    if (bf16) return launch_k(split_operand_kernel<true, true>, grid, dim3(256), 0, st, src, ld, rows, cols, kpad, alpha, dst, ldd, o);
+    return launch_k(split_operand_kernel<true, false>, grid, dim3(256), 0, st, src, ld, rows, cols, kpad, alpha, dst, ldd, o);
   }
-  if (bf16) return launch_k(split_operand_kernel<false, true>, grid, dim3(256), 0, st, src, ld, rows, cols, kpad, alpha, dst, ldd, hi0, hi1, lo0);
-  return launch_k(split_operand_kernel<false, false>, grid, dim3(256), 0, st, src, ld, rows, cols, kpad, alpha, dst, ldd, hi0, hi1, lo0);
+  if (bf16) return launch_k(split_operand_kernel<false, true>, grid, dim3(256), 0, st, src, ld, rows, cols, kpad, alpha, dst, ldd, o);
+  return launch_k(split_operand_kernel<false, false>, grid, dim3(256), 0, st, src, ld, rows, cols, kpad, alpha, dst, ldd, o);
 }
 
 }  // namespace
 
 void tc_matmul_ws(int M, int N, int K, float alpha, bool a_bf16, bool b_bf16, size_t* a_elems, size_t* b_elems) {
   const TcPlan p = tc_plan(K, alpha, a_bf16, b_bf16);
-  *a_elems = static_cast<size_t>(M) * p.ka;
-  *b_elems = static_cast<size_t>(N) * p.kb;
+  *a_elems = static_cast<size_t>(M) * p.n * p.Kp;
+  *b_elems = static_cast<size_t>(N) * p.n * p.Kp;
 }
 
 cudaError_t launch_tc_matmul(bool ta, bool tb, int M, int N, int K, float alpha, const void* A, bool a_bf16,
@@ -310,25 +353,20 @@ cudaError_t launch_tc_matmul(bool ta, bool tb, int M, int N, int K, float alpha,
                              void* wsA, void* wsB, int num_sms, int* status, long long wait_ns, cudaStream_t st) {
   if (M <= 0 || N <= 0 || K <= 0) return cudaSuccess;
   const TcPlan p = tc_plan(K, alpha, a_bf16, b_bf16);
+  const int kw = p.n * p.Kp;
   uint16_t* As = static_cast<uint16_t*>(wsA);
   uint16_t* Bs = static_cast<uint16_t*>(wsB);
   // A_s(i, k) = A(i, k): a transposed read when ta.  B_s(j, k) = B(k, j): transposed unless tb.
-  const int a_hi1 = (!p.a_split && p.b_split) ? p.Kp : -1, a_lo = p.a_split ? p.Kp : -1;
-  cudaError_t e = stage(A, a_bf16, ta, lda, M, K, p.Kp, alpha, As, p.ka, 0, a_hi1, a_lo, st);
+  cudaError_t e = stage(A, a_bf16, ta, lda, M, K, p.Kp, alpha, As, kw, p.a, st);
   if (e != cudaSuccess) return e;
-  int b_hi1 = -1, b_lo = -1;
-  if (p.a_split && p.b_split) { b_hi1 = p.Kp; b_lo = 2 * p.Kp; }
-  else if (p.a_split) { b_hi1 = p.Kp; }
-  else if (p.b_split) { b_lo = p.Kp; }
-  e = stage(B, b_bf16, !tb, ldb, N, K, p.Kp, 1.0f, Bs, p.kb, 0, b_hi1, b_lo, st);
+  e = stage(B, b_bf16, !tb, ldb, N, K, p.Kp, 1.0f, Bs, kw, p.b, st);
   if (e != cudaSuccess) return e;
   GemmDesc d{};
   d.A = As; d.a_rows_total = M; d.a_row_stride = 0;
   d.B = Bs; d.b_rows_total = N; d.b_row_stride = 0;
-  d.M = M; d.N = N; d.K = p.kprime; d.batch = 1;
+  d.M = M; d.N = N; d.K = kw; d.batch = 1;
   d.C = C; d.ldc = ldc; d.c_batch_stride = 0;
   d.epi = EPI_F32; d.status = status; d.wait_ns = wait_ns;
-  if (p.a_split && p.b_split) { d.split3 = 1; d.a_kwrap = 2 * p.Kp; }
   return launch_gemm(d, num_sms, st);
 }
 

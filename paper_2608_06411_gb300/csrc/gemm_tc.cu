@@ -78,11 +78,12 @@ struct Smem {
   static constexpr uint32_t TILES = STAGES * STAGE_BYTES;
   static constexpr uint32_t BARS = (2 * STAGES + 5 + (PROJ ? 1 : 0)) * 8;
   static constexpr uint32_t XPOSE = EPI == EPI_SM_STATS ? 4 * 32 * 33 * 4 : 0;   // per-warp 32x32 transposes
-  // bf16 outputs written by TMA box stores from per-warp staging: hi/lo split epilogues use two
-  // buffers of (hi, lo) 32x32 boxes, EPI_ROPE_SPLIT3 (BN = 128) one buffer of (hi, lo) x 2 halves
+  // bf16 outputs written by TMA box stores from per-warp staging: hi/lo split epilogues use one
+  // buffer of (hi, lo) 32x32 boxes per warp (smaller than two, so that the small CTAs of a row-norm
+  // kernel fit beside the layer-1 GEMM), EPI_ROPE_SPLIT3 (BN = 128) one buffer of (hi, lo) x 2 halves
   static constexpr bool TSTORE_ROPE = EPI == EPI_ROPE_SPLIT3 && BN == 128;
   static constexpr bool TSTORE = EPI == EPI_GELU_SPLIT || EPI == EPI_BIAS_SPLIT || TSTORE_ROPE;
-  static constexpr uint32_t STG = TSTORE ? 4 * 4 * 32 * 32 * 2 : 0;
+  static constexpr uint32_t STG = TSTORE ? (TSTORE_ROPE ? 4 * 4 * 32 * 32 * 2 : 4 * 2 * 32 * 32 * 2) : 0;
   static constexpr uint32_t LSM = PROJ ? BN * BN * 4 : 0;       // L rows of the basis (pitch BN)
   static constexpr uint32_t PEXTRA = PROJ ? BN * 4 : 0;          // 1/r of the basis
   static constexpr uint32_t NSQ = PROJ ? 2 * kBM * 4 : 0;        // ||row||^2 of a tile, per accumulator
@@ -289,11 +290,12 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       if (!mbar_wait(&tempty[acc], acc_phase ^ 1, a.status, abort_flag, a.wait_ns)) break;   // norms slot free
       float s0 = 0.f, s1 = 0.f;
       bool ok = true;
+      const bool sum = a.proj.sqn_in == nullptr;      // norms not known: sum them here
       for (int kb = 0; kb < KB; ++kb) {
         if (!mbar_wait(&full[stage], phase, a.status, abort_flag, a.wait_ns)) { ok = false; break; }
         const uint8_t* At = sA + stage * S::A_BYTES;
 #pragma unroll
-        for (int ch = 0; ch < 8; ++ch) {
+        for (int ch = 0; ch < (sum ? 8 : 0); ++ch) {
           const uint4 x0 = *reinterpret_cast<const uint4*>(At + r0 * 128 + ((ch ^ (r0 & 7)) << 4));
           const uint4 x1 = *reinterpret_cast<const uint4*>(At + r1 * 128 + ((ch ^ (r1 & 7)) << 4));
           const uint32_t w0[4] = {x0.x, x0.y, x0.z, x0.w}, w1[4] = {x1.x, x1.y, x1.z, x1.w};
@@ -589,7 +591,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         const long long tok = static_cast<long long>(c.b) * a.M + row;
         const bool alive = row_ok && __ldg(pj.state + tok) == 0;
         float* erow = pj.Ec + tok * pj.KP;
-        const float sq = sqn_sm[acc * kBM + r_in_tile];
+        const float sq = pj.sqn_in ? (row_ok ? __ldg(pj.sqn_in + tok) : 0.f) : sqn_sm[acc * kBM + r_in_tile];
         float r2 = sq;
 #pragma unroll 1
         for (int b0 = 0; b0 < nb0; b0 += 32) {
@@ -695,8 +697,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           uint32_t r[32];
           tmem_ld32(tbase + ch * 32, r);
           const int cbase = col0 + ch * 32;
-          uint8_t* hb = stg + (ew * 2 + (ch & 1)) * 4096;     // [hi 32x32 | lo 32x32] bf16
-          if (lane == 0) bulk_wait_group_read<1>();      // this buffer's previous store has read it
+          uint8_t* hb = stg + ew * 4096;                 // [hi 32x32 | lo 32x32] bf16
+          if (lane == 0) bulk_wait_group_read<0>();      // the previous chunk's stores have read it
           __syncwarp();
           uint32_t pk[16], pl[16];
 #pragma unroll

@@ -34,6 +34,7 @@ struct ProjArgs {
   int Kcap;
   float lambda, tau;
   float* r2; float* U; float* sqn; int32_t* cstep;   // [B, N] outputs
+  const float* sqn_in;         // [B, N] ||v||^2 already known (nullptr: the kernel sums them)
 };
 
 // Batched C = epi(A @ B^T): A rows [batch][a_row_stride] x K, B rows [batch][b_row_stride] x K
@@ -107,6 +108,10 @@ cudaError_t launch_flags_to_host(const int32_t* a, const int* b, int32_t* a_host
 // Squared row norms of bf16 rows: out[r] = sum_d x[r, d]^2 (fp32).
 cudaError_t launch_row_sqnorm(const void* x, long long rows, int D, float* out, cudaStream_t st);
 
+// The same, launched right after a persistent GEMM on the stream: it runs beside that GEMM on
+// the resources it leaves free (num_sms small CTAs) and completes only after it.
+cudaError_t launch_row_sqnorm_beside(const void* x, long long rows, int D, float* out, int num_sms, cudaStream_t st);
+
 // scores[b, n] = sum_t part[b, t, n] over n_tiles column-tile partial means.
 cudaError_t launch_sum_tiles(const float* part, int B, int N, int n_tiles, float* scores, cudaStream_t st);
 
@@ -130,8 +135,8 @@ cudaError_t launch_assemble(const void* V, const int32_t* idx, const void* T, co
 // ------------------------------------------------------------------ distillation step (fp32)
 // C[i, j] = alpha sum_k A(i, k) B(k, j) on the tcgen05 GEMM, fp32 in (or bf16: a_bf16 / b_bf16)
 // and fp32 out; row-major, A(i, k) = ta ? A[k lda + i] : A[i lda + k], B(k, j) = tb ? B[j ldb + k]
-// : B[k ldb + j].  fp32 operands are staged as bf16 (hi, lo) pairs (split-bf16 products, see
-// distill.cu) in wsA / wsB, of at least the element counts tc_matmul_ws returns; C must be
+// : B[k ldb + j].  fp32 operands are staged as three bf16 terms (split-bf16 products to fp32
+// accuracy, see distill.cu) in wsA / wsB, of at least the element counts tc_matmul_ws returns; C must be
 // 16-byte aligned with ldc % 4 == 0.  Deterministic (fixed summation order).
 void tc_matmul_ws(int M, int N, int K, float alpha, bool a_bf16, bool b_bf16, size_t* a_elems, size_t* b_elems);
 cudaError_t launch_tc_matmul(bool ta, bool tb, int M, int N, int K, float alpha, const void* A, bool a_bf16,
