@@ -198,7 +198,7 @@ GemmDesc linear_desc(map_ctx* c, const void* x, long long rows, int K, const voi
 // the second layer and the projection are one folded matrix Wf = Wp W2 with bias Wp b2.
 int predictor_branch(map_ctx* c, const void* x, long long rows, const void* w1, const void* b1, const void* wf,
                      const float* bf, DevBuf& h1, void* out3, int split_kind, float scale, float* aux,
-                     const int* pos, int pos_mod, cudaStream_t st, int tid_l1, int tid_p, float* sqn_out = nullptr) {
+                     const int* pos, int pos_mod, cudaStream_t st, int tid_l1, int tid_p) {
   const map_config& g = c->cfg;
   MAP_TRY(ensure(h1, static_cast<size_t>(rows) * g.Dh * 4));
   {
@@ -206,10 +206,6 @@ int predictor_branch(map_ctx* c, const void* x, long long rows, const void* w1, 
     GemmDesc d = linear_desc(c, x, rows, g.D, w1, g.Dh, b1, h1.p, mapk::EPI_GELU_SPLIT);
     d.ldc = 2LL * g.Dh;
     MAP_TRY(gemm(c, d, st));
-  }
-  if (sqn_out) {   // ||x||^2 of every row for the selection, beside the layer-1 GEMM (it reads x too)
-    ++c->counters.launches;
-    CU_TRY(mapk::launch_row_sqnorm_beside(x, rows, g.D, sqn_out, c->num_sms, st));
   }
   {
     // K = 3 Dh: h_hi Wf_hi + h_hi Wf_lo + h_lo Wf_hi, A = [hi | lo] against
@@ -234,10 +230,8 @@ int predictor_branch(map_ctx* c, const void* x, long long rows, const void* w1, 
 
 // nv (host, B entries, or nullptr = every image has N tokens): valid visual tokens per image;
 // rows at or past nv[b] are padding, excluded from Eq. 3 (their score is 0).
-// sqn_out (device, B N floats, or nullptr): also writes ||v||^2 of every visual token, for a
-// selection that follows on the same features.
 int score_impl(map_ctx* c, const void* text, const void* vis, const int32_t* lens, const int32_t* nv, int B, int N,
-               float* scores, float* q_out, float* k_out, cudaStream_t st, float* sqn_out = nullptr) {
+               float* scores, float* q_out, float* k_out, cudaStream_t st) {
   if (!c || !text || !vis || !lens || !scores) return MAP_EINVAL;
   if (B < 1 || N < 1) return MAP_EINVAL;
   if (nv)
@@ -289,7 +283,7 @@ int score_impl(map_ctx* c, const void* text, const void* vis, const int32_t* len
                            c->s_aux, MAP_K_GEMM_TEXT, MAP_K_GEMM_TEXT));
   CU_TRY(cudaEventRecord(c->ev_join, c->s_aux));
   MAP_TRY(predictor_branch(c, vis, vrows, c->w[5], c->w[6], c->wkv, c->bkv, c->h1, c->kb.p, 0, 1.0f, k_out, nullptr,
-                           N, st, MAP_K_GEMM_FV1, MAP_K_GEMM_WK, sqn_out));
+                           N, st, MAP_K_GEMM_FV1, MAP_K_GEMM_WK));
   CU_TRY(cudaStreamWaitEvent(st, c->ev_join, 0));
   // Eq. 3 on the tensor cores: logits tile [visual tokens x question tokens] of one image,
   // pass 1 -> per-slab column (max, sum exp), combine -> (max, 1/sum), pass 2 -> mean.
@@ -336,9 +330,8 @@ T* carve(char*& p, size_t n) {
 }
 
 // nv as for score_impl: tokens at or past nv[b] are never retained (K <= every nv[b]).
-// sqn_ready: c->sqn already holds ||v||^2 of these features (written by score_impl).
 int select_impl(map_ctx* c, const float* scores, const void* vis, const int32_t* nv, int B, int N, int K,
-                int32_t* keep, int32_t* order, cudaStream_t st, bool sqn_ready = false) {
+                int32_t* keep, int32_t* order, cudaStream_t st) {
   if (!c || !scores || !vis) return MAP_EINVAL;
   if (B < 1 || N < 1 || K < 0 || K > N) return MAP_EINVAL;
   if (nv)
@@ -419,10 +412,8 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, const int32_t*
   // candidate its exact value (and ||v||^2); otherwise values start from p_hat * ||v||^lambda.
   const bool project = K0 > 0 && K0 < K && K0 <= kProjMaxBasis;
   if (K0 < K && !project) {
-    if (!sqn_ready) {
-      ++c->counters.launches;
-      CU_TRY(mapk::launch_row_sqnorm(vis, BN, g.D, static_cast<float*>(c->sqn.p), st));
-    }
+    ++c->counters.launches;
+    CU_TRY(mapk::launch_row_sqnorm(vis, BN, g.D, static_cast<float*>(c->sqn.p), st));
   } else if (K0 >= K) {
     CU_TRY(cudaMemsetAsync(c->sqn.p, 0, BN * 4, st));
   }
@@ -473,7 +464,6 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, const int32_t*
       pd.proj.basis_tok = s.basis_tok; pd.proj.rnorm = s.rnorm; pd.proj.nbasis = s.nbasis; pd.proj.Kcap = K;
       pd.proj.lambda = g.lambda; pd.proj.tau = g.tau;
       pd.proj.r2 = s.r2; pd.proj.U = s.U; pd.proj.sqn = static_cast<float*>(c->sqn.p); pd.proj.cstep = s.cstep;
-      pd.proj.sqn_in = sqn_ready ? static_cast<const float*>(c->sqn.p) : nullptr;
       auto project_all = [&](bool first) -> int {
         c->counters.launches += 3;
         CU_TRY(mapk::launch_sel_proj_prep(s, first, st));
@@ -788,13 +778,8 @@ int prune_impl(map_ctx* ctx, const void* text_feats, const void* vis_feats, cons
     int32_t* kpc = kp + static_cast<size_t>(b0) * k;
     void* oc = static_cast<char*>(o) + static_cast<size_t>(b0) * k * D * 2;
     const int32_t* nvc = nv ? nv + b0 : nullptr;
-    // the norms of Eq. 4 are summed beside the layer-1 GEMM, which reads the same features
-    const bool norms = k > 0 && k < N;
-    int rc = norms ? ensure(c->sqn, static_cast<size_t>(Bc) * N * 4) : MAP_OK;
-    if (rc == MAP_OK)
-      rc = score_impl(c, tc, vc, lens + b0, nvc, Bc, N, spc, nullptr, nullptr, st,
-                      norms ? static_cast<float*>(c->sqn.p) : nullptr);
-    if (rc == MAP_OK) rc = select_impl(c, spc, vc, nvc, Bc, N, k, kpc, nullptr, st, norms);
+    int rc = score_impl(c, tc, vc, lens + b0, nvc, Bc, N, spc, nullptr, nullptr, st);
+    if (rc == MAP_OK) rc = select_impl(c, spc, vc, nvc, Bc, N, k, kpc, nullptr, st);
     if (rc == MAP_OK) rc = gather_impl(c, vc, kpc, Bc, N, k, oc, st);
     if (rc != MAP_OK) return finish(rc);
     if (host_io) {

@@ -18,9 +18,8 @@
 //               thread), apply bias / GELU / RoPE, store (bf16, bf16 hi/lo pair, or fp32);
 //               release the accumulator so the
 //               MMA warp can start the tile after next while this one drains.
-//   EPI_PROJECT: two more warps (6-7) read every staged A tile and sum each row's squares
-//               (||v||^2) on the CUDA cores; they release the stage together with the MMA
-//               commit and hand the tile's norms to the epilogue with the accumulator.
+//   EPI_PROJECT: the MMA thread also accumulates A A^T (N = 128) of every stage into a second
+//               TMEM accumulator, whose diagonal is ||row||^2.
 // All waits are bounded (ptx.cuh); a timeout sets ST_TIMEOUT and every role drains and exits.
 #include <algorithm>
 #include <cstdio>
@@ -78,18 +77,16 @@ struct Smem {
   static constexpr uint32_t TILES = STAGES * STAGE_BYTES;
   static constexpr uint32_t BARS = (2 * STAGES + 5 + (PROJ ? 1 : 0)) * 8;
   static constexpr uint32_t XPOSE = EPI == EPI_SM_STATS ? 4 * 32 * 33 * 4 : 0;   // per-warp 32x32 transposes
-  // bf16 outputs written by TMA box stores from per-warp staging: hi/lo split epilogues use one
-  // buffer of (hi, lo) 32x32 boxes per warp (smaller than two, so that the small CTAs of a row-norm
-  // kernel fit beside the layer-1 GEMM), EPI_ROPE_SPLIT3 (BN = 128) one buffer of (hi, lo) x 2 halves
+  // bf16 outputs written by TMA box stores from per-warp staging: hi/lo split epilogues use two
+  // buffers of (hi, lo) 32x32 boxes, EPI_ROPE_SPLIT3 (BN = 128) one buffer of (hi, lo) x 2 halves
   static constexpr bool TSTORE_ROPE = EPI == EPI_ROPE_SPLIT3 && BN == 128;
   static constexpr bool TSTORE = EPI == EPI_GELU_SPLIT || EPI == EPI_BIAS_SPLIT || TSTORE_ROPE;
-  static constexpr uint32_t STG = TSTORE ? (TSTORE_ROPE ? 4 * 4 * 32 * 32 * 2 : 4 * 2 * 32 * 32 * 2) : 0;
+  static constexpr uint32_t STG = TSTORE ? 4 * 4 * 32 * 32 * 2 : 0;
   static constexpr uint32_t LSM = PROJ ? BN * BN * 4 : 0;       // L rows of the basis (pitch BN)
   static constexpr uint32_t PEXTRA = PROJ ? BN * 4 : 0;          // 1/r of the basis
-  static constexpr uint32_t NSQ = PROJ ? 2 * kBM * 4 : 0;        // ||row||^2 of a tile, per accumulator
-  static constexpr uint32_t TOTAL = 1024 + TILES + STG + BARS + 16 + XPOSE + LSM + PEXTRA + NSQ;
-  static constexpr uint32_t TMEM_COLS = PROJ ? (2 * BN <= 256 ? 256u : 512u) : 2 * BN;
-  static constexpr int THREADS = PROJ ? 256 : 192;               // + 2 row-norm warps
+  static constexpr uint32_t TOTAL = 1024 + TILES + STG + BARS + 16 + XPOSE + LSM + PEXTRA;
+  static constexpr uint32_t TMEM_COLS = PROJ ? (2 * BN + 2 * kBM <= 256 ? 256u : 512u) : 2 * BN;   // + A A^T
+  static constexpr int THREADS = 192;
 };
 
 // Selection value, squared: p^2 * rho^(2 lambda) orders candidates like p * rho^lambda (both are
@@ -148,16 +145,12 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   float* xpose = reinterpret_cast<float*>(smem + S::TILES + S::STG + S::BARS + 16);
   float* Lsm = xpose + S::XPOSE / 4;
   float* rinv_sm = Lsm + S::LSM / 4;
-  float* sqn_sm = rinv_sm + S::PEXTRA / 4;         // EPI_PROJECT: [2][kBM] row norms per accumulator
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
-    // EPI_PROJECT: a stage is free once the MMA commit and both row-norm warps have arrived, and
-    // an accumulator is full once the MMA commit and both row-norm warps (its norms) have
-    constexpr uint32_t kArrive = S::PROJ ? 3 : 1;
-    for (int s = 0; s < STAGES; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], kArrive); }
+    for (int s = 0; s < STAGES; ++s) { mbar_init(&full[s], 1); mbar_init(&empty[s], 1); }
     // tempty: one arrive per epilogue warp (of both CTAs with CG2, on the leader's barrier)
-    for (int i = 0; i < 2; ++i) { mbar_init(&tfull[i], kArrive); mbar_init(&tempty[i], CG2 ? 8 : 4); }
+    for (int i = 0; i < 2; ++i) { mbar_init(&tfull[i], 1); mbar_init(&tempty[i], CG2 ? 8 : 4); }
     mbar_init(drain, 1);
     if constexpr (S::PROJ) {
       mbar_init(egsync, 128);
@@ -258,6 +251,13 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
 #pragma unroll
             for (int k = 0; k < kBK / 16; ++k)
               umma_bf16(d_tmem, desc_sw128(a0 + k * 32), desc_sw128(b0 + k * 32), IDESC, (kb | k) != 0);
+            if constexpr (S::PROJ) {   // A A^T: its diagonal is ||row||^2
+              const uint32_t n_tmem = tmem_base + 2 * BN + acc * kBM;
+#pragma unroll
+              for (int k = 0; k < kBK / 16; ++k)
+                umma_bf16(n_tmem, desc_sw128(a0 + k * 32), desc_sw128(a0 + k * 32), idesc_bf16(kBM, kBM),
+                          (kb | k) != 0);
+            }
             umma_commit(&empty[stage]);
           }
           issued = true;
@@ -276,51 +276,6 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       }
     }
     __syncwarp();
-  } else if (S::PROJ && warp >= 6) {
-    // ------------------------------------------------------------------ row norms (EPI_PROJECT)
-    // Warp 6 sums rows 0-63 of every staged A tile, warp 7 rows 64-127, two rows per lane.  A
-    // row's 64 values are its own 128-byte line in the 128-byte swizzle (only the 16-byte
-    // chunks are permuted), so lane l reads physical chunk c ^ (row & 7) at step c: the eight
-    // rows of a quarter warp hit distinct banks, and the order of a sum is not an issue.
-    const int r0 = (warp - 6) * 64 + lane, r1 = r0 + 32;
-    uint32_t stage = 0, phase = 0, acc = 0, acc_phase = 0;
-    for (int t = unit0; t < total; t += units_step) {
-      TileCoord c = tile_coord<PAIR>(a, t, m_units, n_tiles, BN, crank);
-      if (c.skip) continue;
-      if (!mbar_wait(&tempty[acc], acc_phase ^ 1, a.status, abort_flag, a.wait_ns)) break;   // norms slot free
-      float s0 = 0.f, s1 = 0.f;
-      bool ok = true;
-      const bool sum = a.proj.sqn_in == nullptr;      // norms not known: sum them here
-      for (int kb = 0; kb < KB; ++kb) {
-        if (!mbar_wait(&full[stage], phase, a.status, abort_flag, a.wait_ns)) { ok = false; break; }
-        const uint8_t* At = sA + stage * S::A_BYTES;
-#pragma unroll
-        for (int ch = 0; ch < (sum ? 8 : 0); ++ch) {
-          const uint4 x0 = *reinterpret_cast<const uint4*>(At + r0 * 128 + ((ch ^ (r0 & 7)) << 4));
-          const uint4 x1 = *reinterpret_cast<const uint4*>(At + r1 * 128 + ((ch ^ (r1 & 7)) << 4));
-          const uint32_t w0[4] = {x0.x, x0.y, x0.z, x0.w}, w1[4] = {x1.x, x1.y, x1.z, x1.w};
-#pragma unroll
-          for (int u = 0; u < 4; ++u) {
-            const float2 f0 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w0[u]));
-            const float2 f1 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w1[u]));
-            s0 = fmaf(f0.x, f0.x, s0);
-            s0 = fmaf(f0.y, f0.y, s0);
-            s1 = fmaf(f1.x, f1.x, s1);
-            s1 = fmaf(f1.y, f1.y, s1);
-          }
-        }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&empty[stage]);
-        if (++stage == STAGES) { stage = 0; phase ^= 1; }
-      }
-      if (!ok) break;
-      sqn_sm[acc * kBM + r0] = s0;
-      sqn_sm[acc * kBM + r1] = s1;
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&tfull[acc]);        // release: the norms are visible to the epilogue
-      acc ^= 1;
-      if (acc == 0) acc_phase ^= 1;
-    }
   } else if (warp < 6) {
     // ------------------------------------------------------------------ epilogue
     const int lane_grp = warp & 3;                 // TMEM lanes this warp may access
@@ -591,7 +546,13 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         const long long tok = static_cast<long long>(c.b) * a.M + row;
         const bool alive = row_ok && __ldg(pj.state + tok) == 0;
         float* erow = pj.Ec + tok * pj.KP;
-        const float sq = pj.sqn_in ? (row_ok ? __ldg(pj.sqn_in + tok) : 0.f) : sqn_sm[acc * kBM + r_in_tile];
+        float sq = 0.f;
+        {
+          uint32_t dg[32];
+          tmem_ld32(tmem_base + (static_cast<uint32_t>(lane_grp * 32) << 16) + 2 * BN + acc * kBM + lane_grp * 32, dg);
+#pragma unroll
+          for (int j = 0; j < 32; ++j) sq = j == lane ? __uint_as_float(dg[j]) : sq;
+        }
         float r2 = sq;
 #pragma unroll 1
         for (int b0 = 0; b0 < nb0; b0 += 32) {
@@ -697,8 +658,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           uint32_t r[32];
           tmem_ld32(tbase + ch * 32, r);
           const int cbase = col0 + ch * 32;
-          uint8_t* hb = stg + ew * 4096;                 // [hi 32x32 | lo 32x32] bf16
-          if (lane == 0) bulk_wait_group_read<0>();      // the previous chunk's stores have read it
+          uint8_t* hb = stg + (ew * 2 + (ch & 1)) * 4096;     // [hi 32x32 | lo 32x32] bf16
+          if (lane == 0) bulk_wait_group_read<1>();      // this buffer's previous store has read it
           __syncwarp();
           uint32_t pk[16], pl[16];
 #pragma unroll

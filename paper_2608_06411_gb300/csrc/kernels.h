@@ -17,9 +17,9 @@ namespace mapk {
 // 32-row slab, then per-row mean over columns of exp(l - max) / sum.
 // EPI_PROJECT: rows = visual tokens, columns = the R0 basis tokens' rows (Gram entries
 // <v_n, v_r>); the epilogue solves for the tokens' Cholesky coordinates against the R0
-// basis (L staged in shared memory), and two extra warps sum ||v_n||^2 from the same
-// shared-memory tiles.  It writes the exact residual, value and coordinate cache of every
-// candidate token (see select.cu).
+// basis (L staged in shared memory); ||v_n||^2 is the diagonal of an A A^T product that the
+// MMA thread accumulates from the same shared-memory tiles.  It writes the exact residual,
+// value and coordinate cache of every candidate token (see select.cu).
 enum Epi { EPI_GELU_BF16 = 0, EPI_BIAS_BF16 = 1, EPI_ROPE_F32 = 2, EPI_F32 = 3, EPI_GELU_SPLIT = 4,
            EPI_BIAS_SPLIT = 5, EPI_ROPE_SPLIT3 = 6, EPI_SM_STATS = 7, EPI_SM_MEAN = 8, EPI_PROJECT = 9 };
 
@@ -34,7 +34,6 @@ struct ProjArgs {
   int Kcap;
   float lambda, tau;
   float* r2; float* U; float* sqn; int32_t* cstep;   // [B, N] outputs
-  const float* sqn_in;         // [B, N] ||v||^2 already known (nullptr: the kernel sums them)
 };
 
 // Batched C = epi(A @ B^T): A rows [batch][a_row_stride] x K, B rows [batch][b_row_stride] x K
@@ -107,10 +106,6 @@ cudaError_t launch_flags_to_host(const int32_t* a, const int* b, int32_t* a_host
 
 // Squared row norms of bf16 rows: out[r] = sum_d x[r, d]^2 (fp32).
 cudaError_t launch_row_sqnorm(const void* x, long long rows, int D, float* out, cudaStream_t st);
-
-// The same, launched right after a persistent GEMM on the stream: it runs beside that GEMM on
-// the resources it leaves free (num_sms small CTAs) and completes only after it.
-cudaError_t launch_row_sqnorm_beside(const void* x, long long rows, int D, float* out, int num_sms, cudaStream_t st);
 
 // scores[b, n] = sum_t part[b, t, n] over n_tiles column-tile partial means.
 cudaError_t launch_sum_tiles(const float* part, int B, int N, int n_tiles, float* scores, cudaStream_t st);

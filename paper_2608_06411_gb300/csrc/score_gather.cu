@@ -10,37 +10,6 @@ namespace {
 
 // ------------------------------------------------------------------ squared norms
 // One warp per row; 16-byte loads; fp32 accumulation in a fixed order.
-// Row norms computed beside the GEMM launched just before on the stream: the kernel does not
-// wait for that grid (its input was complete before the GEMM started) and lets the next kernel
-// be scheduled at once, so its few small CTAs take the SM resources the persistent GEMM leaves
-// free; it waits for the GEMM only at the end, so that the kernel after it still sees the
-// GEMM's results.  One warp per row, grid-stride over the rows.
-__global__ void __launch_bounds__(256) row_sqnorm_beside_kernel(const uint4* __restrict__ x, long long rows,
-                                                                int vec_per_row, float* __restrict__ out) {
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-  const int lane = threadIdx.x & 31;
-  const long long wstep = static_cast<long long>(gridDim.x) * (blockDim.x >> 5);
-  for (long long row = static_cast<long long>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5); row < rows;
-       row += wstep) {
-    const uint4* p = x + row * vec_per_row;
-    float acc = 0.f;
-    for (int v = lane; v < vec_per_row; v += 32) {
-      const uint4 u = __ldg(p + v);
-      const uint32_t w[4] = {u.x, u.y, u.z, u.w};
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const float lo = __uint_as_float(w[i] << 16), hi = __uint_as_float(w[i] & 0xFFFF0000u);
-        acc = fmaf(lo, lo, acc);
-        acc = fmaf(hi, hi, acc);
-      }
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-    if (lane == 0) out[row] = acc;
-  }
-  asm volatile("griddepcontrol.wait;" ::: "memory");
-}
-
 __global__ void row_sqnorm_kernel(const uint4* __restrict__ x, long long rows, int vec_per_row,
                                   float* __restrict__ out) {
   pdl_enter();
@@ -329,23 +298,6 @@ cudaError_t launch_row_sqnorm(const void* x, long long rows, int D, float* out, 
   const int warps = 8;
   const long long blocks = (rows + warps - 1) / warps;
   return launch_k(row_sqnorm_kernel, dim3(static_cast<unsigned>(blocks)), dim3(warps * 32), 0, st,
-                  static_cast<const uint4*>(x), rows, D / 8, out);
-}
-
-cudaError_t launch_row_sqnorm_beside(const void* x, long long rows, int D, float* out, int num_sms, cudaStream_t st) {
-  if (rows <= 0) return cudaSuccess;
-  if (D % 8 != 0) return cudaErrorInvalidValue;
-  const long long blocks = std::min<long long>((rows + 7) / 8, num_sms);
-  // the same shared-memory carveout as the GEMM beside which it runs (an SM holds CTAs of
-  // kernels with different carveouts only after reconfiguring)
-  static bool carveout_set = false;
-  if (!carveout_set) {
-    const cudaError_t e = cudaFuncSetAttribute(row_sqnorm_beside_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
-                                               static_cast<int>(cudaSharedmemCarveoutMaxShared));
-    if (e != cudaSuccess) return e;
-    carveout_set = true;
-  }
-  return launch_k(row_sqnorm_beside_kernel, dim3(static_cast<unsigned>(blocks)), dim3(256), 0, st,
                   static_cast<const uint4*>(x), rows, D / 8, out);
 }
 
