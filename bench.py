@@ -500,6 +500,8 @@ def main():
     ap.add_argument("--only-qcts", action="store_true",
                     help="run only the teacher-selection measurement (for profiling), print its JSON")
     ap.add_argument("--qcts-samples", type=int, default=W.ATTENTION_WORKLOADS["q1"].B)
+    ap.add_argument("--only-distill", action="store_true",
+                    help="run only the distillation-step measurement (for profiling), print its JSON")
     ap.add_argument("--batch", type=int, default=WORKLOAD.B, help="images per GPU (profiling on a smaller case)")
     ap.add_argument("--minimal", action="store_true",
                     help="time the steps only (no clock sampling, latency, e2e or CPU baseline): for ncu runs")
@@ -514,6 +516,10 @@ def main():
     ws, rank, local = dist_env()
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
+    if args.only_distill:
+        if rank == 0:
+            print(json.dumps(bench_distill(mb, dev, torch.cuda.current_stream(), args.steps, False)))
+        return 0
     if args.only_qcts:
         if rank == 0:
             hbm = measured_peaks()[0]

@@ -286,7 +286,7 @@ int score_impl(map_ctx* c, const void* text, const void* vis, const int32_t* len
                            N, st, MAP_K_GEMM_FV1, MAP_K_GEMM_WK));
   CU_TRY(cudaStreamWaitEvent(st, c->ev_join, 0));
   // Eq. 3 on the tensor cores: logits tile [visual tokens x question tokens] of one image,
-  // pass 1 -> per-slab column (max, sum exp), combine -> (max, 1/sum), pass 2 -> mean.
+  // pass 1 -> per-slab column (max, sum exp), combine -> max + ln(sum), pass 2 -> mean.
   const int m_tiles = (N + 127) / 128, nparts = 4 * m_tiles;
   const int ld = ((max_m + 3) / 4) * 4;
   const int n_tiles = (max_m + 255) / 256;

@@ -76,7 +76,8 @@ struct Smem {
   static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr uint32_t TILES = STAGES * STAGE_BYTES;
   static constexpr uint32_t BARS = (2 * STAGES + 5 + (PROJ ? 1 : 0)) * 8;
-  static constexpr uint32_t XPOSE = EPI == EPI_SM_STATS ? 4 * 32 * 33 * 4 : 0;   // per-warp 32x32 transposes
+  // per-warp 32x32 transposes (EPI_SM_STATS) or 32 column normalisers (EPI_SM_MEAN)
+  static constexpr uint32_t XPOSE = EPI == EPI_SM_STATS ? 4 * 32 * 33 * 4 : (EPI == EPI_SM_MEAN ? 4 * 32 * 4 : 0);
   // bf16 outputs written by TMA box stores from per-warp staging: hi/lo split epilogues use two
   // buffers of (hi, lo) 32x32 boxes, EPI_ROPE_SPLIT3 (BN = 128) one buffer of (hi, lo) x 2 halves
   static constexpr bool TSTORE_ROPE = EPI == EPI_ROPE_SPLIT3 && BN == 128;
@@ -508,29 +509,30 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           float sum = 0.f;
           if (m != -INFINITY) {
 #pragma unroll
-            for (int i = 0; i < 32; ++i) sum += expf(tr[i * 33 + lane] - m);
+            for (int i = 0; i < 32; ++i) sum += __expf(tr[i * 33 + lane] - m);
           }
           __syncwarp();
           if (cbase + lane < ncol) part[cbase + lane] = make_float2(m, sum);
         }
       } else if constexpr (EPI == EPI_SM_MEAN) {
-        // p_hat[row] = (1/M_b) sum_col exp(l - max_col) / sum_col
+        // p_hat[row] = (1/M_b) sum_col exp(l - c_col), c_col = max_col + ln(sum_col): each chunk's
+        // 32 column normalisers are loaded once (lane j: column j) into this warp's shared row
+        // and read back as broadcasts
         const int ncol = a.col_count ? min(lim, __ldg(a.col_count + c.b)) : lim;
         const float2* fin = a.stats + static_cast<long long>(c.b) * a.stat_ld;
+        float* cn = xpose + (warp - 2) * 32;
         float acc_p = 0.f;
 #pragma unroll 1
         for (int ch = 0; ch < BN / 32; ++ch) {
           uint32_t r[32];
           tmem_ld32(tbase + ch * 32, r);
           const int cbase = col0 + ch * 32;
-          if (cbase >= ncol) continue;
+          if (cbase >= ncol) continue;                    // uniform in the warp
+          __syncwarp();                                   // the previous chunk's reads are done
+          cn[lane] = cbase + lane < ncol ? __ldg(fin + cbase + lane).x : INFINITY;   // exp(-inf) = 0
+          __syncwarp();
 #pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            if (cbase + j < ncol) {
-              const float2 st = __ldg(fin + cbase + j);
-              acc_p += expf(__uint_as_float(r[j]) - st.x) * st.y;
-            }
-          }
+          for (int j = 0; j < 32; ++j) acc_p += __expf(__uint_as_float(r[j]) - cn[j]);
         }
         if (row < a.M) {   // rows past the image's valid tokens (m_limit) get 0
           float* out = reinterpret_cast<float*>(a.C) + static_cast<long long>(c.b) * a.c_batch_stride;

@@ -55,7 +55,7 @@ struct GemmDesc {
   // batched B rows at per-batch offsets (device) instead of b * b_row_stride
   const int* b_off = nullptr;
   // EPI_SM_STATS: partial (max, sum) per 32-row slab [batch][m_tiles * 4][stat_ld] (float2)
-  // EPI_SM_MEAN:  final (max, 1/sum) per column [batch][stat_ld]; output C = scores
+  // EPI_SM_MEAN:  final (max + ln sum, 1/sum) per column [batch][stat_ld]; output C = scores
   //               [batch][M] when one column tile covers all columns
   float2* stats = nullptr; int stat_ld = 0;
   const int* col_count = nullptr;       // per-batch number of valid columns (M_b)
@@ -110,7 +110,7 @@ cudaError_t launch_row_sqnorm(const void* x, long long rows, int D, float* out, 
 // scores[b, n] = sum_t part[b, t, n] over n_tiles column-tile partial means.
 cudaError_t launch_sum_tiles(const float* part, int B, int N, int n_tiles, float* scores, cudaStream_t st);
 
-// Combines the per-slab softmax statistics into (max, 1/sum) per question token:
+// Combines the per-slab softmax statistics into (max + ln sum, 1/sum) per question token:
 // part [B][nparts][ld] -> fin [B][ld], columns < lens[b].
 cudaError_t launch_stats_combine(const float2* part, int B, int nparts, int ld, const int* lens, float2* fin,
                                  cudaStream_t st);

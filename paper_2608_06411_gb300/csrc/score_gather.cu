@@ -50,7 +50,7 @@ __global__ void gather_rows_kernel(const uint4* __restrict__ V, const int32_t* _
   for (int v = threadIdx.x; v < vec_per_row; v += blockDim.x) d[v] = __ldg(s + v);
 }
 
-// (max, sum) partials of one column over all slabs -> (max, 1/sum).  A block covers 32
+// (max, sum) partials of one column over all slabs -> (max + ln sum, 1/sum).  A block covers 32
 // columns (threadIdx.x, coalesced) with kCombY threads per column splitting the slabs; the
 // kCombY partial maxima and sums are combined in a fixed order in shared memory.
 constexpr int kCombY = 8;
@@ -83,7 +83,8 @@ __global__ void __launch_bounds__(32 * kCombY) stats_combine_kernel(const float2
     float s = red[0][x];
 #pragma unroll
     for (int j = 1; j < kCombY; ++j) s += red[j][x];
-    fin[static_cast<long long>(b) * ld + col] = make_float2(m, 1.0f / s);
+    // one log-normaliser per column: exp(l - m) / s = exp(l - (m + ln s))
+    fin[static_cast<long long>(b) * ld + col] = make_float2(m + logf(s), 1.0f / s);
   }
 }
 
