@@ -40,7 +40,7 @@ struct map_ctx {
   // [hi | hi | lo] of W_Q W_T2 / W_K W_V2 ([dp, 3 Dh]) and fp32 biases W_Q b_T2 / W_K b_V2
   void* wqt = nullptr; void* wkv = nullptr; float* bqt = nullptr; float* bkv = nullptr;
   DevBuf rope;  int rope_rows = 0;
-  DevBuf h1, kb, th1, qb, stats, qoff, post, sqn, pmean, snv, dist, dsa, dsb;
+  DevBuf h1, kb, th1, qb, stats, qoff, post, sqn, pmean, snv, dist, dsa, dsb, dsc;
   // selection
   DevBuf sU, sr2, scstep, sstate, sEc, spicks, sr0, sbt, srn, ssmall, stheta, saslot, sVg, sG;
   // map_prune staging
@@ -882,7 +882,7 @@ int map_distill_grad(map_ctx* ctx, const void* text_feats, const void* vis_feats
   const long long Np = (N + 3) / 4 * 4;              // logits row stride: 16-byte aligned rows
   const int bias_idx[4] = {1, 3, 6, 8};
   const long long floats = 4 * Dh + 5 * (Tv + Tt) * Dh + 4 * (Tv + Tt) * dp + Tt * Np + 2LL * B * N +
-                           static_cast<long long>(B) * nblk + total_m + 64 * 16;
+                           static_cast<long long>(B) * nblk + total_m + 64 * Dh + 64 * 16;
   MAP_TRY(ensure(c->dist, static_cast<size_t>(floats) * 4));
   float* base = static_cast<float*>(c->dist.p);
   auto take = [&](long long n) { float* p = base; base += ((n + 15) / 16) * 16; return p; };
@@ -896,6 +896,7 @@ int map_distill_grad(map_ctx* ctx, const void* text_feats, const void* vis_feats
   float *p_hat = take(static_cast<long long>(B) * N), *gb = take(static_cast<long long>(B) * N);
   float* part = take(static_cast<long long>(B) * nblk);
   int32_t* d_row_img = reinterpret_cast<int32_t*>(take(total_m));
+  float* colpart = take(64 * Dh);                    // partial column sums of the bias gradients
   const float rs = 1.0f / std::sqrt(static_cast<float>(dp));
   // Every contraction of the step, in order: C = alpha A(M x K) B(K x N) with A(i, k) = ta ? A[k lda
   // + i] : A[i lda + k], B(k, j) = tb ? B[j ldb + k] : B[k ldb + j]; bf16 operands are exact.
@@ -929,23 +930,25 @@ int map_distill_grad(map_ctx* ctx, const void* text_feats, const void* vis_feats
   branch_bwd(Tv, dkp, vis_feats, 5, h1v, h2v, dh2v, dh1v, 9);
   branch_bwd(Tt, dqp, text_feats, 0, h1t, h2t, dh2t, dh1t, 4);
   // staging buffers for the split-bf16 operands: the largest any contraction needs
-  size_t wa = 0, wb = 0;
+  size_t wa = 0, wb = 0, wc = 0;
   for (const auto* list : {&fwd, &mid, &bwd})
     for (const Mm& m : *list) {
-      size_t a = 0, bb = 0;
+      size_t a = 0, bb = 0, cc = 0;
       mapk::tc_matmul_ws(static_cast<int>(m.M), static_cast<int>(m.N), static_cast<int>(m.K), m.alpha, m.abf, m.bbf,
-                         &a, &bb);
+                         c->num_sms, &a, &bb, &cc);
       wa = std::max(wa, a);
       wb = std::max(wb, bb);
+      wc = std::max(wc, cc);
     }
   MAP_TRY(ensure(c->dsa, wa * 2));
   MAP_TRY(ensure(c->dsb, wb * 2));
-  long long n_mm = 0;
+  MAP_TRY(ensure(c->dsc, std::max<size_t>(wc, 4) * 4));
+  long long mm_launches = 0;
   auto run_mm = [&](const Mm& m) -> int {
-    ++n_mm;
     cudaError_t e = mapk::launch_tc_matmul(m.ta, m.tb, static_cast<int>(m.M), static_cast<int>(m.N),
                                            static_cast<int>(m.K), m.alpha, m.A, m.abf, m.lda, m.Bm, m.bbf, m.ldb,
-                                           m.C, m.ldc, c->dsa.p, c->dsb.p, c->num_sms, c->status, c->wait_ns, st);
+                                           m.C, m.ldc, c->dsa.p, c->dsb.p, static_cast<float*>(c->dsc.p), c->num_sms,
+                                           c->status, c->wait_ns, st, &mm_launches);
     if (e == cudaErrorInvalidValue) return MAP_EUNSUPPORTED;
     return cuda_err(e);
   };
@@ -976,19 +979,20 @@ int map_distill_grad(map_ctx* ctx, const void* text_feats, const void* vis_feats
     MAP_TRY(run_mm(bwd[j]));                         // dW_p
     MAP_TRY(run_mm(bwd[j + 1]));                     // dh2
     MAP_TRY(run_mm(bwd[j + 2]));                     // dW2
-    CU_TRY(mapk::launch_colsum(dh2, T, Dh, gout[i1 + 3], st));
+    CU_TRY(mapk::launch_colsum(dh2, T, Dh, colpart, gout[i1 + 3], st));
     MAP_TRY(run_mm(bwd[j + 3]));                     // dh1
     CU_TRY(mapk::launch_gelu_back(dh1, z1, T * Dh, st));
     MAP_TRY(run_mm(bwd[j + 4]));                     // dW1
-    CU_TRY(mapk::launch_colsum(dh1, T, Dh, gout[i1 + 1], st));
+    CU_TRY(mapk::launch_colsum(dh1, T, Dh, colpart, gout[i1 + 1], st));
     return MAP_OK;
   };
   MAP_TRY(bwd_tail(0, dk, Tv, nullptr, g.rope_on ? N : 1, dkp, z1v, dh2v, dh1v, 5));
   MAP_TRY(bwd_tail(5, dq, Tt, g.rope_on ? post : nullptr, 1, dqp, z1t, dh2t, dh1t, 0));
-  // query metadata, question-row images, 4 bias conversions, 3 launches per contraction (two
-  // operand stagings, the GEMM), 2 x 3 forward elementwise, 4 loss / softmax-backward kernels,
-  // 2 x 5 backward elementwise
-  c->counters.launches += (B + 1023) / 1024 + (total_m + 2047) / 2048 + 4 + 3 * n_mm + 6 + 4 + 10;
+  // query metadata, question-row images, 4 bias conversions, the contractions (the GEMM, its
+  // operand stagings and the sum of its K slices, as counted by the launcher), 2 x 3 forward
+  // elementwise, 4 loss / softmax-backward kernels, 2 x 6 backward elementwise (RoPE transpose,
+  // GELU', two column sums of two launches each)
+  c->counters.launches += (B + 1023) / 1024 + (total_m + 2047) / 2048 + 4 + mm_launches + 6 + 4 + 12;
   return MAP_OK;
 }
 
@@ -1016,7 +1020,7 @@ void map_destroy(map_ctx* ctx) {
   for (void* p : {ctx->wqt, ctx->wkv, static_cast<void*>(ctx->bqt), static_cast<void*>(ctx->bkv)})
     if (p) cudaFree(p);
   DevBuf* bufs[] = {&ctx->rope, &ctx->h1, &ctx->kb, &ctx->th1, &ctx->qb, &ctx->stats,
-                    &ctx->qoff, &ctx->post, &ctx->sqn, &ctx->pmean, &ctx->snv, &ctx->dist, &ctx->dsa, &ctx->dsb, &ctx->sU, &ctx->sr2, &ctx->scstep, &ctx->sstate,
+                    &ctx->qoff, &ctx->post, &ctx->sqn, &ctx->pmean, &ctx->snv, &ctx->dist, &ctx->dsa, &ctx->dsb, &ctx->dsc, &ctx->sU, &ctx->sr2, &ctx->scstep, &ctx->sstate,
                     &ctx->sEc, &ctx->spicks, &ctx->sr0, &ctx->sbt, &ctx->srn, &ctx->ssmall, &ctx->stheta,
                     &ctx->saslot, &ctx->sVg, &ctx->sG, &ctx->pvis, &ctx->ptext, &ctx->pout, &ctx->pkeep,
                     &ctx->pscores};

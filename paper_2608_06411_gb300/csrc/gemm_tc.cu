@@ -49,12 +49,13 @@ struct KArgs {
   const int* col_count;
   int b_base;
   ProjArgs proj;
-  int a_kwrap;
+  int a_kwrap, b_kwrap;
   int split3;
   const float* biasf;
   const int* blist; const int* bcount;
   const int* m_limit;
   unsigned long long wait_ns;   // limit of the role waits (the drain waits keep kWaitLimitNs)
+  int ksplit; long long c_split_stride;   // EPI_F32 split-K: partial sums per K slice
 };
 
 __device__ __forceinline__ float gelu_erf(float x) {
@@ -100,17 +101,21 @@ __device__ __forceinline__ float proj_value(float p, float r2, float sq, float l
   return v > 0.f ? v : 0.f;
 }
 
-struct TileCoord { int b, m_blk, n_blk; bool skip; };
+struct TileCoord { int b, m_blk, n_blk, ks; bool skip; };
 
 // Work unit t -> tile.  With PAIR the unit is a pair of vertically adjacent M tiles with the
 // same N tile, processed by the two CTAs of a cluster (rank 0 the upper, rank 1 the lower).
+// With split-K (ksplit > 1) a unit is also one K slice ks of its tile.
 template <bool PAIR>
 __device__ __forceinline__ TileCoord tile_coord(const KArgs& a, int t, int m_units, int n_tiles, int BN,
                                                 uint32_t crank) {
   TileCoord c;
-  int per = m_units * n_tiles;
+  const int tiles = m_units * n_tiles;
+  int per = tiles * a.ksplit;
   c.b = t / per;
   int rem = t - c.b * per;
+  c.ks = rem / tiles;
+  rem -= c.ks * tiles;
   if (a.blist) c.b = __ldg(a.blist + c.b);
   const int mu = rem / n_tiles;
   c.n_blk = rem - mu * n_tiles;
@@ -173,8 +178,13 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   const int m_tiles = (a.M + kBM - 1) / kBM;
   const int m_units = PAIR ? (m_tiles + 1) / 2 : m_tiles;
   const int n_tiles = (a.N + BN - 1) / BN;
-  const int total = (a.blist ? min(a.batch, *a.bcount) : a.batch) * m_units * n_tiles;
+  const int total = (a.blist ? min(a.batch, *a.bcount) : a.batch) * m_units * n_tiles * a.ksplit;
   const int KB = a.K / kBK;
+  // K blocks of a unit's slice (the whole K without split-K)
+  auto kb_range = [&](const TileCoord& c, int& kb0, int& kb1) {
+    kb0 = c.ks * KB / a.ksplit;
+    kb1 = (c.ks + 1) * KB / a.ksplit;
+  };
   // K block kb -> (A column, B column)
   auto kcols = [&](int kb, int& ac, int& bc) {
     if (a.split3) {
@@ -188,7 +198,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       }
     } else {
       ac = a.a_kwrap > 0 ? (kb * kBK) % a.a_kwrap : kb * kBK;
-      bc = kb * kBK;
+      bc = a.b_kwrap > 0 ? (kb * kBK) % a.b_kwrap : kb * kBK;
     }
   };
 
@@ -206,7 +216,9 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         if (c.skip) continue;
         const int arow = c.b * a.a_row_stride + c.m_blk * kBM;
         const int brow = (a.b_off ? __ldg(a.b_off + c.b) : c.b * a.b_row_stride + a.b_base) + c.n_blk * BN;
-        for (int kb = 0; kb < KB; ++kb) {
+        int kb0, kb1;
+        kb_range(c, kb0, kb1);
+        for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1, a.status, abort_flag, a.wait_ns)) { ok = false; break; }
           int ac, bc;
           kcols(kb, ac, bc);
@@ -238,7 +250,9 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         if (!mbar_wait(&tempty[acc], acc_phase ^ 1, a.status, abort_flag, a.wait_ns)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + acc * BN;
-        for (int kb = 0; kb < KB; ++kb) {
+        int kb0, kb1;
+        kb_range(c, kb0, kb1);
+        for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(&full[stage], phase, a.status, abort_flag, a.wait_ns)) { ok = false; break; }
           tc_fence_after();
           const uint32_t a0 = smem_u32(sA + stage * S::A_BYTES);
@@ -246,18 +260,18 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           if constexpr (CG2) {
 #pragma unroll
             for (int k = 0; k < kBK / 16; ++k)
-              umma_bf16_cg2(d_tmem, desc_sw128(a0 + k * 32), desc_sw128(b0 + k * 32), IDESC, (kb | k) != 0);
+              umma_bf16_cg2(d_tmem, desc_sw128(a0 + k * 32), desc_sw128(b0 + k * 32), IDESC, (kb != kb0 || k != 0));
             umma_commit_cg2_mc(&empty[stage], static_cast<uint16_t>(3));
           } else {
 #pragma unroll
             for (int k = 0; k < kBK / 16; ++k)
-              umma_bf16(d_tmem, desc_sw128(a0 + k * 32), desc_sw128(b0 + k * 32), IDESC, (kb | k) != 0);
+              umma_bf16(d_tmem, desc_sw128(a0 + k * 32), desc_sw128(b0 + k * 32), IDESC, (kb != kb0 || k != 0));
             if constexpr (S::PROJ) {   // A A^T: its diagonal is ||row||^2
               const uint32_t n_tmem = tmem_base + 2 * BN + acc * kBM;
 #pragma unroll
               for (int k = 0; k < kBK / 16; ++k)
                 umma_bf16(n_tmem, desc_sw128(a0 + k * 32), desc_sw128(a0 + k * 32), idesc_bf16(kBM, kBM),
-                          (kb | k) != 0);
+                          (kb != kb0 || k != 0));
             }
             umma_commit(&empty[stage]);
           }
@@ -630,7 +644,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
           pj.cstep[tok] = nb0;
         }
       } else if constexpr (EPI == EPI_F32) {
-        float* out = reinterpret_cast<float*>(a.C) + crow + col0;
+        float* out = reinterpret_cast<float*>(a.C) + crow + col0 + c.ks * a.c_split_stride;
 #pragma unroll 1
         for (int ch = 0; ch < BN / 32; ++ch) {
           uint32_t r[32];
@@ -792,7 +806,8 @@ cudaError_t run(const GemmDesc& d, const KArgs& ka, int num_sms, cudaStream_t st
   using S = Smem<BN, STAGES, EPI, PAIR>;
   CUtensorMap ta, tb;
   if (!make_map(&ta, d.A, d.a_rows_total, d.a_kwrap > 0 ? d.a_kwrap : d.K, kBM)) return cudaErrorInvalidValue;
-  if (!make_map(&tb, d.B, d.b_rows_total, d.K, PAIR ? BN / 2 : BN)) return cudaErrorInvalidValue;
+  if (!make_map(&tb, d.B, d.b_rows_total, d.b_kwrap > 0 ? d.b_kwrap : d.K, PAIR ? BN / 2 : BN))
+    return cudaErrorInvalidValue;
   CUtensorMap tc = ta;
   if constexpr (S::TSTORE) {       // output [rows, ldc] bf16, 32x32 boxes, 64-byte swizzle
     // box stores clip at a_rows_total, which is the row bound M only for one flat batch
@@ -817,7 +832,7 @@ cudaError_t run(const GemmDesc& d, const KArgs& ka, int num_sms, cudaStream_t st
   }
   const int m_tiles = (d.M + kBM - 1) / kBM, n_tiles = (d.N + BN - 1) / BN;
   if (PAIR) {
-    const int units = d.batch * ((m_tiles + 1) / 2) * n_tiles;
+    const int units = d.batch * ((m_tiles + 1) / 2) * n_tiles * ka.ksplit;
     if (units == 0) return cudaSuccess;
     const int grid = 2 * std::max(1, std::min(units, num_sms / 2));
     cudaLaunchConfig_t cfg = {};
@@ -836,7 +851,7 @@ cudaError_t run(const GemmDesc& d, const KArgs& ka, int num_sms, cudaStream_t st
     cfg.numAttrs = 2;
     return cudaLaunchKernelEx(&cfg, kern, ta, tb, tc, ka);
   }
-  const int tiles = d.batch * m_tiles * n_tiles;
+  const int tiles = d.batch * m_tiles * n_tiles * ka.ksplit;
   if (tiles == 0) return cudaSuccess;
   const int grid = std::max(1, std::min(tiles, num_sms));
   return launch_k(kern, dim3(grid), dim3(S::THREADS), S::TOTAL, st, ta, tb, tc, ka);
@@ -847,6 +862,8 @@ cudaError_t run(const GemmDesc& d, const KArgs& ka, int num_sms, cudaStream_t st
 cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t st) {
   if (d.K <= 0 || d.K % kBK != 0 || d.M < 0 || d.N <= 0 || d.batch <= 0) return cudaErrorInvalidValue;
   if (d.a_kwrap < 0 || d.a_kwrap % kBK != 0 || d.a_kwrap > d.K) return cudaErrorInvalidValue;
+  if (d.b_kwrap < 0 || d.b_kwrap % kBK != 0 || d.b_kwrap > d.K || (d.b_kwrap > 0 && d.split3))
+    return cudaErrorInvalidValue;
   if (d.split3 && (d.K % (3 * kBK) != 0 || d.a_kwrap != 2 * (d.K / 3))) return cudaErrorInvalidValue;
   if ((reinterpret_cast<uintptr_t>(d.A) | reinterpret_cast<uintptr_t>(d.B)) & 15) return cudaErrorInvalidValue;
   if (d.M == 0) return cudaSuccess;
@@ -873,10 +890,14 @@ cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t st) {
   ka.split_kind = d.split_kind; ka.scale = d.scale; ka.aux = d.aux; ka.b_off = d.b_off;
   ka.stats = d.stats; ka.stat_ld = d.stat_ld; ka.col_count = d.col_count;
   ka.b_base = d.b_base; ka.proj = d.proj;
-  ka.a_kwrap = d.a_kwrap; ka.biasf = d.biasf; ka.split3 = d.split3;
+  ka.a_kwrap = d.a_kwrap; ka.b_kwrap = d.b_kwrap; ka.biasf = d.biasf; ka.split3 = d.split3;
   ka.blist = d.blist; ka.bcount = d.blist ? d.bcount : nullptr;
   ka.m_limit = d.m_limit;
   ka.wait_ns = d.wait_ns > 0 ? static_cast<unsigned long long>(d.wait_ns) : kWaitLimitNs;
+  // split-K: fp32 partial tiles only, every slice at least one K block
+  if (d.ksplit < 1 || (d.ksplit > 1 && (d.epi != EPI_F32 || d.ksplit > d.K / kBK || d.c_split_stride % 4 != 0)))
+    return cudaErrorInvalidValue;
+  ka.ksplit = d.ksplit; ka.c_split_stride = d.c_split_stride;
   if (d.blist && !d.bcount) return cudaErrorInvalidValue;
   switch (d.epi) {
     case EPI_GELU_BF16:

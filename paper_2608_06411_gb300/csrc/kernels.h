@@ -65,6 +65,8 @@ struct GemmDesc {
   // A has a_kwrap columns; its K coordinate wraps (k mod a_kwrap), so a K-segment of A can
   // be read twice against different B segments (0: A has K columns)
   int a_kwrap = 0;
+  // B has b_kwrap columns and its K coordinate wraps likewise (0: B has K columns)
+  int b_kwrap = 0;
   // split3 = 1 (with K = 3 Dh, A = [hi | lo] and B = [W_hi | W_hi | W_lo]): K blocks are taken
   // as (hi_j, W_hi_j), (hi_j, W_lo_j) for every j, then (lo_j, W_hi_j), so each block of A_hi
   // is read twice back to back (the second time from L2)
@@ -79,6 +81,9 @@ struct GemmDesc {
   // Limit (ns) of the producer / MMA / epilogue waits; 0 = the default 2 s.  The waits that
   // let in-flight copies and MMAs land before an aborting CTA exits keep the default.
   long long wait_ns = 0;
+  // EPI_F32 split-K: ksplit K slices, each unit one slice of a tile, slice s writing its partial
+  // sum at C + s * c_split_stride (elements, a multiple of 4); the caller adds the slices
+  int ksplit = 1; long long c_split_stride = 0;
 };
 
 // Returns cudaSuccess, or an error for an unsupported shape (cudaErrorInvalidValue).
@@ -133,10 +138,15 @@ cudaError_t launch_assemble(const void* V, const int32_t* idx, const void* T, co
 // : B[k ldb + j].  fp32 operands are staged as three bf16 terms (split-bf16 products to fp32
 // accuracy, see distill.cu) in wsA / wsB, of at least the element counts tc_matmul_ws returns; C must be
 // 16-byte aligned with ldc % 4 == 0.  Deterministic (fixed summation order).
-void tc_matmul_ws(int M, int N, int K, float alpha, bool a_bf16, bool b_bf16, size_t* a_elems, size_t* b_elems);
+// wsC: K-slice partial sums when the output has too few tiles to fill the GPU.  A bf16 operand
+// that is K-major, dense and 64-aligned is read in place.  *launches (if given) counts the
+// kernels launched.
+void tc_matmul_ws(int M, int N, int K, float alpha, bool a_bf16, bool b_bf16, int num_sms, size_t* a_elems,
+                  size_t* b_elems, size_t* c_elems);
 cudaError_t launch_tc_matmul(bool ta, bool tb, int M, int N, int K, float alpha, const void* A, bool a_bf16,
                              long long lda, const void* B, bool b_bf16, long long ldb, float* C, long long ldc,
-                             void* wsA, void* wsB, int num_sms, int* status, long long wait_ns, cudaStream_t st);
+                             void* wsA, void* wsB, float* wsC, int num_sms, int* status, long long wait_ns,
+                             cudaStream_t st, long long* launches);
 cudaError_t launch_bf16_to_f32(const void* x, long long n, float* y, cudaStream_t st);
 // z += b (per column); h = GELU(z)
 cudaError_t launch_bias_gelu(float* z, const float* b, long long rows, int cols, float* h, cudaStream_t st);
@@ -153,7 +163,7 @@ cudaError_t launch_distill_loss_grad(float* S, long long ld, long long total_m, 
                                      float* g, float* part, float* loss, cudaStream_t st);
 // dh *= GELU'(z)
 cudaError_t launch_gelu_back(float* dh, const float* z, long long n, cudaStream_t st);
-// out[c] = sum_r X[r, c]
-cudaError_t launch_colsum(const float* X, long long rows, int cols, float* out, cudaStream_t st);
+// out[c] = sum_r X[r, c], in a fixed order; part: 64 * cols floats of workspace
+cudaError_t launch_colsum(const float* X, long long rows, int cols, float* part, float* out, cudaStream_t st);
 
 }  // namespace mapk
