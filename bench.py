@@ -585,7 +585,7 @@ def main():
     total_ms = evs[0].elapsed_time(evs[-1])
     fv1_ms, fv1_n = ctx.read_timing(mb.K_GEMM_FV1)
     other = {name: ctx.read_timing(kid) for name, kid in
-             [("wk", mb.K_GEMM_WK), ("text", mb.K_GEMM_TEXT), ("scores", mb.K_SCORES),
+             [("wk", mb.K_GEMM_WK), ("text_stream_span", mb.K_GEMM_TEXT), ("scores", mb.K_SCORES),
               ("select", mb.K_SELECT), ("gather", mb.K_GATHER)]}
     ctx.set_timing(False)
     total_ms = max_over_ranks(total_ms, dev)
