@@ -19,7 +19,7 @@ namespace {
 
 constexpr int kSelS = 256;          // active-set size of the selection (Gram block rows)
 constexpr int kMaxKDiverse = 1024;  // k limit when the diversity term is on (shared-memory staging)
-constexpr int kProjMaxBasis = 128;  // R0 size up to which the projection pass is used
+constexpr int kProjMaxBasis = 128;  // basis vectors one projection pass takes
 constexpr int kMaxK = 4096;
 constexpr int kMaxN = 16384;
 
@@ -408,9 +408,13 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, const int32_t*
   s.theta = static_cast<uint64_t*>(c->stheta.p);
   s.aslot = static_cast<int32_t*>(c->saslot.p);
 
-  // With 0 < K0 <= 128, one tensor-core pass over V after the R0 rounds gives every
-  // candidate its exact value (and ||v||^2); otherwise values start from p_hat * ||v||^lambda.
-  const bool project = K0 > 0 && K0 < K && K0 <= kProjMaxBasis;
+  // With 0 < K0 < K, one tensor-core pass over V after the first R0 tokens gives every
+  // candidate its exact value on their basis (and ||v||^2); otherwise values start from
+  // p_hat * ||v||^lambda.  The first K0c <= 128 tokens of R0 are factored before the pass; the
+  // rest of R0 (K0 > 128) is retained in the first round after it, as forced picks, and every
+  // value the pass gave stays a valid upper bound (values only shrink as the basis grows).
+  const int K0c = std::min(K0, mapk::kCholMax);
+  const bool project = K0 > 0 && K0 < K;
   if (K0 < K && !project) {
     ++c->counters.launches;
     CU_TRY(mapk::launch_row_sqnorm(vis, BN, g.D, static_cast<float*>(c->sqn.p), st));
@@ -445,12 +449,16 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, const int32_t*
       c->counters.launches += 3;
       CU_TRY(mapk::launch_sel_choose(s, st));
       {
-        GemmDesc d0 = d;              // only the K0 x K0 corner of the block
-        d0.M = K0; d0.N = K0;
+        GemmDesc d0 = d;              // only the K0c x K0c corner of the block
+        d0.M = K0c; d0.N = K0c;
         take_list(d0);
         MAP_TRY(gemm(c, d0, st));
       }
-      CU_TRY(mapk::launch_sel_chol(s, st));
+      {
+        mapk::SelState sc = s;        // the first K0c tokens of R0
+        sc.K0 = K0c;
+        CU_TRY(mapk::launch_sel_chol(sc, st));
+      }
       ++c->counters.select_rounds;
       // every candidate's exact value: one tensor-core pass over V against the R0 basis
       GemmDesc pd{};
@@ -473,12 +481,12 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, const int32_t*
         CU_TRY(mapk::launch_sel_proj_done(s, st));
         return MAP_OK;
       };
-      pd.N = K0 <= 96 ? 96 : kProjMaxBasis;   // basis columns the R0 projection needs
+      pd.N = K0c <= 96 ? 96 : kProjMaxBasis;   // basis columns the R0 projection needs
       MAP_TRY(project_all(true));
       pd.N = kProjMaxBasis;
-      // one greedy round, then the images still selecting are projected again on their whole
-      // basis (when it has at most kReprojMax vectors): exact values for every candidate make
-      // the next active set the true top S
+      // one round (greedy, or the rest of R0 when K0 > K0c), then the images still selecting are
+      // projected again on their whole basis (when it has at most kReprojMax vectors): exact
+      // values for every candidate make the next active set the true top S
       c->counters.launches += 4;
       CU_TRY(mapk::launch_sel_choose(s, st));
       take_list(d);

@@ -391,7 +391,8 @@ def test_batched_serving_config_every_image():
 
 def test_high_token_config_every_image():
     """16 images, N = 7290, D = 3584, k = 405, questions up to 512 tokens (two column tiles
-    in Eq. 3) and K0 = 202 (no projection pass; coordinates in global memory)."""
+    in Eq. 3) and K0 = 202 (the projection pass on the first 128 R0 tokens, the other 74
+    retained as forced picks in the next round; coordinates in global memory)."""
     assert W.make_lens(W.WORKLOADS["c4"]).max() > 256
     _full_batch_parity("c4")
 
