@@ -500,6 +500,8 @@ def main():
     ap.add_argument("--only-qcts", action="store_true",
                     help="run only the teacher-selection measurement (for profiling), print its JSON")
     ap.add_argument("--qcts-samples", type=int, default=W.ATTENTION_WORKLOADS["q1"].B)
+    ap.add_argument("--only-config", choices=["c0", "c4"], default=None,
+                    help="time only that configuration through map_prune (for profiling), print its JSON")
     ap.add_argument("--only-distill", action="store_true",
                     help="run only the distillation-step measurement (for profiling), print its JSON")
     ap.add_argument("--batch", type=int, default=WORKLOAD.B, help="images per GPU (profiling on a smaller case)")
@@ -516,6 +518,12 @@ def main():
     ws, rank, local = dist_env()
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
+    if args.only_config:
+        if rank == 0:
+            hbm, bf16_burst, _, _ = measured_peaks()
+            print(json.dumps(bench_config(mb, dev, torch.cuda.current_stream(), args.only_config, args.steps,
+                                          bf16_burst, hbm)))
+        return 0
     if args.only_distill:
         if rank == 0:
             print(json.dumps(bench_distill(mb, dev, torch.cuda.current_stream(), args.steps, False)))
