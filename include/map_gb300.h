@@ -116,7 +116,7 @@ int map_score(map_ctx *ctx, const void *text_feats, const void *vis_feats,
  * k > N is MAP_EINVAL.  Supported: N <= 16384; k <= 4096 for plain top-k (lambda = 0 or
  * K0 = k), k <= 1024 with the diversity term (MAP_EUNSUPPORTED beyond).
  * Asynchronous like the other calls: after its first rounds the selection runs as a
- * device-side loop (a CUDA graph whose WHILE node repeats two rounds while an image still
+ * device-side loop (a CUDA graph whose WHILE node repeats a round while an image still
  * selects; built on the first call of a shape and workspace, then cached in the context), so
  * the host never waits for it.  A device-side failure (a bounded wait that ran out, or the
  * loop's iteration cap, which no input reaches) is reported by map_status.

@@ -17,7 +17,6 @@ using mapk::GemmDesc;
 
 namespace {
 
-constexpr int kSelS = 256;          // active-set size of the selection (Gram block rows)
 constexpr int kMaxKDiverse = 1024;  // k limit when the diversity term is on (shared-memory staging)
 constexpr int kProjMaxBasis = 128;  // basis vectors one projection pass takes
 constexpr int kMaxK = 4096;
@@ -61,7 +60,7 @@ struct map_ctx {
   int deferred = MAP_OK;
   long long wait_ns = 0;            // GEMM role-wait limit (0: the kernels' default)
   mapk::SelLoopCache* loops = nullptr;   // cached graphs of the selection's device-side round loop
-  long long* loop_iters_total = nullptr; // device: loop iterations run so far (two rounds each)
+  long long* loop_iters_total = nullptr; // device: loop iterations run so far (one round each)
 };
 
 namespace {
@@ -353,7 +352,7 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, const int32_t*
   if (g.lambda == 0.f) K0 = K;        // values are p_hat alone: plain top-K
   if (K0 < K && K > kMaxKDiverse) return MAP_EUNSUPPORTED;
   const long long BN = static_cast<long long>(B) * N;
-  const int S = kSelS, R = ((kSelS + K + 15) / 16) * 16;   // row stride of Vg and G (16-byte rows)
+  const int S = mapk::kActiveSlots, R = ((S + K + 15) / 16) * 16;   // row stride of Vg and G (16-byte rows)
 
   mapk::SelState s{};
   const int KP = ((K + 3) / 4) * 4;
@@ -410,10 +409,10 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, const int32_t*
 
   // With 0 < K0 < K, one tensor-core pass over V after the first R0 tokens gives every
   // candidate its exact value on their basis (and ||v||^2); otherwise values start from
-  // p_hat * ||v||^lambda.  The first K0c <= 128 tokens of R0 are factored before the pass; the
-  // rest of R0 (K0 > 128) is retained in the first round after it, as forced picks, and every
+  // p_hat * ||v||^lambda.  The first K0c <= min(128, S) tokens of R0 are factored before the pass;
+  // the rest of R0 is retained in the rounds after it, as forced picks, and every
   // value the pass gave stays a valid upper bound (values only shrink as the basis grows).
-  const int K0c = std::min(K0, mapk::kCholMax);
+  const int K0c = std::min({K0, mapk::kCholMax, S});
   const bool project = K0 > 0 && K0 < K;
   if (K0 < K && !project) {
     ++c->counters.launches;
@@ -487,7 +486,7 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, const int32_t*
       // one round (greedy, or the rest of R0 when K0 > K0c), then the images still selecting are
       // projected again on their whole basis (when it has at most kReprojMax vectors): exact
       // values for every candidate make the next active set the true top S
-      c->counters.launches += 4;
+      c->counters.launches += 5;
       CU_TRY(mapk::launch_sel_choose(s, st));
       take_list(d);
       MAP_TRY(gemm(c, d, st));
@@ -495,14 +494,14 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, const int32_t*
       ++c->counters.select_rounds;
       MAP_TRY(project_all(false));
     }
-    // The remaining rounds run as a device-side loop (a CUDA graph whose WHILE node repeats two
-    // rounds while an image still selects): the host never waits for them.
+    // The remaining rounds run as a device-side loop (a CUDA graph whose WHILE node repeats a
+    // round while an image still selects): the host never waits for them.
     if (!c->loops) c->loops = mapk::sel_loop_cache_create();
     if (!c->loops) return MAP_ENOMEM;
     GemmDesc dl = d;
     dl.wait_ns = c->wait_ns;
     ++c->counters.launches;            // the test kernel ahead of the loop; iterations are counted on the device
-    CU_TRY(mapk::launch_sel_loop(c->loops, s, dl, c->num_sms, static_cast<int>((cap + 1) / 2), loop_iters,
+    CU_TRY(mapk::launch_sel_loop(c->loops, s, dl, c->num_sms, static_cast<int>(cap), loop_iters,
                                  c->loop_iters_total, st));
   } else {
     ++c->counters.launches;
@@ -1069,7 +1068,7 @@ int map_get_counters(map_ctx* ctx, map_counters* out) {
       cudaMemcpy(&iters, ctx->loop_iters_total, sizeof(iters), cudaMemcpyDeviceToHost) != cudaSuccess)
     return MAP_ECUDA;
   out->launches += mapk::kSelLoopKernelsPerIter * iters;
-  out->select_rounds += 2 * iters;
+  out->select_rounds += iters;
   return MAP_OK;
 }
 

@@ -46,7 +46,7 @@ CtxView ctx_view(map_ctx* c);
 namespace {
 
 constexpr size_t kNoAllocScratchBytes = MAP_NOALLOC_SCRATCH_BYTES;
-constexpr int kSelS = 256;
+constexpr int kSelS = mapk::kActiveSlots;
 constexpr int kMaxDevices = 64;
 constexpr int kMaxN = 16384;
 constexpr int kMaxK = 4096;          // plain top-k
@@ -174,10 +174,10 @@ extern "C" int map_select_noalloc(map_ctx* ctx, const float* scores, const void*
     d.epi = mapk::EPI_F32; d.status = v.status;
     const long long cap = 8LL * (K + N / S) + 64;
     long long rounds = 0;
-    int burst = (K0 + S - 1) / S + 6;
+    int burst = (K0 + mapk::kRoundPicks - 1) / mapk::kRoundPicks + 6;
     for (;;) {
       for (int r = 0; r < burst; ++r) {
-        *v.launches += 5;
+        *v.launches += 6;
         if ((rc = rc_of(mapk::launch_sel_choose(s, st))) != MAP_OK) return rc;
         cudaError_t e = mapk::launch_gemm(d, v.num_sms, st);
         if (e == cudaErrorInvalidValue) return MAP_EUNSUPPORTED;

@@ -22,6 +22,8 @@
 //            new basis tokens into a compact buffer Vg.
 //   gram   : G_blk = Vg[A] Vg[A u new basis]^T on tcgen05 (gemm_tc.cu).
 //   update : bring each A member's coordinates up to date (exact values).
+//   resgram: replace G[A, A] by the Gram matrix of the residuals on the current basis, so
+//            that the picks need only the coordinates added during the round.
 //   greedy : pick while the best exact value in A beats the largest bound outside A (theta):
 //            such a pick is the exact argmax over all candidates.  Each pick updates the
 //            other A members.  Values are compared as the 64-bit key (value bits, ~index),
@@ -314,11 +316,11 @@ __global__ void __launch_bounds__(kGatherThreads) sel_gather_kernel(SelState s) 
 }
 
 // ------------------------------------------------------------------ coordinates
-// Per-slot coordinate rows: [S][P] in shared memory, P = KP rounded up to 8, plus 4, so that
-// eight lanes reading 16 bytes each from eight rows hit disjoint banks.
+// Per-slot coordinate rows in shared memory have a pitch of 4 (mod 8) floats, so that eight
+// lanes reading 16 bytes each from eight rows hit disjoint banks.
 constexpr int kChunk = 32;
-constexpr int kRegCoords = 128;
 constexpr int kUpdSlots = 32;
+constexpr int kRoundPitch = kRoundPicks + 4;
 
 __host__ __device__ inline int coord_pitch(int KP) { return ((KP + 7) / 8) * 8 + 4; }
 
@@ -529,26 +531,149 @@ __global__ void __launch_bounds__(kCholThreads, 1) sel_chol_kernel(SelState s) {
   }
 }
 
-// ------------------------------------------------------------------ greedy
-// One CTA of S threads per image; thread = active slot.  Every active token's coordinates
-// are current (sel_update_kernel ran first); they are held in the slot rows ([S][P] shared
-// memory when it fits, else the tokens' global cache rows) and, for the first kRegCoords,
-// in registers.  The picks take one block barrier each: the winning slot is carried in the
-// low bits of the key, and every slot's residual is published in shared memory, so all
-// threads derive the basis update from the same values; the winner's row is read as 16-byte
-// broadcasts and its Gram entry is loaded while the dot product runs.
+// ------------------------------------------------------------------ residual Gram
+// When a round's picks start, every active token's coordinates are current on the c0 basis
+// vectors of the round (sel_update_kernel).  Over that basis the residual Gram matrix of
+// the active set is
+//   G'[i][k] = <v_i, v_k> - sum_{q < c0} e_q[i] e_q[k]   (the inner product of the residuals),
+// and a pick then needs only the coordinates added during the round (sel_greedy_kernel).
+// It replaces the A x A part of the Gram block in place.  One CTA of 64 threads per 32 x 32
+// tile of the upper triangle (the matrix is symmetric: the mirrored tile is written from the
+// same values), 4 x 4 outputs per thread; the coordinates are staged in 16-column chunks,
+// transposed, in two shared buffers, the next chunk loaded during the products of the
+// current one.  Small tiles keep several CTAs on every SM, so the chunk loop's latency is
+// hidden, with few images (c0 is large) as with many.
+constexpr int kRgTile = 32, kRgChunk = 16, kRgPad = kRgTile + 4, kRgThreads = 64;
 
-template <bool SMEM>
-struct Coords {
-  float* Es;            // SMEM: [S][P]
-  float* Ec;            // global cache rows
-  long long base;
-  int P, KP;
-  __device__ __forceinline__ float* row(int slot, int tok) const {
-    if constexpr (SMEM) return Es + static_cast<long long>(slot) * P;
-    else return Ec + (base + tok) * KP;
+__global__ void __launch_bounds__(kRgThreads) sel_resgram_kernel(SelState s) {
+  pdl_enter();
+  // two buffers of both operands' chunks; after the products, the output tile
+  __shared__ __align__(16) float sbuf[4 * kRgChunk * kRgPad];
+  static_assert(4 * kRgChunk * kRgPad >= kRgTile * (kRgTile + 1), "tile staging");
+  float(*Ei)[kRgChunk][kRgPad] = reinterpret_cast<float(*)[kRgChunk][kRgPad]>(sbuf);
+  float(*Ek)[kRgChunk][kRgPad] = reinterpret_cast<float(*)[kRgChunk][kRgPad]>(sbuf + 2 * kRgChunk * kRgPad);
+  __shared__ int toki[kRgTile], tokk[kRgTile];
+  const int b = blockIdx.y;
+  if (s.done[b]) return;
+  const int c0 = s.nbasis[b];
+  if (c0 == 0) return;
+  const int S = s.S, KP = s.KP;
+  int t = blockIdx.x, ti = 0;
+  const int T = S / kRgTile;
+  while (t >= T - ti) { t -= T - ti; ++ti; }
+  const int tk = ti + t;
+  const int32_t* aslot = s.aslot + static_cast<long long>(b) * S;
+  const int tid = threadIdx.x;
+  if (tid < kRgTile) toki[tid] = aslot[ti * kRgTile + tid];
+  else tokk[tid - kRgTile] = aslot[tk * kRgTile + tid - kRgTile];
+  // a tile whose rows or columns are all empty slots writes nothing
+  const bool any_i = __syncthreads_or(tid < kRgTile && toki[tid] >= 0);
+  const bool any_k = __syncthreads_or(tid < kRgTile && tokk[tid] >= 0);
+  if (!any_i || !any_k) return;
+  const long long base = static_cast<long long>(b) * s.N;
+  // staging: threads 0-31 the rows of the tile's row slots, 32-63 those of its column slots
+  const int lr = tid & (kRgTile - 1);
+  const int ltok = tid < kRgTile ? toki[lr] : tokk[lr];
+  const float* row = ltok >= 0 ? s.Ec + (base + ltok) * KP : nullptr;
+  float(*Eop)[kRgChunk][kRgPad] = tid < kRgTile ? Ei : Ek;
+  auto load16 = [&](int q, float* x) {
+#pragma unroll
+    for (int j = 0; j < 16; ++j) x[j] = 0.f;
+    if (!row) return;
+    if (q + 16 <= c0) {
+#pragma unroll
+      for (int j = 0; j < 16; j += 4) {
+        const float4 u = *reinterpret_cast<const float4*>(row + q + j);
+        x[j] = u.x; x[j + 1] = u.y; x[j + 2] = u.z; x[j + 3] = u.w;
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < 16; ++j)
+        if (q + j < c0) x[j] = row[q + j];
+    }
+  };
+  const int tx = tid & 7, ty = tid >> 3;             // outputs: rows ty*4 .. +3, columns tx*4 .. +3
+  float acc[4][4];
+#pragma unroll
+  for (int r = 0; r < 4; ++r)
+#pragma unroll
+    for (int c = 0; c < 4; ++c) acc[r][c] = 0.f;
+  float x[16];
+  load16(0, x);
+  int buf = 0;
+#pragma unroll
+  for (int j = 0; j < 16; ++j) Eop[0][j][lr] = x[j];
+  __syncthreads();
+  for (int q0 = 0; q0 < c0; q0 += kRgChunk, buf ^= 1) {
+    const bool more = q0 + kRgChunk < c0;
+    if (more) load16(q0 + kRgChunk, x);              // next chunk in flight during the products
+#pragma unroll
+    for (int q = 0; q < kRgChunk; ++q) {
+      const float4 a = *reinterpret_cast<const float4*>(&Ei[buf][q][ty * 4]);
+      const float4 c = *reinterpret_cast<const float4*>(&Ek[buf][q][tx * 4]);
+      const float av[4] = {a.x, a.y, a.z, a.w}, cv[4] = {c.x, c.y, c.z, c.w};
+#pragma unroll
+      for (int r = 0; r < 4; ++r)
+#pragma unroll
+        for (int cc = 0; cc < 4; ++cc) acc[r][cc] = fmaf(av[r], cv[cc], acc[r][cc]);
+    }
+    if (more) {                                      // the other buffer was last read a chunk ago
+#pragma unroll
+      for (int j = 0; j < 16; ++j) Eop[buf ^ 1][j][lr] = x[j];
+    }
+    __syncthreads();
   }
-};
+  // G' = G - acc through a shared tile, so that both the tile and its mirror are read and
+  // written in whole rows (coalesced)
+  float(*Tt)[kRgTile + 1] = reinterpret_cast<float(*)[kRgTile + 1]>(sbuf);
+#pragma unroll
+  for (int r = 0; r < 4; ++r)
+#pragma unroll
+    for (int cc = 0; cc < 4; ++cc) Tt[ty * 4 + r][tx * 4 + cc] = acc[r][cc];
+  __syncthreads();
+  float* Gb = s.G + static_cast<long long>(b) * S * s.R;
+  constexpr int kRowsPer = kRgTile * kRgTile / kRgThreads;   // rows of the tile per thread
+  {
+    const int c = tid & (kRgTile - 1), r0 = tid / kRgTile;
+    const bool okc = tokk[c] >= 0;
+    float* g0 = Gb + static_cast<long long>(ti * kRgTile) * s.R + tk * kRgTile + c;
+    float gv[kRowsPer];                              // every load in flight before the stores
+#pragma unroll
+    for (int m = 0; m < kRowsPer; ++m) {
+      const int r = r0 + m * (kRgThreads / kRgTile);
+      gv[m] = okc && toki[r] >= 0 ? g0[static_cast<long long>(r) * s.R] : 0.f;
+    }
+#pragma unroll
+    for (int m = 0; m < kRowsPer; ++m) {
+      const int r = r0 + m * (kRgThreads / kRgTile);
+      if (okc && toki[r] >= 0) {
+        const float v = gv[m] - Tt[r][c];
+        g0[static_cast<long long>(r) * s.R] = v;
+        Tt[r][c] = v;
+      }
+    }
+    if (ti != tk) {
+      __syncthreads();
+      float* m0 = Gb + static_cast<long long>(tk * kRgTile) * s.R + ti * kRgTile + c;
+#pragma unroll
+      for (int m = 0; m < kRowsPer; ++m) {         // row r of the mirror: column r of the tile
+        const int r = r0 + m * (kRgThreads / kRgTile);
+        if (tokk[r] >= 0 && toki[c] >= 0) m0[static_cast<long long>(r) * s.R] = Tt[c][r];
+      }
+    }
+  }
+}
+
+// ------------------------------------------------------------------ greedy
+// One CTA of S threads per image; thread = active slot.  The A x A part of the Gram block
+// holds the residual Gram matrix G' on the c0 basis vectors of the round (above), so a pick
+// of slot j updates slot i with the coordinates added in this launch only:
+//   e_new[i] = (G'[j][i] - sum_{c0 <= q < nb} e_q[j] e_q[i]) / r_j.
+// Each slot keeps its round coordinates in a shared-memory row: its own side of the dot
+// products, and the other side for every thread (16-byte broadcasts) when that slot wins.  The picks take one block barrier each: the winning slot is carried in the low bits
+// of the key, and every slot's residual is published in shared memory, so all threads
+// derive the basis update from the same values; the winner's G' entry is loaded while the
+// dot product runs.  At most kRoundPicks picks per launch (the next round continues).
 
 // key of a candidate inside the round: (value bits, 0xFFFF - token, slot); the upper 48
 // bits order like make_key (value descending, lower token first).
@@ -565,8 +690,7 @@ __device__ __forceinline__ uint64_t warp_max_key(uint32_t hi, uint32_t lo) {
   return (static_cast<uint64_t>(h) << 32) | l;
 }
 
-template <bool SMEM>
-__global__ void __launch_bounds__(256, 1) sel_greedy_kernel(SelState s) {
+__global__ void __launch_bounds__(kActiveSlots, 1) sel_greedy_kernel(SelState s) {
   pdl_enter();
   extern __shared__ __align__(16) float shf[];
   __shared__ uint64_t wkey[2][32];
@@ -576,22 +700,22 @@ __global__ void __launch_bounds__(256, 1) sel_greedy_kernel(SelState s) {
   float* r2s = shf;                                  // [S] published residuals
   float* sqs = r2s + S;                              // [S]
   int32_t* tks = reinterpret_cast<int32_t*>(sqs + S);   // [S] tokens of the slots
-  int32_t* ends = tks + S;                           // [S] valid coordinates of the slots at the end
-  int32_t* pk_tok = ends + S;                        // [KP] this launch's picks
-  float* pk_r2 = reinterpret_cast<float*>(pk_tok + KP);  // [KP] their residuals (-1: no basis vector)
-  const Coords<SMEM> E{pk_r2 + KP, s.Ec, static_cast<long long>(b) * s.N, coord_pitch(KP), KP};
-  const long long base = E.base;
+  int32_t* ends = tks + S;                           // [S] round coordinates of the slots at the end
+  int32_t* pk_tok = ends + S;                        // [kRoundPicks] this launch's picks
+  float* pk_r2 = reinterpret_cast<float*>(pk_tok + kRoundPicks);  // their residuals (-1: no basis vector)
+  float* Er = pk_r2 + kRoundPicks;                   // [S][kRoundPitch] round coordinates
+  const long long base = static_cast<long long>(b) * s.N;
   const int slot = threadIdx.x;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
   const int tok = s.aslot[static_cast<long long>(b) * S + slot];
   const float* Gb = s.G + static_cast<long long>(b) * S * R;
   int nb = s.nbasis[b], np = s.npicks[b];
+  const int c0 = nb;
   const bool forced = s.mode[b] == 1;
   const uint64_t th48 = theta48(s.theta[b]);
-  float* me = tok >= 0 ? E.row(slot, tok) : nullptr;
+  float* me = Er + slot * kRoundPitch;
 
   float r2 = 0.f, sq = 0.f, p = 0.f, val = 0.f;
-  const int c0 = nb;                                 // coordinates cached at the start (all current)
   int mine = nb;                                     // valid coordinates at the end
   bool alive = false;
   if (tok >= 0) {
@@ -604,21 +728,10 @@ __global__ void __launch_bounds__(256, 1) sel_greedy_kernel(SelState s) {
     r2 = s.r2[base + tok];
     sq = s.sqn[base + tok];
   }
-  if constexpr (SMEM) {
-    // the slot's row: cached coordinates, zeros after them
-    float4* row4 = reinterpret_cast<float4*>(E.row(slot, tok));
-    const float4* g = tok >= 0 ? reinterpret_cast<const float4*>(s.Ec + (base + tok) * KP) : nullptr;
-    for (int q = 0; q < E.P; q += 4) {
-      float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (tok >= 0 && q < c0) {
-        v = g[q / 4];
-        if (q + 1 >= c0) v.y = 0.f;
-        if (q + 2 >= c0) v.z = 0.f;
-        if (q + 3 >= c0) v.w = 0.f;
-      }
-      row4[q / 4] = v;
-    }
-    if (slot < 8) reinterpret_cast<float4*>(E.row(S, 0))[slot] = make_float4(0.f, 0.f, 0.f, 0.f);
+  {
+    // zero rows: the unrolled dot products read a winner's row up to the next multiple of 32
+    float4* row4 = reinterpret_cast<float4*>(me);
+    for (int q = 0; q < kRoundPitch / 4; ++q) row4[q] = make_float4(0.f, 0.f, 0.f, 0.f);
   }
   tks[slot] = tok;
   if (tok >= 0) val = sel_value(p, r2, sq, s.lambda, s.tau);
@@ -626,17 +739,8 @@ __global__ void __launch_bounds__(256, 1) sel_greedy_kernel(SelState s) {
   sqs[slot] = sq;
   __syncthreads();
 
-  // the first nreg coordinates of this slot, in registers for the picks
-  float ereg[kRegCoords];
-  const int nreg = min(nb, kRegCoords) & ~3;
-#pragma unroll
-  for (int g = 0; g < kRegCoords / 4; ++g) {
-    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (alive && 4 * g < nreg) v = *reinterpret_cast<const float4*>(me + 4 * g);
-    ereg[4 * g] = v.x; ereg[4 * g + 1] = v.y; ereg[4 * g + 2] = v.z; ereg[4 * g + 3] = v.w;
-  }
-
-  for (int step = 0, buf = 0; np < s.K; ++step, buf ^= 1) {
+  int nr = 0;                                        // round coordinates so far (uniform)
+  for (int step = 0, buf = 0; np < s.K && step < kRoundPicks; ++step, buf ^= 1) {
     {
       const uint32_t vb = alive ? __float_as_uint(val > 0.f ? val : 0.f) : 0u;
       const uint32_t lo = alive ? ((0xFFFFu - static_cast<uint32_t>(tok)) << 16) | static_cast<uint32_t>(slot) : 0u;
@@ -667,54 +771,32 @@ __global__ void __launch_bounds__(256, 1) sel_greedy_kernel(SelState s) {
       if (alive) {
         const float gji = Gb[static_cast<long long>(jslot) * R + slot];   // in flight during the dot product
         const float rinv = 1.0f / sqrtf(r2j);
-        const float* cj = E.row(jslot, jt);
+        const float* cj = Er + jslot * kRoundPitch;
         float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
-        if constexpr (SMEM) {
-          // 32 coordinates per branch, so the loads of a block issue together; shared rows
-          // are zero past their valid coordinates and ereg is zero past nreg
+        // 32 coordinates per branch, so that the loads of a block issue together; rows are
+        // zero past the round's coordinates
 #pragma unroll
-          for (int blk = 0; blk < kRegCoords / 32; ++blk) {
-            if (32 * blk < nreg) {
+        for (int blk = 0; blk < kRoundPicks / 32; ++blk) {
+          if (32 * blk < nr) {
 #pragma unroll
-              for (int g = 8 * blk; g < 8 * blk + 8; ++g) {
-                const float4 c = *reinterpret_cast<const float4*>(cj + 4 * g);
-                a0 = fmaf(c.x, ereg[4 * g], a0);
-                a1 = fmaf(c.y, ereg[4 * g + 1], a1);
-                a2 = fmaf(c.z, ereg[4 * g + 2], a2);
-                a3 = fmaf(c.w, ereg[4 * g + 3], a3);
-              }
-            }
-          }
-        } else {
-#pragma unroll
-          for (int g = 0; g < kRegCoords / 4; ++g) {
-            if (4 * g < nreg) {
+            for (int g = 8 * blk; g < 8 * blk + 8; ++g) {
               const float4 c = *reinterpret_cast<const float4*>(cj + 4 * g);
-              a0 = fmaf(c.x, ereg[4 * g], a0);
-              a1 = fmaf(c.y, ereg[4 * g + 1], a1);
-              a2 = fmaf(c.z, ereg[4 * g + 2], a2);
-              a3 = fmaf(c.w, ereg[4 * g + 3], a3);
+              const float4 m = *reinterpret_cast<const float4*>(me + 4 * g);
+              a0 = fmaf(c.x, m.x, a0);
+              a1 = fmaf(c.y, m.y, a1);
+              a2 = fmaf(c.z, m.z, a2);
+              a3 = fmaf(c.w, m.w, a3);
             }
           }
         }
-        int q = nreg;
-#pragma unroll 4
-        for (; q + 4 <= nb; q += 4) {
-          const float4 c = *reinterpret_cast<const float4*>(cj + q);
-          const float4 m = *reinterpret_cast<const float4*>(me + q);
-          a0 = fmaf(c.x, m.x, a0);
-          a1 = fmaf(c.y, m.y, a1);
-          a2 = fmaf(c.z, m.z, a2);
-          a3 = fmaf(c.w, m.w, a3);
-        }
-        for (; q < nb; ++q) a0 = fmaf(cj[q], me[q], a0);
         const float e = (gji - ((a0 + a1) + (a2 + a3))) * rinv;
-        me[nb] = e;
+        me[nr] = e;
         r2 = fmaf(-e, e, r2);
         val = sel_value(p, r2, sq, s.lambda, s.tau);
         r2s[slot] = r2;
       }
       ++nb;
+      ++nr;
     }
     ++np;
   }
@@ -741,17 +823,15 @@ __global__ void __launch_bounds__(256, 1) sel_greedy_kernel(SelState s) {
     s.r2[base + tok] = r2;
     s.U[base + tok] = val;
   }
-  if constexpr (SMEM) {
-    // coordinates [c0, mine) of every slot's row, one warp per row
-    ends[slot] = tok >= 0 ? mine : c0;
-    __syncthreads();
-    for (int r = warp; r < S; r += nwarps) {
-      const int t = tks[r], end = ends[r];
-      if (t < 0) continue;
-      float* g = s.Ec + (base + t) * KP;
-      const float* src = E.row(r, t);
-      for (int q = c0 + lane; q < end; q += 32) g[q] = src[q];
-    }
+  // coordinates [c0, mine) of every slot: its round row, one warp per row
+  ends[slot] = tok >= 0 ? mine : c0;
+  __syncthreads();
+  for (int r = warp; r < S; r += nwarps) {
+    const int t = tks[r], end = ends[r];
+    if (t < 0) continue;
+    float* g = s.Ec + (base + t) * KP;
+    const float* src = Er + r * kRoundPitch;
+    for (int q = c0 + lane; q < end; q += 32) g[q] = src[q - c0];
   }
   if (threadIdx.x == 0) {
     s.nbasis[b] = nb;
@@ -835,11 +915,14 @@ __global__ void sel_loop_init_kernel(SelState s, cudaGraphConditionalHandle h, i
   }
 }
 
-// Last node of the WHILE body: run another two rounds while an image still selects, no kernel
-// has reported an error and the iteration cap has not been reached (then ST_INTERNAL).
+// Last node of the WHILE body: run another round while an image still selects, no kernel
+// has reported an error and the iteration cap has not been reached (then ST_INTERNAL).  It
+// also clears the image-list count the round's choose appended to (the Gram block has read
+// it), so that the next iteration's choose starts from zero on the same counter.
 __global__ void sel_loop_cond_kernel(SelState s, cudaGraphConditionalHandle h, int32_t* iters, int cap_iters,
                                      long long* iters_total) {
   if (threadIdx.x == 0) {
+    s.bcount[s.bc_par] = 0;
     const int it = *iters + 1;
     *iters = it;
     *iters_total += 1;
@@ -853,11 +936,9 @@ __global__ void sel_loop_cond_kernel(SelState s, cudaGraphConditionalHandle h, i
 
 size_t sel_init_smem(int N, int K0) { return (static_cast<size_t>(N) + pow2_at_least(std::max(K0, 1))) * 8; }
 size_t sel_choose_smem(int N) { return static_cast<size_t>(N) * 8; }
-size_t sel_greedy_smem(int KP, int S, bool* smem_coords) {
-  const size_t small = static_cast<size_t>(S) * 16 + static_cast<size_t>(KP) * 8;
-  const size_t es = (static_cast<size_t>(coord_pitch(KP)) * S + 32) * 4;   // + zeros read past the last row
-  *smem_coords = small + es <= 200 * 1024;
-  return *smem_coords ? small + es : small;
+size_t sel_greedy_smem(int S) {
+  return static_cast<size_t>(S) * 16 + static_cast<size_t>(kRoundPicks) * 8 +
+         static_cast<size_t>(S) * kRoundPitch * 4;
 }
 size_t sel_chol_smem(int K0) {
   return (static_cast<size_t>(K0) * ((K0 + 3) & ~3) + static_cast<size_t>(K0) * coord_pitch(K0)) * 4;
@@ -882,22 +963,19 @@ cudaError_t launch_sel_choose(const SelState& s, cudaStream_t st) {
 }
 
 cudaError_t launch_sel_greedy(const SelState& s, cudaStream_t st) {
+  if (s.S != kActiveSlots) return cudaErrorInvalidValue;
   const size_t um = sel_update_smem(s.KP);
   cudaError_t e = cudaFuncSetAttribute(sel_update_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(um));
   if (e != cudaSuccess) return e;
   e = launch_k(sel_update_kernel, dim3((s.S + kUpdSlots - 1) / kUpdSlots, s.B), dim3(kUpdSlots * kUpdWarps), um, st, s);
   if (e != cudaSuccess) return e;
-  bool in_smem = false;
-  const size_t sm = sel_greedy_smem(s.KP, s.S, &in_smem);
-  if (in_smem) {
-    e = cudaFuncSetAttribute(sel_greedy_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(sm));
-    if (e != cudaSuccess) return e;
-    return launch_k(sel_greedy_kernel<true>, dim3(s.B), dim3(s.S), sm, st, s);
-  } else {
-    e = cudaFuncSetAttribute(sel_greedy_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(sm));
-    if (e != cudaSuccess) return e;
-    return launch_k(sel_greedy_kernel<false>, dim3(s.B), dim3(s.S), sm, st, s);
-  }
+  const int T = s.S / kRgTile;
+  e = launch_k(sel_resgram_kernel, dim3(T * (T + 1) / 2, s.B), dim3(kRgThreads), 0, st, s);
+  if (e != cudaSuccess) return e;
+  const size_t sm = sel_greedy_smem(s.S);
+  e = cudaFuncSetAttribute(sel_greedy_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(sm));
+  if (e != cudaSuccess) return e;
+  return launch_k(sel_greedy_kernel, dim3(s.B), dim3(s.S), sm, st, s);
 }
 
 cudaError_t launch_sel_chol(const SelState& s, cudaStream_t st) {
@@ -977,7 +1055,8 @@ std::vector<long long> loop_key(const SelState& s, const GemmDesc& g, int num_sm
           g.wait_ns, num_sms, cap_iters, pbits(iters), pbits(iters_total)};
 }
 
-// Builds the graph: [test kernel] -> WHILE { 2 x (choose + gather, Gram, update + greedy); test }.
+// Builds the graph: [test kernel] -> WHILE { choose + gather, Gram, update + residual Gram +
+// greedy; test }.
 cudaError_t build_loop(SelLoopCache* c, const SelState& s, const GemmDesc& gram, int num_sms, int cap_iters,
                        int32_t* iters, long long* iters_total, SelLoopEntry& out) {
   cudaError_t e = cudaSuccess;
@@ -1012,13 +1091,11 @@ cudaError_t build_loop(SelLoopCache* c, const SelState& s, const GemmDesc& gram,
     return fail(e);
   pdl_disabled() = true;
   SelState r = s;
-  for (int round = 0; round < 2 && e == cudaSuccess; ++round) {
+  {
     GemmDesc d = gram;
     d.bcount = r.bcount + r.bc_par;              // the count this round's choose appends to
-    if ((e = launch_sel_choose(r, c->cap)) != cudaSuccess) break;
-    if ((e = launch_gemm(d, num_sms, c->cap)) != cudaSuccess) break;
-    r.bc_par ^= 1;
-    e = launch_sel_greedy(r, c->cap);
+    if ((e = launch_sel_choose(r, c->cap)) == cudaSuccess && (e = launch_gemm(d, num_sms, c->cap)) == cudaSuccess)
+      e = launch_sel_greedy(r, c->cap);
   }
   if (e == cudaSuccess) e = launch_k(sel_loop_cond_kernel, dim3(1), dim3(32), 0, c->cap, r, h, iters, cap_iters, iters_total);
   pdl_disabled() = false;

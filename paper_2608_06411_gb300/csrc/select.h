@@ -52,10 +52,15 @@ struct SelState {
 
 size_t sel_init_smem(int N, int K0);
 size_t sel_choose_smem(int N);
-size_t sel_greedy_smem(int KP, int S, bool* smem_coords);
+// Active-set size (Gram block rows, threads of the greedy CTA) and the most picks one greedy
+// launch makes (their coordinates are held in registers; the next round continues).
+constexpr int kActiveSlots = 256;
+constexpr int kRoundPicks = 128;
+size_t sel_greedy_smem(int S);
 cudaError_t launch_sel_init(const SelState& s, cudaStream_t st);
 cudaError_t launch_sel_choose(const SelState& s, cudaStream_t st);
-// sel_update_kernel (coordinates of the active tokens up to the current basis), then the picks.
+// sel_update_kernel (coordinates of the active tokens up to the current basis), the residual
+// Gram matrix of the active set on that basis, then the picks.
 cudaError_t launch_sel_greedy(const SelState& s, cudaStream_t st);
 // The K0 forced R0 picks from the Gram block G[R0, R0] of a forced round (K0 <= kCholMax, <= S).
 cudaError_t launch_sel_chol(const SelState& s, cudaStream_t st);
@@ -74,8 +79,9 @@ cudaError_t launch_sel_proj_done(const SelState& s, cudaStream_t st);
 
 // ------------------------------------------------------------------ device-side round loop
 // The selection rounds after the first ones run as a CUDA graph: a kernel node that tests
-// whether any image still selects, then a WHILE conditional node whose body is two rounds
-// (choose + gather, Gram block, coordinate update + greedy picks) followed by the same test.
+// whether any image still selects, then a WHILE conditional node whose body is one round
+// (choose + gather, Gram block, coordinate update + residual Gram + greedy picks) followed by
+// the same test.
 // The host never waits for the rounds.  Graphs are cached per shape and workspace.
 struct GemmDesc;
 struct SelLoopCache;
@@ -86,6 +92,6 @@ void sel_loop_cache_destroy(SelLoopCache* c);
 // selecting the loop stops and sets ST_INTERNAL.
 cudaError_t launch_sel_loop(SelLoopCache* cache, const SelState& s, const GemmDesc& gram, int num_sms, int cap_iters,
                             int32_t* iters, long long* iters_total, cudaStream_t st);
-constexpr int kSelLoopKernelsPerIter = 11;
+constexpr int kSelLoopKernelsPerIter = 7;
 
 }  // namespace mapk
