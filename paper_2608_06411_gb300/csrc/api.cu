@@ -439,6 +439,8 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, const int32_t*
     d.M = S; d.N = R; d.K = g.D; d.batch = B; d.n_limit = s.nlimit;
     d.C = s.G; d.ldc = R; d.c_batch_stride = static_cast<long long>(S) * R;
     d.epi = mapk::EPI_F32; d.status = c->status;
+    d.sym = 1;                                   // A x A tiles load their rows once
+    d.n_outer = 1;                               // the basis columns are often skipped
     d.blist = s.blist;                           // images still selecting (built by choose)
     // the GEMM after a list producer reads the count that producer appended through
     auto take_list = [&](GemmDesc& g) { g.bcount = s.bcount + s.bc_par; s.bc_par ^= 1; };

@@ -56,6 +56,8 @@ struct KArgs {
   const int* m_limit;
   unsigned long long wait_ns;   // limit of the role waits (the drain waits keep kWaitLimitNs)
   int ksplit; long long c_split_stride;   // EPI_F32 split-K: partial sums per K slice
+  int sym;                                 // B is A: the diagonal tile reads its A stage as B
+  int n_outer;                             // unit order: column tiles outermost
 };
 
 __device__ __forceinline__ float gelu_erf(float x) {
@@ -107,18 +109,32 @@ struct TileCoord { int b, m_blk, n_blk, ks; bool skip; };
 // same N tile, processed by the two CTAs of a cluster (rank 0 the upper, rank 1 the lower).
 // With split-K (ksplit > 1) a unit is also one K slice ks of its tile.
 template <bool PAIR>
-__device__ __forceinline__ TileCoord tile_coord(const KArgs& a, int t, int m_units, int n_tiles, int BN,
+__device__ __forceinline__ TileCoord tile_coord(const KArgs& a, int t, int nbatch, int m_units, int n_tiles, int BN,
                                                 uint32_t crank) {
   TileCoord c;
-  const int tiles = m_units * n_tiles;
-  int per = tiles * a.ksplit;
-  c.b = t / per;
-  int rem = t - c.b * per;
-  c.ks = rem / tiles;
-  rem -= c.ks * tiles;
+  int mu;
+  if (a.n_outer) {
+    // column tiles outermost: the units of one column tile of every batch entry are
+    // consecutive, so that when whole column tiles are skipped (n_limit) the remaining units
+    // still spread over all CTAs
+    const int per_n = nbatch * m_units * a.ksplit;
+    c.n_blk = t / per_n;
+    int rem = t - c.n_blk * per_n;
+    c.b = rem / (m_units * a.ksplit);
+    rem -= c.b * (m_units * a.ksplit);
+    c.ks = rem / m_units;
+    mu = rem - c.ks * m_units;
+  } else {
+    const int tiles = m_units * n_tiles;
+    const int per = tiles * a.ksplit;
+    c.b = t / per;
+    int rem = t - c.b * per;
+    c.ks = rem / tiles;
+    rem -= c.ks * tiles;
+    mu = rem / n_tiles;
+    c.n_blk = rem - mu * n_tiles;
+  }
   if (a.blist) c.b = __ldg(a.blist + c.b);
-  const int mu = rem / n_tiles;
-  c.n_blk = rem - mu * n_tiles;
   c.m_blk = PAIR ? 2 * mu + static_cast<int>(crank) : mu;
   int lim = a.n_limit ? min(a.N, __ldg(a.n_limit + c.b)) : a.N;
   c.skip = c.n_blk * BN >= lim;
@@ -178,7 +194,8 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   const int m_tiles = (a.M + kBM - 1) / kBM;
   const int m_units = PAIR ? (m_tiles + 1) / 2 : m_tiles;
   const int n_tiles = (a.N + BN - 1) / BN;
-  const int total = (a.blist ? min(a.batch, *a.bcount) : a.batch) * m_units * n_tiles * a.ksplit;
+  const int nbatch = a.blist ? min(a.batch, *a.bcount) : a.batch;
+  const int total = nbatch * m_units * n_tiles * a.ksplit;
   const int KB = a.K / kBK;
   // K blocks of a unit's slice (the whole K without split-K)
   auto kb_range = [&](const TileCoord& c, int& kb0, int& kb1) {
@@ -202,6 +219,16 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     }
   };
 
+  // With a.sym, a tile whose B rows (this CTA's half of them with 2-SM pairs) are its A rows
+  // loads them once: the same stage layout serves as both operands (BN / 2 or BN == kBM rows).
+  // Both CTAs of a pair and all roles reach the same answer (the row offsets cancel).
+  auto b_is_a = [&](const TileCoord& c) {
+    if (!a.sym || (CG2 ? BN / 2 : BN) != kBM) return false;
+    const int arow = c.b * a.a_row_stride + c.m_blk * kBM;
+    const int brow = c.b * a.b_row_stride + a.b_base + c.n_blk * BN + (CG2 ? static_cast<int>(crank) * (BN / 2) : 0);
+    return arow == brow;
+  };
+
   // Producer: parity of the last load issued into each stage (-1: none), for the drain below.
   int last_par[STAGES];
 #pragma unroll
@@ -212,17 +239,32 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       uint32_t stage = 0, phase = 0;
       bool ok = true;
       for (int t = unit0; t < total && ok; t += units_step) {
-        TileCoord c = tile_coord<PAIR>(a, t, m_units, n_tiles, BN, crank);
+        TileCoord c = tile_coord<PAIR>(a, t, nbatch, m_units, n_tiles, BN, crank);
         if (c.skip) continue;
         const int arow = c.b * a.a_row_stride + c.m_blk * kBM;
         const int brow = (a.b_off ? __ldg(a.b_off + c.b) : c.b * a.b_row_stride + a.b_base) + c.n_blk * BN;
+        const bool alias = b_is_a(c);
+        const int kstep = alias ? 2 : 1;           // alias: two K blocks per stage (A and B buffers)
         int kb0, kb1;
         kb_range(c, kb0, kb1);
-        for (int kb = kb0; kb < kb1; ++kb) {
+        for (int kb = kb0; kb < kb1; kb += kstep) {
           if (!mbar_wait(&empty[stage], phase ^ 1, a.status, abort_flag, a.wait_ns)) { ok = false; break; }
           int ac, bc;
           kcols(kb, ac, bc);
-          if constexpr (CG2) {
+          if (alias) {
+            // K block kb into the A buffer, kb + 1 (when in range) into the B buffer; no kwrap
+            const int n2 = kb + 1 < kb1 ? 2 : 1;
+            if constexpr (CG2) {
+              if (crank == 0) mbar_arrive_expect_tx(&full[stage], 2 * n2 * S::A_BYTES);
+              const uint32_t fb = mapa_u32(&full[stage], 0);
+              tma_load_2d_cg2(sA + stage * S::A_BYTES, &tmA, fb, ac, arow);
+              if (n2 == 2) tma_load_2d_cg2(sB + stage * S::B_BYTES, &tmA, fb, ac + kBK, arow);
+            } else {
+              mbar_arrive_expect_tx(&full[stage], n2 * S::A_BYTES);
+              tma_load_2d(sA + stage * S::A_BYTES, &tmA, &full[stage], ac, arow);
+              if (n2 == 2) tma_load_2d(sB + stage * S::B_BYTES, &tmA, &full[stage], ac + kBK, arow);
+            }
+          } else if constexpr (CG2) {
             // both CTAs' copies complete on the leader's full barrier, which expects them all
             if (crank == 0) mbar_arrive_expect_tx(&full[stage], 2 * S::STAGE_BYTES);
             const uint32_t fb = mapa_u32(&full[stage], 0);
@@ -245,19 +287,36 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       uint32_t stage = 0, phase = 0, acc = 0, acc_phase = 0;
       bool issued = false, ok = true;
       for (int t = unit0; t < total && ok; t += units_step) {
-        TileCoord c = tile_coord<PAIR>(a, t, m_units, n_tiles, BN, crank);
+        TileCoord c = tile_coord<PAIR>(a, t, nbatch, m_units, n_tiles, BN, crank);
         if (c.skip) continue;
         if (!mbar_wait(&tempty[acc], acc_phase ^ 1, a.status, abort_flag, a.wait_ns)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + acc * BN;
+        const bool alias = b_is_a(c);
+        const int kstep = alias ? 2 : 1;
         int kb0, kb1;
         kb_range(c, kb0, kb1);
-        for (int kb = kb0; kb < kb1; ++kb) {
+        for (int kb = kb0; kb < kb1; kb += kstep) {
           if (!mbar_wait(&full[stage], phase, a.status, abort_flag, a.wait_ns)) { ok = false; break; }
           tc_fence_after();
           const uint32_t a0 = smem_u32(sA + stage * S::A_BYTES);
-          const uint32_t b0 = smem_u32(sB + stage * S::B_BYTES);
-          if constexpr (CG2) {
+          const uint32_t b0 = alias ? a0 : smem_u32(sB + stage * S::B_BYTES);
+          if (alias) {
+            // each buffer is both operands of its K block (the tile's B rows are its A rows)
+            const uint32_t a1 = smem_u32(sB + stage * S::B_BYTES);
+            const int n2 = kb + 1 < kb1 ? 2 : 1;
+            for (int h = 0; h < n2; ++h) {
+              const uint32_t x = h == 0 ? a0 : a1;
+#pragma unroll
+              for (int k = 0; k < kBK / 16; ++k) {
+                const uint32_t acc_on = (kb != kb0 || h != 0 || k != 0);
+                if constexpr (CG2) umma_bf16_cg2(d_tmem, desc_sw128(x + k * 32), desc_sw128(x + k * 32), IDESC, acc_on);
+                else umma_bf16(d_tmem, desc_sw128(x + k * 32), desc_sw128(x + k * 32), IDESC, acc_on);
+              }
+            }
+            if constexpr (CG2) umma_commit_cg2_mc(&empty[stage], static_cast<uint16_t>(3));
+            else umma_commit(&empty[stage]);
+          } else if constexpr (CG2) {
 #pragma unroll
             for (int k = 0; k < kBK / 16; ++k)
               umma_bf16_cg2(d_tmem, desc_sw128(a0 + k * 32), desc_sw128(b0 + k * 32), IDESC, (kb != kb0 || k != 0));
@@ -300,7 +359,7 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     uint32_t eg_phase = 0;
     bool eg_ok = true;
     for (int t = unit0; t < total && eg_ok; t += units_step) {
-      TileCoord c = tile_coord<PAIR>(a, t, m_units, n_tiles, BN, crank);
+      TileCoord c = tile_coord<PAIR>(a, t, nbatch, m_units, n_tiles, BN, crank);
       if (c.skip) continue;
       if constexpr (S::PROJ) {
         if (c.b != staged_b) {                     // stage L and 1/r of this image's R0 basis
@@ -899,6 +958,11 @@ cudaError_t launch_gemm(const GemmDesc& d, int num_sms, cudaStream_t st) {
     return cudaErrorInvalidValue;
   ka.ksplit = d.ksplit; ka.c_split_stride = d.c_split_stride;
   if (d.blist && !d.bcount) return cudaErrorInvalidValue;
+  if (d.sym && (d.A != d.B || d.a_row_stride != d.b_row_stride || d.a_rows_total != d.b_rows_total || d.b_off ||
+                d.a_kwrap || d.b_kwrap || d.split3))
+    return cudaErrorInvalidValue;
+  ka.sym = d.sym;
+  ka.n_outer = d.n_outer;
   switch (d.epi) {
     case EPI_GELU_BF16:
       if (d.N % 256 == 0) return run<256, 4, EPI_GELU_BF16>(d, ka, num_sms, st);

@@ -81,6 +81,13 @@ struct GemmDesc {
   // Limit (ns) of the producer / MMA / epilogue waits; 0 = the default 2 s.  The waits that
   // let in-flight copies and MMAs land before an aborting CTA exits keep the default.
   long long wait_ns = 0;
+  // A and B are the same matrix (same pointer, rows and strides, no K wrap): a tile whose B
+  // rows are its A rows (the diagonal tile of a Gram block) loads them once and the MMA reads
+  // the A stage as B
+  int sym = 0;
+  // Units ordered column tile first (then batch entry, K slice, row tile): with n_limit
+  // skipping whole column tiles of some entries, the other units stay spread over all CTAs
+  int n_outer = 0;
   // EPI_F32 split-K: ksplit K slices, each unit one slice of a tile, slice s writing its partial
   // sum at C + s * c_split_stride (elements, a multiple of 4); the caller adds the slices
   int ksplit = 1; long long c_split_stride = 0;

@@ -172,6 +172,8 @@ extern "C" int map_select_noalloc(map_ctx* ctx, const float* scores, const void*
     d.M = S; d.N = R; d.K = g.D; d.batch = B; d.n_limit = s.nlimit;
     d.C = s.G; d.ldc = R; d.c_batch_stride = static_cast<long long>(S) * R;
     d.epi = mapk::EPI_F32; d.status = v.status;
+    d.sym = 1;                                   // A x A tiles load their rows once
+    d.n_outer = 1;                               // the basis columns are often skipped
     const long long cap = 8LL * (K + N / S) + 64;
     long long rounds = 0;
     int burst = (K0 + mapk::kRoundPicks - 1) / mapk::kRoundPicks + 6;
