@@ -114,7 +114,7 @@ int map_score(map_ctx *ctx, const void *text_feats, const void *vis_feats,
  *               were retained (R0 in p_hat order first).
  * k == N keeps every token (keep_idx = pick_order = 0..N-1); k == 0 is a no-op;
  * k > N is MAP_EINVAL.  Supported: N <= 16384; k <= 4096 for plain top-k (lambda = 0 or
- * K0 = k), k <= 1024 with the diversity term (MAP_EUNSUPPORTED beyond).
+ * K0 = k), k <= 768 with the diversity term (MAP_EUNSUPPORTED beyond).
  * Asynchronous like the other calls: after its first rounds the selection runs as a
  * device-side loop (a CUDA graph whose WHILE node repeats a round while an image still
  * selects; built on the first call of a shape and workspace, then cached in the context), so

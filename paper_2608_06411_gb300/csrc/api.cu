@@ -17,7 +17,8 @@ using mapk::GemmDesc;
 
 namespace {
 
-constexpr int kMaxKDiverse = 1024;  // k limit when the diversity term is on (shared-memory staging)
+constexpr int kMaxKDiverse = 768;   // k limit when the diversity term is on (the coordinate update
+                                    // stages 32 slot rows and 32 basis rows of k floats in shared memory)
 constexpr int kProjMaxBasis = 128;  // basis vectors one projection pass takes
 constexpr int kMaxK = 4096;
 constexpr int kMaxN = 16384;

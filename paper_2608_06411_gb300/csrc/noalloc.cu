@@ -50,7 +50,7 @@ constexpr int kSelS = mapk::kActiveSlots;
 constexpr int kMaxDevices = 64;
 constexpr int kMaxN = 16384;
 constexpr int kMaxK = 4096;          // plain top-k
-constexpr int kMaxKDiverse = 1024;   // with the diversity term
+constexpr int kMaxKDiverse = 768;    // with the diversity term (as map_select)
 
 static __device__ __align__(256) unsigned char g_scratch[kNoAllocScratchBytes];
 

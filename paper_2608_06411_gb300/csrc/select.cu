@@ -328,105 +328,152 @@ __host__ __device__ inline int coord_pitch(int KP) { return ((KP + 7) / 8) * 8 +
 // Brings every active token's coordinates up to the current basis (nb vectors) by forward
 // substitution before the picks:
 //   e_beta[i] = (G[j_beta, i] - sum_{beta' < beta} e_beta'[j_beta] e_beta'[i]) / r_beta,
-// 32 basis vectors at a time.  A CTA serves 32 slots (lane = slot) with kUpdWarps warps: the
-// 32 rows of L (the basis tokens' own coordinate rows) are staged in shared memory, each warp
-// forms the products with the known coordinates for its share of the 32 rows, and warp 0
-// then solves the 32 x 32 triangle.  An image's slots spread over S / 32 CTAs.  Writes Ec,
-// r2 and cstep = nb.
+// 32 basis vectors (a chunk) at a time.  A CTA serves 32 slots, their coordinate rows in
+// shared memory.  For a chunk starting at b0 the products with the coordinates before it,
+// P[slot][row] = sum_{q < b0} e_q[slot] L[row][q] (L rows: the chunk's basis tokens' own
+// coordinate rows), form a 32 x 32 x b0 matrix product: each warp takes every fourth
+// 16-column block with 4 slots x 8 rows per thread (every loaded value feeds 4 or 8 FMAs).
+// Warp 0 then adds the four partial products and solves the chunk's 32 x 32 triangle
+// right-looking (lane = slot: each new coordinate is subtracted from the later ones at once,
+// so a step waits for one FMA), while warps 1-3 copy the next chunk's L rows, triangle,
+// Gram entries and basis norms into shared memory (cp.async), so that no chunk waits for a
+// global load.  An image's slots spread over S / 32 CTAs.  Writes Ec, r2 and cstep = nb.
 constexpr int kUpdWarps = 4;
-constexpr int kUpdRows = kChunk / kUpdWarps;
 
 __global__ void __launch_bounds__(kUpdSlots * kUpdWarps, 1) sel_update_kernel(SelState s) {
   pdl_enter();
-  extern __shared__ __align__(16) float shu[];
-  __shared__ float rinv_c[kChunk];
-  __shared__ float accs[kChunk][kUpdSlots];
+  extern __shared__ __align__(16) float shu[];           // [32][P] slot rows, then [32][KP] L rows
+  __shared__ float Lt[2][kChunk][kChunk + 1];            // a chunk's triangle L[i][b0 + q], q < i
+  __shared__ float gsm[2][kUpdSlots][kChunk + 1];        // its Gram entries G[slot][b0 + i]
+  __shared__ float rn[2][kChunk];                        // its basis norms
+  __shared__ float part[kUpdWarps][kUpdSlots][kChunk + 1];
+  __shared__ int tok_s[kUpdSlots], c0_s[kUpdSlots];
   const int b = blockIdx.y;
   if (s.done[b]) return;
   const int S = s.S, R = s.R, KP = s.KP, P = coord_pitch(KP);
+  float* Lb = shu + kUpdSlots * P;
   const int nb = s.nbasis[b], gbase = s.gbase[b];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int slot = blockIdx.x * kUpdSlots + lane;
   const long long base = static_cast<long long>(b) * s.N;
-  const int tok = slot < S ? s.aslot[static_cast<long long>(b) * S + slot] : -1;
-  const int c0 = tok >= 0 ? min(s.cstep[base + tok], nb) : nb;
-  if (!__syncthreads_or(c0 < nb)) return;
-  float* Lc = shu;                                   // [kChunk][KP]
-  float* me = shu + kChunk * KP + lane * P;          // this slot's row
-  if (tok >= 0 && warp == 0) {
-    const float* g = s.Ec + (base + tok) * KP;
-    for (int q = 0; q < c0; q += 4) cp_async16(me + q, g + q);
+  if (threadIdx.x < kUpdSlots) {
+    const int slot = blockIdx.x * kUpdSlots + threadIdx.x;
+    const int tok = slot < S ? s.aslot[static_cast<long long>(b) * S + slot] : -1;
+    tok_s[threadIdx.x] = tok;
+    c0_s[threadIdx.x] = tok >= 0 ? min(s.cstep[base + tok], nb) : nb;
   }
-  const int32_t* btok = s.basis_tok + static_cast<long long>(b) * s.K;
+  __syncthreads();
+  int cmin = nb;                                     // fewest cached coordinates over the slots
+  for (int i = 0; i < kUpdSlots; ++i) cmin = min(cmin, c0_s[i]);
+  if (cmin >= nb) return;                            // uniform
+  const int32_t* btok_g = s.basis_tok + static_cast<long long>(b) * s.K;
   const float* rnorm = s.rnorm + static_cast<long long>(b) * s.K;
-  const float* Gr = s.G + (static_cast<long long>(b) * S + (tok >= 0 ? slot : 0)) * R;
-  float r2 = tok >= 0 ? s.r2[base + tok] : 0.f;
-  for (int b0 = 0; b0 < nb; b0 += kChunk) {
-    const int b1 = min(nb, b0 + kChunk);
-    if (!__syncthreads_or(tok >= 0 && b1 > c0)) continue;   // uniform; also fences the last chunk
-    {
-      // row i of L: basis token j_{b0+i}'s coordinates 0 .. b0+i-1 (all that is read of it)
-      const int bt = lane < b1 - b0 ? btok[b0 + lane] : 0;
-      for (int i = warp; i < b1 - b0; i += kUpdWarps) {
-        const int ti = __shfl_sync(0xffffffffu, bt, i);
-        const float* src = s.Ec + (base + ti) * KP;
-        for (int q = 4 * lane; q < b0 + i; q += 128) cp_async16(Lc + i * KP + q, src + q);
-      }
-      cp_async_wait_all();
+  const float* Gb = s.G + (static_cast<long long>(b) * S + blockIdx.x * kUpdSlots) * R;
+  // everything chunk c needs, copied by threads t0, t0 + stride, ... (one commit group)
+  auto stage = [&](int c, int buf, int t0, int stride) {
+    const int nch = min(nb, c + kChunk) - c, v4 = c / 4;
+    for (int e = t0; e < nch * v4; e += stride) {    // L rows, columns [0, c)
+      const int row = e / v4, q = (e - row * v4) * 4;
+      cp_async16(Lb + row * KP + q, s.Ec + (base + __ldg(btok_g + c + row)) * KP + q);
     }
-    if (threadIdx.x < b1 - b0) rinv_c[threadIdx.x] = 1.0f / rnorm[b0 + threadIdx.x];
-    __syncthreads();
-    const bool work = tok >= 0 && b1 > c0;
-    if (work) {
-      // this warp's rows: G entries minus the products with coordinates 0 .. b0-1
-      const int i0 = warp * kUpdRows;
-      float acc[kUpdRows];
-#pragma unroll
-      for (int r = 0; r < kUpdRows; ++r) {
-        const int beta = b0 + i0 + r;
-        acc[r] = (beta < b1 && beta >= c0) ? Gr[S + beta - gbase] : 0.f;
-      }
-#pragma unroll 2
-      for (int q = 0; q < b0; q += 4) {
-        const float4 eq = *reinterpret_cast<const float4*>(me + q);
-#pragma unroll
-        for (int r = 0; r < kUpdRows; ++r) {
-          const float4 l = *reinterpret_cast<const float4*>(Lc + (i0 + r) * KP + q);
-          acc[r] = fmaf(-l.x, eq.x, acc[r]);
-          acc[r] = fmaf(-l.y, eq.y, acc[r]);
-          acc[r] = fmaf(-l.z, eq.z, acc[r]);
-          acc[r] = fmaf(-l.w, eq.w, acc[r]);
-        }
-      }
-#pragma unroll
-      for (int r = 0; r < kUpdRows; ++r) accs[i0 + r][lane] = acc[r];
+    for (int e = t0; e < nch * kChunk; e += stride) {   // the triangle: row i, columns c .. c + i - 1
+      const int i = e / kChunk, q = e - i * kChunk;
+      if (q < i) cp_async4(&Lt[buf][i][q], s.Ec + (base + __ldg(btok_g + c + i)) * KP + c + q);
     }
+    for (int e = t0; e < kUpdSlots * nch; e += stride) {   // Gram entries of the slots that need them
+      const int sl = e / nch, i = e - sl * nch;
+      if (tok_s[sl] >= 0 && c + i >= c0_s[sl]) cp_async4(&gsm[buf][sl][i], Gb + static_cast<long long>(sl) * R + S + c + i - gbase);
+    }
+    for (int e = t0; e < nch; e += stride) cp_async4(&rn[buf][e], rnorm + c + e);
+    cp_async_commit();
+  };
+  for (int r = warp; r < kUpdSlots; r += kUpdWarps) {   // cached coordinates [0, c0) of every slot
+    const int tok = tok_s[r], c0 = c0_s[r];
+    if (tok < 0) continue;
+    const float* g = s.Ec + (base + tok) * KP;
+    float* me = shu + r * P;
+    for (int q = 4 * lane; q < c0; q += 128) cp_async16(me + q, g + q);
+  }
+  const int first = (cmin / kChunk) * kChunk;
+  stage(first, 0, threadIdx.x, blockDim.x);
+  const int mtok = tok_s[lane], mc0 = c0_s[lane];    // warp 0: this lane's slot
+  float r2 = warp == 0 && mtok >= 0 ? s.r2[base + mtok] : 0.f;
+  const int sg = lane >> 2, rg = lane & 3;           // products: slots 4 sg + 0..3, rows rg + 4 j
+  int buf = 0;
+  for (int b0 = first; b0 < nb; b0 += kChunk, buf ^= 1) {
+    const int nch = min(nb, b0 + kChunk) - b0;
+    cp_async_wait_all();                             // this chunk's copies (and the slot rows)
     __syncthreads();
-    if (work && warp == 0) {
-      float e[kChunk];
+    float acc[4][8];
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+#pragma unroll
+      for (int j = 0; j < 8; ++j) acc[u][j] = 0.f;
+    for (int qa = 16 * warp; qa < b0; qa += 16 * kUpdWarps) {   // whole 16-column blocks (b0 % 32 == 0)
+#pragma unroll
+      for (int q4 = 0; q4 < 16; q4 += 4) {
+        float4 m[4], l[8];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) m[u] = *reinterpret_cast<const float4*>(shu + (4 * sg + u) * P + qa + q4);
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+          l[j] = rg + 4 * j < nch ? *reinterpret_cast<const float4*>(Lb + (rg + 4 * j) * KP + qa + q4)
+                                  : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            float t = acc[u][j];
+            t = fmaf(m[u].x, l[j].x, t);
+            t = fmaf(m[u].y, l[j].y, t);
+            t = fmaf(m[u].z, l[j].z, t);
+            acc[u][j] = fmaf(m[u].w, l[j].w, t);
+          }
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+#pragma unroll
+      for (int j = 0; j < 8; ++j) part[warp][4 * sg + u][rg + 4 * j] = acc[u][j];
+    __syncthreads();                                 // products done: Lb is free
+    if (warp != 0) {
+      if (b0 + kChunk < nb) stage(b0 + kChunk, buf ^ 1, threadIdx.x - 32, blockDim.x - 32);
+    } else if (mtok >= 0) {
+      float* me = shu + lane * P;
+      float av[kChunk];
+#pragma unroll
+      for (int i = 0; i < kChunk; ++i)
+        av[i] = (i < nch && b0 + i >= mc0)
+                    ? gsm[buf][lane][i] - ((part[0][lane][i] + part[1][lane][i]) + (part[2][lane][i] + part[3][lane][i]))
+                    : 0.f;
 #pragma unroll
       for (int i = 0; i < kChunk; ++i) {
-        const int beta = b0 + i;
-        if (beta < b1) {
-          if (beta >= c0) {
-            float a = accs[i][lane];
-#pragma unroll
-            for (int q = 0; q < i; ++q) a = fmaf(-Lc[i * KP + b0 + q], e[q], a);
-            e[i] = a * rinv_c[i];
-            me[beta] = e[i];
-            r2 = fmaf(-e[i], e[i], r2);
+        if (i < nch) {
+          const int beta = b0 + i;
+          float ei;
+          if (beta >= mc0) {
+            ei = av[i] / rn[buf][i];
+            me[beta] = ei;
+            r2 = fmaf(-ei, ei, r2);
           } else {
-            e[i] = me[beta];
+            ei = me[beta];
           }
+#pragma unroll
+          for (int j = i + 1; j < kChunk; ++j) av[j] = fmaf(-Lt[buf][j][i], ei, av[j]);
         }
       }
     }
+    __syncthreads();                                 // this chunk's coordinates are written
   }
-  if (warp == 0 && tok >= 0 && c0 < nb) {
+  if (warp == 0 && mtok >= 0 && mc0 < nb) {
+    s.r2[base + mtok] = r2;
+    s.cstep[base + mtok] = nb;
+  }
+  for (int r = warp; r < kUpdSlots; r += kUpdWarps) {   // new coordinates [c0, nb), a warp per row
+    const int tok = tok_s[r], c0 = c0_s[r];
+    if (tok < 0 || c0 >= nb) continue;
     float* g = s.Ec + (base + tok) * KP;
-    for (int q = c0; q < nb; ++q) g[q] = me[q];
-    s.r2[base + tok] = r2;
-    s.cstep[base + tok] = nb;
+    const float* me = shu + r * P;
+    for (int q = c0 + lane; q < nb; q += 32) g[q] = me[q];
   }
 }
 
@@ -944,7 +991,7 @@ size_t sel_chol_smem(int K0) {
   return (static_cast<size_t>(K0) * ((K0 + 3) & ~3) + static_cast<size_t>(K0) * coord_pitch(K0)) * 4;
 }
 size_t sel_update_smem(int KP) {
-  return (static_cast<size_t>(kChunk) * KP + static_cast<size_t>(kUpdSlots) * coord_pitch(KP)) * 4;
+  return (static_cast<size_t>(kUpdSlots) * coord_pitch(KP) + static_cast<size_t>(kChunk) * KP) * 4;
 }
 
 cudaError_t launch_sel_init(const SelState& s, cudaStream_t st) {

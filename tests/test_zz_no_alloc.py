@@ -90,7 +90,7 @@ def test_noalloc_select_rejects_oversized_workspace():
     with pytest.raises(mb.MapError) as e:
         ctx.select_noalloc(p, vis, wl.K, keep)
     assert e.value.code == mb.MAP_EUNSUPPORTED
-    with pytest.raises(mb.MapError) as e:    # diversity term on: k <= 1024, as for map_select
-        ctx.select_noalloc(p[:1], vis[:1], 1100, torch.empty((1, 1100), dtype=torch.int32, device=DEV))
+    with pytest.raises(mb.MapError) as e:    # diversity term on: k <= 768, as for map_select
+        ctx.select_noalloc(p[:1], vis[:1], 800, torch.empty((1, 800), dtype=torch.int32, device=DEV))
     assert e.value.code == mb.MAP_EUNSUPPORTED
     ctx.close()
