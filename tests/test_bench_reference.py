@@ -20,6 +20,11 @@ def test_reference_arm_prints_one_contract_line():
                 "scaling", "vs_baseline", "dtype", "data", "config", "cpu_baseline", "e2e"):
         assert key in d, key
     assert d["config"]["workload"] == "c3_batch64_n2880_k160"
+    # the same config object as the GPU arm's line, so the two lines describe one workload
+    sys.path.insert(0, ROOT)
+    import bench
+    from paper_2608_06411_gb300 import workloads as W
+    assert d["config"] == bench.workload_config(W.make_lens(bench.WORKLOAD), 1)
     assert d["value"] > 0 and d["unit"] == "images/s" and d["higher_is_better"] is True
     assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["cores"] >= 1
     assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["e2e"]["d2h_bytes_per_step"] == 0
