@@ -214,10 +214,22 @@ __global__ void __launch_bounds__(1024) sel_init_kernel(SelState s) {
     const int cap = pow2_at_least(s.K0);
     for (int i = threadIdx.x; i < s.N; i += blockDim.x)
       if (sh64[i] >= T) sel[atomicAdd(&cnt, 1)] = sh64[i];
-    for (int i = s.K0 + threadIdx.x; i < cap; i += blockDim.x) sel[i] = 0ull;
-    __syncthreads();
-    block_sort_desc(sel, cap);
-    for (int i = threadIdx.x; i < s.K0; i += blockDim.x) s.r0[static_cast<long long>(b) * s.K + i] = key_index(sel[i]);
+    if (s.K0 <= static_cast<int>(blockDim.x)) {
+      // The keys are distinct (each holds its token index), so a key's place in descending
+      // order is the number of larger keys: one pass, no sorting network.
+      __syncthreads();
+      if (static_cast<int>(threadIdx.x) < s.K0) {
+        const uint64_t x = sel[threadIdx.x];
+        int rank = 0;
+        for (int j = 0; j < s.K0; ++j) rank += sel[j] > x ? 1 : 0;
+        s.r0[static_cast<long long>(b) * s.K + rank] = key_index(x);
+      }
+    } else {
+      for (int i = s.K0 + threadIdx.x; i < cap; i += blockDim.x) sel[i] = 0ull;
+      __syncthreads();
+      block_sort_desc(sel, cap);
+      for (int i = threadIdx.x; i < s.K0; i += blockDim.x) s.r0[static_cast<long long>(b) * s.K + i] = key_index(sel[i]);
+    }
   }
 }
 
@@ -931,6 +943,20 @@ __global__ void sel_finalize_kernel(const int32_t* picks, int K, int32_t* keep, 
     if (order) order[static_cast<long long>(b) * K + i] = p[i];
   }
   __syncthreads();
+  if (K <= static_cast<int>(blockDim.x)) {
+    // place = number of smaller picks (equal ones, which a valid selection never has, by position)
+    const int i = threadIdx.x;
+    if (i < K) {
+      const int32_t x = sh32[i];
+      int rank = 0;
+      for (int j = 0; j < K; ++j) {
+        const int32_t y = sh32[j];
+        rank += (y < x || (y == x && j < i)) ? 1 : 0;
+      }
+      keep[static_cast<long long>(b) * K + rank] = x;
+    }
+    return;
+  }
   block_sort_asc_i32(sh32, K, pow2_at_least(K));
   for (int i = threadIdx.x; i < K; i += blockDim.x) keep[static_cast<long long>(b) * K + i] = sh32[i];
 }
