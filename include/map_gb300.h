@@ -157,24 +157,26 @@ int map_assemble(map_ctx *ctx, const void *vis_feats, const int32_t *keep_idx,
 
 /*
  * map_select without allocating memory in the call (the paper has no counterpart; this
- * is a deployment variant of map_select).  Same arguments, results and limits as
- * map_select, but every scratch buffer is carved from one static device array of
- * MAP_NOALLOC_SCRATCH_BYTES held by each GPU that loads the library until the process
- * exits.  It is for callers that cannot allocate device memory while they prune: code
- * that runs inside another framework's caching pool or under a fixed device-memory
- * budget, where a cudaMalloc would take memory the budget does not have or fail, and
- * serving paths that must not stall on the allocator (cudaMalloc and cudaFree may
- * synchronise the device).  The call makes no cudaMalloc / cudaFree and allocates through
- * no library.
+ * is a deployment variant of map_select).  Same arguments and limits as map_select, and
+ * the same exact greedy picks (a near-tie below fp32 resolution may go either way, as
+ * between any two fp32 evaluations), but every scratch buffer is carved from one static
+ * device array of MAP_NOALLOC_SCRATCH_BYTES, held by each GPU that loads the library
+ * until the process exits.  It is for callers that cannot allocate device memory while
+ * they prune: code that runs inside another framework's caching pool or under a fixed
+ * device-memory budget, where a cudaMalloc would take memory the budget does not have or
+ * fail, and serving paths that must not stall on the allocator (cudaMalloc and cudaFree
+ * may synchronise the device).  The call makes no cudaMalloc / cudaFree and allocates
+ * through no library.
  * Workspace needed, in bytes (each array rounded up to 256): 17 B*N + 16 B*k + 4 B*256
  * + 8 B + small per-image counters, plus, when the diversity term is on (lambda > 0 and
  * K0 < k), 4 B*N*ceil4(k) + 2 B*R*D + 4 B*256*R with R = ceil16(256 + k).  A request
  * that does not fit returns MAP_EUNSUPPORTED and does nothing.  One LLaVA-NeXT image
  * (N = 2880, k = 160, D = 4096) needs about 6 MB.
- * Like map_select it waits for the selection rounds on the host (it synchronises
- * `stream`), and a device-side error is also recorded for map_status.  It skips
- * map_select's tensor-core projection pass (every candidate starts from its bound
- * p_hat * ||v||^lambda), so it runs more selection rounds for the same picks.
+ * Unlike map_select, whose later rounds run as a device-side loop, it waits on the host
+ * for bursts of selection rounds (it synchronises `stream`); a device-side error is
+ * returned and also recorded for map_status.  It skips map_select's tensor-core
+ * projection pass (every candidate starts from its bound p_hat * ||v||^lambda), so it
+ * runs more selection rounds for the same picks.
  * The first call on a device looks the array's address up (device must be current);
  * make that call before any stream capture.  All calls share the array and it keeps the
  * last call's contents; calls whose GPU work overlaps (other streams, other threads)
