@@ -17,6 +17,7 @@ from oracle import qcts_oracle as Q
 import test_distill_pins
 import test_golden
 import test_oracle_pins
+import test_parity_rule_pins
 import test_qcts_pins
 
 
@@ -45,7 +46,8 @@ def _some_pin_fails(*modules) -> bool:
 
 
 def test_pins_pass_unmodified():
-    assert not _some_pin_fails(test_oracle_pins, test_golden, test_qcts_pins, test_distill_pins)
+    assert not _some_pin_fails(test_oracle_pins, test_golden, test_qcts_pins, test_distill_pins,
+                               test_parity_rule_pins)
 
 
 # ------------------------------------------------------------------ scoring and selection oracle
@@ -292,3 +294,55 @@ def _mlp_backward_mean_bias(dh2, x, z1, h1, w2):
 def test_distillation_mistakes_are_caught(monkeypatch, attr, bad):
     monkeypatch.setattr(DO, attr, bad)
     assert _some_pin_fails(test_distill_pins)
+
+
+# ------------------------------------------------------------------ parity rules and batch helpers
+
+def _teacher_rule_accepts_anything(js_oracle, layer_gpu, margin=P.QCTS_LAYER_MARGIN):
+    return True, ""
+
+
+def _teacher_rule_argmax_only(js_oracle, layer_gpu, margin=P.QCTS_LAYER_MARGIN):
+    ok = layer_gpu == int(np.argmax(np.asarray(js_oracle)))
+    return ok, ""
+
+
+def _score_err_absolute(p_gpu, p_ref):
+    return float(np.abs(np.asarray(p_gpu, dtype=np.float64) - p_ref).max())
+
+
+def _grad_err_without_scale(g_gpu, g_ref, scale=0.0):
+    g_ref = np.asarray(g_ref, dtype=np.float64)
+    return float(np.abs(np.asarray(g_gpu, dtype=np.float64) - g_ref).max() / max(float(np.abs(g_ref).max()), 1e-300))
+
+
+def _unpack_reversed(attn_bits, lens, L, H, N):
+    out, o = [], 0
+    for M in (int(x) for x in reversed(list(lens))):
+        n = L * H * M * N
+        out.append(attn_bits[o:o + n].reshape(L, H, M, N))
+        o += n
+    return out[::-1]
+
+
+_orig_distill_batch = DO.distill_batch
+
+
+def _distill_batch_first_question_only(text_bits, vis_bits, lens, teachers, weights_bits, rope_base=10000.0,
+                                       rope_on=True):
+    m0 = int(lens[0])
+    text = np.concatenate([text_bits[:m0]] * len(lens))
+    return _orig_distill_batch(text, vis_bits, [m0] * len(lens), teachers, weights_bits, rope_base, rope_on)
+
+
+@pytest.mark.parametrize("target,attr,bad", [
+    (P, "check_teacher_layer", _teacher_rule_accepts_anything),
+    (P, "check_teacher_layer", _teacher_rule_argmax_only),
+    (P, "score_rel_err", _score_err_absolute),
+    (P, "distill_grad_err", _grad_err_without_scale),
+    (Q, "unpack_attention", _unpack_reversed),
+    (DO, "distill_batch", _distill_batch_first_question_only),
+])
+def test_parity_rule_and_batch_helper_mistakes_are_caught(monkeypatch, target, attr, bad):
+    monkeypatch.setattr(target, attr, bad)
+    assert _some_pin_fails(test_parity_rule_pins)
