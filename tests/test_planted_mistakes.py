@@ -346,3 +346,47 @@ def _distill_batch_first_question_only(text_bits, vis_bits, lens, teachers, weig
 def test_parity_rule_and_batch_helper_mistakes_are_caught(monkeypatch, target, attr, bad):
     monkeypatch.setattr(target, attr, bad)
     assert _some_pin_fails(test_parity_rule_pins)
+
+
+# ------------------------------------------------------------------ hand-off and compaction oracles
+
+_orig_assemble = O.assemble
+
+
+def _assemble_questions_at_m(vis_bits, keep, text_bits, lens, pos_offset=0, n_valid=None):
+    seq, pos = _orig_assemble(vis_bits, keep, text_bits, lens, pos_offset, n_valid)
+    N = vis_bits.shape[1]
+    pos = pos.copy()
+    k = np.asarray(keep).shape[1]
+    o = 0
+    for b in range(vis_bits.shape[0]):
+        M = int(lens[b])
+        Nb = N if n_valid is None else int(n_valid[b])
+        pos[o + k:o + k + M] -= Nb                     # question token m at position m
+        o += k + M
+    return seq, pos
+
+
+def _assemble_offset_on_kept_only(vis_bits, keep, text_bits, lens, pos_offset=0, n_valid=None):
+    seq, pos = _orig_assemble(vis_bits, keep, text_bits, lens, 0, n_valid)
+    pos = pos.copy()
+    k = np.asarray(keep).shape[1]
+    o = 0
+    for b in range(vis_bits.shape[0]):
+        pos[o:o + k] += pos_offset
+        o += k + int(lens[b])
+    return seq, pos
+
+
+def _gather_from_first_image(vis_bits, keep):
+    return np.stack([vis_bits[0][np.asarray(keep[b], dtype=np.int64)] for b in range(vis_bits.shape[0])])
+
+
+@pytest.mark.parametrize("attr,bad", [
+    ("assemble", _assemble_questions_at_m),
+    ("assemble", _assemble_offset_on_kept_only),
+    ("gather", _gather_from_first_image),
+])
+def test_handoff_and_gather_mistakes_are_caught(monkeypatch, attr, bad):
+    monkeypatch.setattr(O, attr, bad)
+    assert _some_pin_fails(test_oracle_pins)
