@@ -212,7 +212,7 @@ class AttentionWorkload:
     grid: int
     m_lo: int       # question length range (inclusive)
     m_hi: int
-    m_ref: int      # tokens of the reference question ("What is shown in this image?")
+    m_ref: int      # tokens of the generic reference question (what the image shows)
 
     @property
     def N(self) -> int:
