@@ -119,7 +119,8 @@ int map_score(map_ctx *ctx, const void *text_feats, const void *vis_feats,
  * device-side loop (a CUDA graph whose WHILE node repeats a round while an image still
  * selects; built on the first call of a shape and workspace, then cached in the context), so
  * the host never waits for it.  A device-side failure (a bounded wait that ran out, or the
- * loop's iteration cap, which no input reaches) is reported by map_status.
+ * loop's iteration cap, set at the most rounds the selection can take:
+ * k * (ceil(N / 256) + 1) + ceil(k / 128) + 64) is reported by map_status.
  */
 int map_select(map_ctx *ctx, const float *scores, const void *vis_feats, int B, int N,
                int k, int32_t *keep_idx, int32_t *pick_order, void *stream);

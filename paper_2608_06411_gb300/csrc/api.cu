@@ -445,7 +445,10 @@ int select_impl(map_ctx* c, const float* scores, const void* vis, const int32_t*
     d.blist = s.blist;                           // images still selecting (built by choose)
     // the GEMM after a list producer reads the count that producer appended through
     auto take_list = [&](GemmDesc& g) { g.bcount = s.bcount + s.bc_par; s.bc_par ^= 1; };
-    const long long cap = 8LL * (K + N / S) + 64;   // rounds; far above what any input needs
+    // Rounds: every round picks or makes S stale bounds exact, so at most ceil(N / S) rounds
+    // without a pick come before each pick; one more per kRoundPicks picks of a launch.
+    const long long cap = static_cast<long long>(K) * ((N + S - 1) / S + 1) +
+                          (K + mapk::kRoundPicks - 1) / mapk::kRoundPicks + 64;
     if (project) {
       // R0: gather its rows, G[R0, R0] on the tensor cores, then its Cholesky factor.
       c->counters.launches += 3;

@@ -174,7 +174,10 @@ extern "C" int map_select_noalloc(map_ctx* ctx, const float* scores, const void*
     d.epi = mapk::EPI_F32; d.status = v.status;
     d.sym = 1;                                   // A x A tiles load their rows once
     d.n_outer = 1;                               // the basis columns are often skipped
-    const long long cap = 8LL * (K + N / S) + 64;
+    // every round picks or makes S stale bounds exact: at most ceil(N / S) rounds without a
+    // pick come before each pick
+    const long long cap = static_cast<long long>(K) * ((N + S - 1) / S + 1) +
+                          (K + mapk::kRoundPicks - 1) / mapk::kRoundPicks + 64;
     long long rounds = 0;
     int burst = (K0 + mapk::kRoundPicks - 1) / mapk::kRoundPicks + 6;
     for (;;) {
