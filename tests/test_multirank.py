@@ -100,3 +100,43 @@ def test_two_gloo_ranks_average_distillation_gradients():
         assert lr == pytest.approx(loss, rel=1e-12)
         for k in g:
             np.testing.assert_allclose(gr[k], g[k], rtol=1e-10, atol=1e-14)
+
+
+def _leaving_rank_worker(rank, world, port, out):
+    import datetime
+    import time
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world, timeout=datetime.timedelta(seconds=5))
+    dist.barrier()                              # both ranks are up
+    if rank == 1:
+        out[1] = "left"
+        os._exit(0)                             # leaves between steps, without joining the next collective
+    t0 = time.monotonic()
+    try:
+        max_over_ranks(1.0)
+        out[0] = ("no error", time.monotonic() - t0)
+    except Exception as e:                      # the collective's error is the failure signal
+        out[0] = (type(e).__name__, time.monotonic() - t0)
+    os._exit(0)                                 # the group is broken: skip its teardown
+
+
+def test_a_rank_that_leaves_is_reported_not_waited_for():
+    """A rank that leaves between steps: the other rank's next collective (the max over ranks
+    that the benchmark takes) ends with an error within the process group's timeout."""
+    import time
+    world = 2
+    mgr = mp.get_context("spawn").Manager()
+    out = mgr.dict()
+    ctx = mp.start_processes(_leaving_rank_worker, args=(world, _free_port(), out), nprocs=world,
+                             start_method="spawn", join=False)
+    deadline = time.monotonic() + 120
+    while not ctx.join(timeout=5):
+        if time.monotonic() > deadline:
+            for p in ctx.processes:
+                p.kill()
+            pytest.fail("ranks did not finish")
+    assert out[1] == "left"
+    name, waited = out[0]
+    assert name != "no error"
+    assert waited < 60
